@@ -1,0 +1,435 @@
+#!/usr/bin/env python
+"""Throughput of the fractal KV-cache archive path on one GB300.
+
+Workload: a GPT-2-shaped full KV cache -- 12 layers x 8 sequences x 12 heads x
+1024 positions x 64 dims, fp16, synthetic (seeded Irwin-Hall values with 4
+outlier key channels per head), per-head RVQ codebooks with 4 key stages and 2
+value stages of 256 codewords, alphabet N = 256 at r = r_256, span length 6.
+
+One step is one pass of the whole archive path over that cache:
+  1. exact-window split: positions [4, 992) of every (layer, sequence) leave
+     the 4-sink + 32-recent window and are archived;
+  2. RVQ assignment of their K and V head vectors into token records;
+  3. span encoding of the 96 (sequence, layer) symbol streams (append from empty);
+  4. decode-time append: position 992 leaves the window -> RVQ + tail append;
+  5. full decode of the archive and reconstruction of K/V at [4, 993);
+  6. 4096 random record reads (K and V of all heads of one position).
+value = archived KV positions (sequence x layer x position records) per second
+over the whole step.  Inputs (302 MB) are larger than L2, so no flush is needed.
+
+--impl reference times the float64 CPU oracle on a bounded sample of the same
+workload (the paper ships no GPU implementation; the oracle is the reference).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "archived KV positions/s (RVQ+span encode) and decoded KV GB/s, % of roofline"
+UNIT = "archived KV positions/s"
+N_READS = 4096
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+# FP64 add/mul issue rate measured on this machine's GB300 (1.6 per clock per SM,
+# 504 Gop/s at the clock of that run); the span encoder is bound by it.
+FP64_OPS_PER_CLK_SM = 1.6
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- GPU arm --
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import paper_2607_07144_gb300 as fkv
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    base = synth.CFG1
+    cfg = synth.dataclasses.replace(base, cfg_id=base.cfg_id + 1000 * rank) if rank else base
+    cbk, cbv = synth.codebooks(base, 0), synth.codebooks(base, 1)     # replicated codebooks
+    K = synth.gpu_kv_cache(cfg, 0, device=dev)
+    V = synth.gpu_kv_cache(cfg, 1, device=dev)
+    ctx = fkv.Context(256, codebooks=(cbk, cbv))
+    R = ctx.record_len()
+    ns = cfg.batch * cfg.n_layers
+    t0, t1 = cfg.t0, cfg.t1                      # archived range [4, 992)
+    P = t1 - t0
+    n_rec = P + 1                                # + the appended position 992
+    sym = torch.empty((ns, P * R), dtype=torch.uint8, device=dev)
+    rec = torch.empty((ns, R), dtype=torch.uint8, device=dev)
+    st = fkv.Streams(ctx, ns, capacity=n_rec * R)
+    Kr = torch.zeros_like(K)
+    Vr = torch.zeros_like(V)
+    g = torch.Generator().manual_seed(7 + rank)
+    req = torch.stack([torch.randint(0, ns, (N_READS,), generator=g),
+                       torch.randint(0, n_rec, (N_READS,), generator=g)], dim=1).to(dev)
+    out = torch.empty((N_READS, 2, cfg.n_heads, cfg.dim), dtype=K.dtype, device=dev)
+    stream = torch.cuda.current_stream()
+    names = ["rvq_k", "rvq_v", "span_encode", "append_rvq", "append", "decode_kv", "read_kv"]
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
+
+    def step(record=False):
+        e = iter(ev) if record else None
+        rec_ = (lambda: next(e).record(stream)) if record else (lambda: None)
+        rec_()
+        ctx.rvq_encode(0, K, t0, t1, sym)
+        rec_()
+        ctx.rvq_encode(1, V, t0, t1, sym)
+        rec_()
+        st.reset()
+        st.append(sym)
+        rec_()
+        ctx.rvq_encode(0, K, t1, t1 + 1, rec)
+        ctx.rvq_encode(1, V, t1, t1 + 1, rec)
+        rec_()
+        st.append(rec)
+        rec_()
+        ctx.decode_kv(st.points(), n_rec, Kr, Vr, t0=t0)
+        rec_()
+        ctx.read_kv(st.points(), n_rec, req, out)
+        rec_()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if ctx.sync_status() != 0:
+        raise RuntimeError("device status error during warm-up")
+
+    # per-phase durations (CUDA events on the launching stream), averaged
+    phase = np.zeros(len(names))
+    for _ in range(max(1, min(args.steps, 5))):
+        step(record=True)
+        torch.cuda.synchronize()
+        phase += np.array([ev[i].elapsed_time(ev[i + 1]) for i in range(len(names))])
+    phase /= max(1, min(args.steps, 5))
+
+    # timed region: K steps, barrier + sync on both sides
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    time.sleep(0.3)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(args.steps):
+        step()
+    stop.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    ms = start.elapsed_time(stop) / args.steps
+    clk = clocks.stop()
+    ok = ctx.sync_status() == 0
+
+    # end-to-end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        Kh = K.cpu().pin_memory()
+        Vh = V.cpu().pin_memory()
+        Krh = torch.empty_like(Kh).pin_memory()
+        Vrh = torch.empty_like(Vh).pin_memory()
+        ptsh = torch.empty((ns, ctx.n_spans(n_rec * R), 2), dtype=torch.float64).pin_memory()
+
+        def step_e2e():
+            K.copy_(Kh, non_blocking=True)
+            V.copy_(Vh, non_blocking=True)
+            step()
+            ptsh.copy_(st.points()[:, :ptsh.shape[1]], non_blocking=True)
+            Krh.copy_(Kr, non_blocking=True)
+            Vrh.copy_(Vr, non_blocking=True)
+        for _ in range(2):
+            step_e2e()
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        s2, t2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(args.steps):
+            step_e2e()
+        t2.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = s2.elapsed_time(t2) / args.steps
+        h2d = Kh.numel() * Kh.element_size() * 2
+        d2h = ptsh.numel() * 8 + Krh.numel() * Krh.element_size() * 2
+        e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
+
+    units = ns * n_rec
+    return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
+                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L)
+
+
+def roofline(res, peaks, launches_traffic=None):
+    cfg = res["cfg"]
+    ph = res["phase"]
+    D, H = cfg.dim, cfg.n_heads
+    nvec = cfg.batch * cfg.n_layers * H * res["P"]
+    flops_k = nvec * cfg.stages_k * 2 * D * 256
+    flops_v = nvec * cfg.stages_v * 2 * D * 256
+    rvq_ms = ph["rvq_k"] + ph["rvq_v"]
+    rvq_tf = (flops_k + flops_v) / (rvq_ms * 1e-3) / 1e12
+    symbols = res["ns"] * res["P"] * res["R"]
+    spans = res["ns"] * res["P"] * res["R"] // res["L"]
+    enc_bytes = symbols + spans * 16
+    out_bytes = res["ns"] * res["n_rec"] * 2 * H * D * cfg.elem_bytes
+    dec_bytes = res["ns"] * res["n_rec"] * res["R"] * 1 + res["spans"] * res["ns"] * 16 + out_bytes
+    sm_mhz = res["clocks"].get("sm_mhz") or 1900.0
+    fp64_peak = FP64_OPS_PER_CLK_SM * 152 * sm_mhz * 1e6
+    kernels = {
+        "rvq (tcgen05)": {"bound": "tensor", "achieved_tflops": rvq_tf, "ms": rvq_ms,
+                          "frac": rvq_tf / peaks["bf16_tflops"]},
+        "span_encode": {"bound": "fp64", "ms": ph["span_encode"],
+                        "achieved_gbs": enc_bytes / (ph["span_encode"] * 1e-3) / 1e9,
+                        "frac_hbm": enc_bytes / (ph["span_encode"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                        "frac_fp64": symbols * 6 / (ph["span_encode"] * 1e-3) / fp64_peak},
+        "decode_kv (decode + gather)": {"bound": "hbm", "ms": ph["decode_kv"],
+                                        "achieved_gbs": dec_bytes / (ph["decode_kv"] * 1e-3) / 1e9,
+                                        "frac": dec_bytes / (ph["decode_kv"] * 1e-3) / 1e9 / peaks["hbm_gbs"]},
+    }
+    dominant = {
+        "bound": "tensor", "achieved": rvq_tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+        "frac": rvq_tf / peaks["bf16_tflops"], "traffic": launches_traffic,
+        "kernel": "k_rvq<64> (RVQ assignment), algorithmic 2*64*256 flop per vector-stage, %s peak (fp16 dense = bf16 rate)"
+                  % ("of measured" if peaks["source"] == "measured" else "of fallback"),
+    }
+    return dominant, kernels, dec_bytes, out_bytes
+
+
+# ----------------------------------------------------------- CPU oracle ---
+def oracle_sample(budget_s, cfg=synth.CFG1, max_streams=None):
+    """The float64 oracle on whole (sequence, layer) streams of the workload
+    until `budget_s` seconds of work: RVQ, serialisation, span encode, append,
+    decode, reconstruction and random reads."""
+    import oracle
+    oracle.build()
+    cbk, cbv = synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)
+    r = oracle.packing_ratio(256)
+    L = oracle.max_span_len(r)
+    H = cfg.n_heads
+    P = cfg.n_archived
+    streams = [(b, l) for b in range(cfg.batch) for l in range(cfg.n_layers)]
+    done = 0
+    t_work = 0.0
+    rng = np.random.default_rng(1)
+    for (b, l) in streams:
+        if max_streams is not None and done >= max_streams:
+            break
+        pos = np.arange(cfg.t0, cfg.t1 + 1)                      # archived + appended position
+        hh, tt = np.meshgrid(np.arange(H), pos, indexing="ij")
+        Kx = synth.storage_to_f64(synth.kv_elements(cfg, 0, l, b, hh, tt), cfg.dtype)
+        Vx = synth.storage_to_f64(synth.kv_elements(cfg, 1, l, b, hh, tt), cfg.dtype)
+        t_start = time.perf_counter()
+        ik = np.stack([oracle.rvq_encode(Kx[h], cbk[l, h])[0] for h in range(H)])
+        iv = np.stack([oracle.rvq_encode(Vx[h], cbv[l, h])[0] for h in range(H)])
+        stream = oracle.records_from_indices(ik[:, :P], iv[:, :P])
+        pts = oracle.span_encode(stream, 256, r, L)
+        tail = oracle.records_from_indices(ik[:, P:], iv[:, P:])
+        pts = oracle.append(stream, tail, 256, r, L)
+        full = np.concatenate([stream, tail])
+        dec, _, bad = oracle.span_decode(pts, full.size, 256, r, L)
+        k2, v2 = oracle.indices_from_records(dec, H, cfg.stages_k, cfg.stages_v)
+        for h in range(H):
+            oracle.round_to(oracle.rvq_decode(k2[h], cbk[l, h]), cfg.dtype)
+            oracle.round_to(oracle.rvq_decode(v2[h], cbv[l, h]), cfg.dtype)
+        reads = rng.integers(0, full.size, N_READS // len(streams) + 1)
+        oracle.read(pts, full.size, reads, 256, r, L)
+        t_work += time.perf_counter() - t_start
+        done += 1
+        if t_work >= budget_s:
+            break
+    records = done * (P + 1)
+    return records / t_work, done, t_work, oracle.threads()
+
+
+def cpu_desc():
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True).stdout
+        for ln in out.splitlines():
+            if ln.startswith("Model name"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return "unknown"
+
+
+# ---------------------------------------------------------------- main ----
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="fkv", choices=["fkv", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        per_step = max(1.0, 150.0 / (args.steps + args.warmup))
+        for _ in range(args.warmup):
+            oracle_sample(per_step / 4, max_streams=1)
+        vals = []
+        tot_rec = tot_t = 0.0
+        cores = 1
+        for _ in range(args.steps):
+            v, done, t, cores = oracle_sample(per_step)
+            vals.append(v)
+            tot_rec += v * t
+            tot_t += t
+        value = tot_rec / tot_t
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot_t / args.steps * 1e3,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic",
+                "config": {"workload": "gpt2-shaped full KV cache: 12 layers x batch 8 x 12 heads x 1024 tok x 64, fp16; "
+                                       "K 4 / V 2 RVQ stages x 256; N=256, r=r_256, L=6; bounded sample of whole "
+                                       "(sequence, layer) streams per step", "sample": "whole streams"},
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                 "sample": "whole (sequence, layer) streams, %.0f s of oracle work per step" % per_step,
+                                 "cpu": cpu_desc()},
+                "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    res = run_gpu(args, rank, world, local_rank)
+    ms = res["ms"]
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+        e = torch.tensor([res["e2e"]["ms"] if res["e2e"] else 0.0], device="cuda")
+        torch.distributed.all_reduce(e, op=torch.distributed.ReduceOp.MAX)
+        if res["e2e"]:
+            res["e2e"]["ms"] = float(e.item())
+    if rank != 0:
+        torch.distributed.destroy_process_group()
+        return
+    peaks = load_peaks()
+    traffic = None
+    tp = os.path.join(ROOT, "profiles", "rvq_traffic.json")
+    if os.path.exists(tp):
+        with open(tp) as f:
+            traffic = json.load(f).get("bytes_per_launch_pair")
+    dominant, kernels, dec_bytes, out_bytes = roofline(res, peaks, traffic)
+    units = res["units"] * world
+    value = units / (ms * 1e-3)
+    cpu = None
+    if world == 1 and not args.no_cpu:
+        v, done, t, cores = oracle_sample(args.cpu_budget)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": "%d whole (sequence, layer) streams of the workload (%d records), %.1f s" %
+                         (done, done * res["n_rec"], t), "cpu": cpu_desc()}
+    e2e = None
+    if res["e2e"]:
+        e2e = {"value": units / (res["e2e"]["ms"] * 1e-3), "unit": UNIT,
+               "h2d_bytes_per_step": res["e2e"]["h2d"], "d2h_bytes_per_step": res["e2e"]["d2h"],
+               "ms_per_step": res["e2e"]["ms"]}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "fp16 in / fp16-split tensor / f64 codec", "data": "synthetic",
+        "config": {"workload": "gpt2-shaped full KV cache: 12 layers x batch 8 x 12 heads x 1024 tok x 64 dims, "
+                               "fp16; 4+32 exact window; K 4 / V 2 RVQ stages x 256; N=256, r=r_256, L=6",
+                   "records_per_step": res["units"], "global_batch": 8 * world, "seq_len": 1024,
+                   "l2": "inputs (302 MB) larger than L2; no flush", "parallelism": "replicas (weak)"},
+        "decoded_kv_gbs": out_bytes / (res["phase"]["decode_kv"] * 1e-3) / 1e9,
+        "write_positions_per_s": res["units"] / ((res["phase"]["rvq_k"] + res["phase"]["rvq_v"]
+                                                 + res["phase"]["span_encode"]) * 1e-3),
+        "phase_ms": res["phase"],
+        "roofline": dominant,
+        "kernels": kernels,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 10 * args.steps,
+        "clocks": res["clocks"],
+        "status_ok": res["ok"],
+    }
+    print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,248 @@
+/*
+ * fkv.h -- C ABI of the GB300 fractal KV-cache archive.
+ *
+ * The archive of arXiv 2607.07144: archived K/V head vectors are reduced to
+ * per-head residual-VQ indices (Sec. 3 "Setup"), the indices of each
+ * (sequence, layer) form a symbol stream, and the stream is stored by the
+ * contractive iterated-map code of Sec. 1 "The code" -- one float64 point per
+ * fixed-length span -- which gives lossless, linear-time encoding, O(1)
+ * random access and O(1) amortised append (Sec. 2, Table 1).
+ *
+ * Conventions for every call
+ *   - Return value: FKV_OK (0) or a negative FKV_E* code; on error the reason
+ *     is available from fkv_last_error(ctx) and nothing was launched.
+ *   - Pointers named *_dev (and every data pointer unless stated "host") are
+ *     CUDA device pointers owned by the caller; the library never frees them.
+ *   - `stream` is a cudaStream_t passed as void*; NULL is the legacy default
+ *     stream.  Every call is asynchronous on that stream.
+ *   - Errors found on the device (corrupt points, a failed anchor check) are
+ *     recorded in a per-context status word; fkv_sync_status() waits for the
+ *     stream and returns (and clears) it.  Kernels never trap.
+ *   - A context is not thread-safe: calls on one context must be serialised.
+ *   - Symbols are uint8: alphabets N <= 256 (the paper's k = 256 codebooks).
+ *   - A point is two float64 (x, y), 16 bytes; one point per span.
+ */
+#ifndef FKV_H
+#define FKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FKV_OK 0
+#define FKV_EINVAL (-1)      /* bad argument: range, null pointer, shape */
+#define FKV_ERANGE (-2)      /* a position or record index outside a stream */
+#define FKV_ENOMEM (-3)      /* device or host allocation failed */
+#define FKV_ECUDA (-4)       /* a CUDA runtime/driver call failed */
+#define FKV_ECORRUPT (-5)    /* device status: anchor check failed / bad point */
+#define FKV_ETIMEOUT (-6)    /* device status: a bounded device wait ran out */
+
+/* Element types of K/V caches. */
+#define FKV_F32 0
+#define FKV_F16 1
+#define FKV_BF16 2
+
+typedef struct fkv_ctx fkv_ctx;
+typedef struct fkv_streams fkv_streams;
+
+/* ------------------------------------------------------------ geometry --- */
+
+/* Sec. 1 and Fig. 1 caption: the packing ("kissing") ratio r_N, the largest
+ * contraction ratio for which the N cells V(c) + r (P - V(c)) of the regular
+ * N-gon P are disjoint.  The paper prints no formula; this library uses the
+ * touching ratio of adjacent cells,
+ *     r_N = 1 / (2 (1 + sum_{k=1}^{floor(N/4)} cos(2 pi k / N))),
+ * which is exactly 1/2 for N = 3 and N = 4 as the paper states.
+ * Returns 0.0 for N < 3 or N > 256. */
+double fkv_packing_ratio(int N);
+
+/* Sec. 1: inversion amplifies rounding by 1/r per step, so one IEEE-754
+ * double carries about 44 / log2(1/r) symbols.  Returns
+ * floor(44 / log2(1/r)), or 0 when r is outside (0, 1/2]. */
+int fkv_max_span_len(double r);
+
+/* ----------------------------------------------------------- context --- */
+
+/* Per-head residual-VQ codebooks (Sec. 3 "Setup"; 256 codewords per stage,
+ * one codebook per layer, KV head, K or V and stage).  All host memory,
+ * float32, row-major:
+ *   k: [n_layers][n_heads][stages_k][256][dim]
+ *   v: [n_layers][n_heads][stages_v][256][dim]
+ * dim must be 64 or 128; stages_k, stages_v in [1, 8]. */
+typedef struct {
+    int n_layers;
+    int n_heads;
+    int dim;
+    int stages_k;
+    int stages_v;
+    const float *k;
+    const float *v;
+} fkv_codebooks;
+
+/* Create a context for alphabet size N in [3, 256], contraction ratio r in
+ * (0, r_N] (r_N per fkv_packing_ratio, with a relative slack of 1e-12) and
+ * span length span_len in [1, fkv_max_span_len(r)] (Sec. 1).  cb may be NULL
+ * for a symbol-only codec; when given, its codebooks are copied to the
+ * current CUDA device (the caller keeps ownership of cb's arrays) and N must
+ * be 256.  The context owns the vertex table V(c) (Sec. 1: unit circumradius,
+ * V(0) = (1, 0), counter-clockwise), the codebook copies and a status word.
+ * *out receives the context, or NULL on failure.  Synchronous. */
+int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx **out);
+
+/* Free a context and everything it owns.  NULL is accepted.  Synchronises
+ * the device. */
+int fkv_destroy(fkv_ctx *ctx);
+
+/* Copy the vertex table V(c), c = 0..N-1, to host memory out[N][2]. */
+int fkv_vertices(const fkv_ctx *ctx, double *out);
+
+/* Alphabet size, ratio and span length of a context (any pointer may be NULL). */
+int fkv_params(const fkv_ctx *ctx, int *N, double *r, int *span_len);
+
+/* Last error message of the context (static storage, never NULL). */
+const char *fkv_last_error(const fkv_ctx *ctx);
+
+/* Wait for `stream`, then return and clear the device status word:
+ * FKV_OK, FKV_ECORRUPT or FKV_ETIMEOUT. */
+int fkv_sync_status(fkv_ctx *ctx, void *stream);
+
+/* -------------------------------------------------- bulk symbol codec --- */
+
+/* Sec. 1 / Sec. 2: span-parallel encoding.  Encodes n_streams streams of n
+ * symbols each.  Stream i's symbols are sym_dev[i * sym_stride + k],
+ * k < n (sym_stride in bytes, >= n).  Every span of span_len symbols starts
+ * at the anchor (0, 0) and applies, per symbol c, p <- V(c) + r (p - V(c))
+ * as the binary64 sequence d = p - V(c), t = r * d, p = V(c) + t (no FMA);
+ * the point after the span's last symbol is stored.  The last span of a
+ * stream holds n mod span_len symbols when that is nonzero.  Output: stream i,
+ * span j is the point at pts_dev[2 * (i * pt_stride + j)] (x then y),
+ * pt_stride (in points) >= ceil(n / span_len).  Symbols >= N are reported as
+ * FKV_ECORRUPT in the status word (their span's point is written as NaN). */
+int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int64_t n,
+                    int64_t sym_stride, double *pts_dev, int64_t pt_stride, void *stream);
+
+/* Sec. 1: span-parallel decoding, the inverse of fkv_span_encode (same
+ * layouts).  Each span is decoded from its stored point, last symbol first:
+ * the symbol is the vertex whose cell holds the point (the nearest vertex,
+ * since r <= r_N puts every cell inside its vertex's Voronoi region), then
+ * p <- (p - (1 - r) V(c)) / r.  After a span's first symbol the point must be
+ * back at the anchor: a residual above 2^-4 in either coordinate sets
+ * FKV_ECORRUPT in the status word (the symbols are still written). */
+int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n,
+                    int64_t pt_stride, uint8_t *sym_dev, int64_t sym_stride, void *stream);
+
+/* Sec. 2, Table 1: O(1) random access.  For each request q < n_req,
+ * req_dev[2q] = stream index, req_dev[2q + 1] = symbol position, writes the
+ * symbol at that position to out_dev[q] by decoding only the span holding it
+ * (at most span_len backward steps).  Points laid out as in fkv_span_encode.
+ * A request outside [0, n_streams) x [0, n) writes 0xFF to out_dev[q] and
+ * sets FKV_ECORRUPT. */
+int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
+             const int64_t *req_dev, int64_t n_req, uint8_t *out_dev, void *stream);
+
+/* -------------------------------------------------- K/V archive path ---- */
+
+/* A K or V cache tensor on the device: head vectors of `dim` contiguous
+ * elements indexed by (layer, sequence, head, position) with the element
+ * strides below.  The usual layout [n_layers][batch][n_heads][seq][dim] has
+ * stride_pos = dim, stride_head = seq * dim, and so on. */
+typedef struct {
+    void *data;
+    int dtype;              /* FKV_F32, FKV_F16 or FKV_BF16 */
+    int64_t batch;          /* sequences */
+    int64_t seq;            /* positions per (layer, sequence, head) */
+    int64_t stride_layer;
+    int64_t stride_batch;
+    int64_t stride_head;
+    int64_t stride_pos;
+} fkv_cache;
+
+/* Symbols per token record: n_heads * (stages_k + stages_v). */
+int fkv_record_len(const fkv_ctx *ctx);
+
+/* Sec. 3 "Setup": per-head residual-VQ assignment of every archived vector.
+ * kv = 0 quantises keys (stages_k stages), kv = 1 values (stages_v).  For
+ * each layer l, sequence b, head h and position t in [t0, t1) of `x`, stage
+ * by stage the index is the codeword of codebook (l, h, kv, stage) nearest in
+ * squared L2 to the running residual (lowest index on a tie), and the
+ * residual then drops that codeword.  Indices are written in token-record
+ * order (the paper does not fix one): stream (b * n_layers + l) starts at
+ * sym_dev + (b * n_layers + l) * stream_stride; the record of position t is
+ * record rec0 + (t - t0) of R = fkv_record_len symbols, holding the key
+ * indices of heads 0..H-1 (stages inner) then the value indices likewise.
+ * Only the kv half of each record is written.  Runs on the tensor cores
+ * (tcgen05) with split-fp16 operands whose score error is below 5e-5 of the
+ * residual's squared norm; ties closer than that may differ from a float64
+ * search. */
+int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
+                   uint8_t *sym_dev, int64_t stream_stride, int64_t rec0, void *stream);
+
+/* Sec. 3 "Setup": the reconstruction is the sum of the selected centroids.
+ * Rebuilds positions [t0, t0 + n_rec) of every (layer, sequence, head) of
+ * k_out and v_out (either may be NULL) from records 0..n_rec-1 of the symbol
+ * streams laid out as in fkv_rvq_encode: sum of the stage codewords in
+ * float32, stage order, rounded to nearest-even into the cache dtype. */
+int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, int64_t n_rec,
+                   fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
+
+/* Sec. 1-3: full archive read.  Decodes records 0..n_rec-1 of the
+ * batch * n_layers streams (stream (b * n_layers + l) holds n_rec * R symbols,
+ * its points at pts_dev + 2 * (b * n_layers + l) * pt_stride) and writes the
+ * reconstructed K and V at positions [t0, t0 + n_rec), as fkv_span_decode
+ * followed by fkv_rvq_decode.  Uses a context-owned scratch buffer of
+ * batch * n_layers * n_rec * R bytes, grown on demand (a synchronous
+ * allocation the first time a larger archive is decoded). */
+int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
+                  fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
+
+/* Sec. 2 random access at record granularity: for each request q,
+ * req_dev[2q] = stream (b * n_layers + l), req_dev[2q + 1] = record index,
+ * decode only the spans of that record and write its K and V head vectors to
+ * out_dev, laid out [n_req][2 (K, V)][n_heads][dim] in `dtype`.  Streams hold
+ * n_rec records each, points as in fkv_decode_kv.  Out-of-range requests
+ * write zeros and set FKV_ECORRUPT. */
+int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec,
+                int64_t pt_stride, const int64_t *req_dev, int64_t n_req, void *out_dev,
+                int dtype, void *stream);
+
+/* ------------------------------------------------- appendable streams --- */
+
+/* A set of n_streams symbol streams of equal length, owned by the library on
+ * the device: points [n_streams][capacity_spans][2] float64, the last point
+ * of a stream being its partial tail span's point.  Initial length 0. */
+int fkv_streams_create(fkv_ctx *ctx, int64_t n_streams, int64_t capacity_symbols,
+                       fkv_streams **out);
+int fkv_streams_destroy(fkv_streams *s);
+
+/* Empty every stream of the set (length 0), keeping its device buffer. */
+int fkv_streams_reset(fkv_streams *s);
+
+/* Current geometry: symbols per stream, point stride (points between
+ * streams) and the device point buffer (valid until the next append that
+ * grows the set).  Any output pointer may be NULL. */
+int fkv_streams_info(const fkv_streams *s, int64_t *n_streams, int64_t *length,
+                     int64_t *pt_stride, double **pts_dev);
+
+/* Sec. 2, Table 1: O(1) amortised append.  Appends m symbols to every stream:
+ * stream i's new symbols are sym_dev[i * sym_stride + k], k < m.  Only the
+ * tail is re-walked: the partial last span continues from its stored point,
+ * later spans start at the anchor; sealed spans are never touched.  The
+ * result is bit-identical to encoding the extended streams from scratch.
+ * The point buffer grows geometrically (x2) when full, with a device copy. */
+int fkv_append(fkv_ctx *ctx, fkv_streams *s, const uint8_t *sym_dev, int64_t m,
+               int64_t sym_stride, void *stream);
+
+/* Checkpoint: copy a stream set's length and points to host memory
+ * (host_pts: [n_streams][ceil(length / span_len)][2]), and rebuild a set
+ * from such a copy.  The archive is its own serialised form. */
+int fkv_streams_export(const fkv_streams *s, int64_t *length, double *host_pts, void *stream);
+int fkv_streams_import(fkv_ctx *ctx, int64_t n_streams, int64_t length, const double *host_pts,
+                       fkv_streams **out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FKV_H */

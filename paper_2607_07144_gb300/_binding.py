@@ -1,0 +1,317 @@
+"""ctypes binding of libfkv.so (include/fkv.h).  Argument marshalling only:
+every step of the archive path runs in the library's CUDA kernels.  PyTorch
+supplies device memory and the current CUDA stream."""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libfkv.so")
+
+OK, EINVAL, ERANGE, ENOMEM, ECUDA, ECORRUPT, ETIMEOUT = 0, -1, -2, -3, -4, -5, -6
+F32, F16, BF16 = 0, 1, 2
+_DTYPE = {torch.float32: F32, torch.float16: F16, torch.bfloat16: BF16}
+_ERRNAME = {EINVAL: "EINVAL", ERANGE: "ERANGE", ENOMEM: "ENOMEM", ECUDA: "ECUDA",
+            ECORRUPT: "ECORRUPT", ETIMEOUT: "ETIMEOUT"}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class FkvError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__("%s (%d): %s" % (_ERRNAME.get(code, "?"), code, msg))
+        self.code = code
+
+
+class _Codebooks(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int), ("n_heads", ctypes.c_int), ("dim", ctypes.c_int),
+                ("stages_k", ctypes.c_int), ("stages_v", ctypes.c_int),
+                ("k", ctypes.c_void_p), ("v", ctypes.c_void_p)]
+
+
+class _Cache(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("dtype", ctypes.c_int), ("batch", ctypes.c_int64),
+                ("seq", ctypes.c_int64), ("stride_layer", ctypes.c_int64),
+                ("stride_batch", ctypes.c_int64), ("stride_head", ctypes.c_int64),
+                ("stride_pos", ctypes.c_int64)]
+
+
+# name -> (restype, argtypes)
+_P, _I, _I64, _D = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
+SIGNATURES = {
+    "fkv_packing_ratio": (_D, [_I]),
+    "fkv_max_span_len": (_I, [_D]),
+    "fkv_create": (_I, [_I, _D, _I, _P, ctypes.POINTER(_P)]),
+    "fkv_destroy": (_I, [_P]),
+    "fkv_vertices": (_I, [_P, _P]),
+    "fkv_params": (_I, [_P, _P, _P, _P]),
+    "fkv_last_error": (ctypes.c_char_p, [_P]),
+    "fkv_sync_status": (_I, [_P, _P]),
+    "fkv_span_encode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
+    "fkv_span_decode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
+    "fkv_read": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _P]),
+    "fkv_record_len": (_I, [_P]),
+    "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
+    "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
+    "fkv_decode_kv": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
+    "fkv_read_kv": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _I, _P]),
+    "fkv_streams_create": (_I, [_P, _I64, _I64, ctypes.POINTER(_P)]),
+    "fkv_streams_destroy": (_I, [_P]),
+    "fkv_streams_reset": (_I, [_P]),
+    "fkv_streams_info": (_I, [_P, _P, _P, _P, _P]),
+    "fkv_append": (_I, [_P, _P, _P, _I64, _I64, _P]),
+    "fkv_streams_export": (_I, [_P, _P, _P, _P]),
+    "fkv_streams_import": (_I, [_P, _I64, _I64, _P, ctypes.POINTER(_P)]),
+}
+
+
+def lib():
+    """The loaded library.  Raises if it has not been built: there is no
+    fallback implementation."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError("libfkv.so is not built (run __graft_entry__.build())")
+            L = ctypes.CDLL(LIB_PATH)
+            for name, (res, args) in SIGNATURES.items():
+                f = getattr(L, name)
+                f.restype = res
+                f.argtypes = args
+            _lib = L
+        return _lib
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t: torch.Tensor):
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _rows(t: torch.Tensor, unit: int = 1) -> int:
+    """Row stride of a [rows, ...] tensor in units of `unit` elements; a
+    single row has no meaningful stride, so report its own extent."""
+    if t.shape[0] <= 1:
+        return max(1, t[0].numel() // unit if t.shape[0] else 1)
+    return t.stride(0) // unit
+
+
+def packing_ratio(N: int) -> float:
+    return lib().fkv_packing_ratio(int(N))
+
+
+def max_span_len(r: float) -> int:
+    return lib().fkv_max_span_len(float(r))
+
+
+def cache_view(t: torch.Tensor) -> _Cache:
+    """fkv_cache view of a CUDA tensor shaped [n_layers, batch, n_heads, seq, dim]
+    (any strides with a contiguous last dimension)."""
+    if t.dim() != 5 or t.stride(4) != 1 or not t.is_cuda:
+        raise ValueError("cache must be a CUDA tensor [layers, batch, heads, seq, dim] with contiguous dim")
+    c = _Cache()
+    c.data = t.data_ptr()
+    c.dtype = _DTYPE[t.dtype]
+    c.batch = t.shape[1]
+    c.seq = t.shape[3]
+    c.stride_layer, c.stride_batch, c.stride_head, c.stride_pos = t.stride(0), t.stride(1), t.stride(2), t.stride(3)
+    return c
+
+
+class Context:
+    """An fkv_ctx: alphabet N, ratio r (default r_N), span length (default
+    floor(44/log2(1/r))) and optional per-head codebooks (k, v) as float32
+    arrays [n_layers, n_heads, stages, 256, dim]."""
+
+    def __init__(self, N: int, r: float = None, span_len: int = None, codebooks=None):
+        L = lib()
+        self.N = int(N)
+        self.r = float(r) if r is not None else L.fkv_packing_ratio(self.N)
+        self.L = int(span_len) if span_len is not None else L.fkv_max_span_len(self.r)
+        self._h = ctypes.c_void_p()
+        cbp = None
+        if codebooks is not None:
+            k, v = (np.ascontiguousarray(a, np.float32) for a in codebooks)
+            if k.ndim != 5 or v.ndim != 5 or k.shape[:2] != v.shape[:2] or k.shape[4] != v.shape[4]:
+                raise ValueError("codebooks must be [layers, heads, stages, 256, dim]")
+            self._cb_arrays = (k, v)          # keep alive during create
+            cb = _Codebooks(k.shape[0], k.shape[1], k.shape[4], k.shape[2], v.shape[2],
+                            k.ctypes.data, v.ctypes.data)
+            cbp = ctypes.byref(cb)
+            self.n_layers, self.n_heads, self.dim = k.shape[0], k.shape[1], k.shape[4]
+            self.stages_k, self.stages_v = k.shape[2], v.shape[2]
+        rc = L.fkv_create(self.N, self.r, self.L, cbp, ctypes.byref(self._h))
+        self._cb_arrays = None
+        if rc != OK:
+            raise FkvError(rc, "fkv_create(N=%d, r=%r, span_len=%d) rejected" % (self.N, self.r, self.L))
+
+    # -- plumbing
+    def _check(self, rc):
+        if rc != OK:
+            raise FkvError(rc, lib().fkv_last_error(self._h).decode())
+
+    def close(self):
+        if self._h:
+            lib().fkv_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def handle(self):
+        return self._h
+
+    # -- ABI calls
+    def vertices(self) -> np.ndarray:
+        out = np.empty((self.N, 2), np.float64)
+        self._check(lib().fkv_vertices(self._h, out.ctypes.data))
+        return out
+
+    def record_len(self) -> int:
+        return lib().fkv_record_len(self._h)
+
+    def sync_status(self, stream=None) -> int:
+        return lib().fkv_sync_status(self._h, _stream(stream))
+
+    def n_spans(self, n: int) -> int:
+        return (int(n) + self.L - 1) // self.L
+
+    def span_encode(self, sym: torch.Tensor, pts: torch.Tensor = None, stream=None) -> torch.Tensor:
+        """sym uint8 [n_streams, n] -> pts float64 [n_streams, spans, 2]."""
+        ns, n = sym.shape
+        if pts is None:
+            pts = torch.empty((ns, self.n_spans(n), 2), dtype=torch.float64, device=sym.device)
+        self._check(lib().fkv_span_encode(self._h, _ptr(sym), ns, n, _rows(sym), _ptr(pts), _rows(pts, 2),
+                                          _stream(stream)))
+        return pts
+
+    def span_decode(self, pts: torch.Tensor, n: int, sym: torch.Tensor = None, stream=None) -> torch.Tensor:
+        ns = pts.shape[0]
+        if sym is None:
+            sym = torch.empty((ns, n), dtype=torch.uint8, device=pts.device)
+        self._check(lib().fkv_span_decode(self._h, _ptr(pts), ns, n, _rows(pts, 2), _ptr(sym), _rows(sym),
+                                          _stream(stream)))
+        return sym
+
+    def read(self, pts: torch.Tensor, n: int, req: torch.Tensor, out: torch.Tensor = None, stream=None):
+        """req int64 [n_req, 2] = (stream, position) -> uint8 [n_req]."""
+        if out is None:
+            out = torch.empty(req.shape[0], dtype=torch.uint8, device=pts.device)
+        self._check(lib().fkv_read(self._h, _ptr(pts), pts.shape[0], n, _rows(pts, 2), _ptr(req), req.shape[0],
+                                   _ptr(out), _stream(stream)))
+        return out
+
+    def rvq_encode(self, kv: int, x: torch.Tensor, t0: int, t1: int, sym: torch.Tensor, rec0: int = 0, stream=None):
+        """x: cache [layers, batch, heads, seq, dim]; sym: uint8 [batch*layers, >= (rec0+t1-t0)*R]."""
+        c = cache_view(x)
+        self._check(lib().fkv_rvq_encode(self._h, int(kv), ctypes.byref(c), t0, t1, _ptr(sym), _rows(sym), rec0,
+                                         _stream(stream)))
+        return sym
+
+    def rvq_decode(self, sym: torch.Tensor, n_rec: int, k_out: torch.Tensor = None, v_out: torch.Tensor = None,
+                   t0: int = 0, stream=None):
+        ck = cache_view(k_out) if k_out is not None else None
+        cv = cache_view(v_out) if v_out is not None else None
+        self._check(lib().fkv_rvq_decode(self._h, _ptr(sym), _rows(sym), n_rec,
+                                         ctypes.byref(ck) if ck else None, ctypes.byref(cv) if cv else None,
+                                         t0, _stream(stream)))
+
+    def decode_kv(self, pts: torch.Tensor, n_rec: int, k_out: torch.Tensor = None, v_out: torch.Tensor = None,
+                  t0: int = 0, stream=None):
+        ck = cache_view(k_out) if k_out is not None else None
+        cv = cache_view(v_out) if v_out is not None else None
+        self._check(lib().fkv_decode_kv(self._h, _ptr(pts), n_rec, _rows(pts, 2),
+                                        ctypes.byref(ck) if ck else None, ctypes.byref(cv) if cv else None,
+                                        t0, _stream(stream)))
+
+    def read_kv(self, pts: torch.Tensor, n_rec: int, req: torch.Tensor, out: torch.Tensor, stream=None):
+        """req int64 [n_req, 2] = (stream, record) -> out [n_req, 2, heads, dim]."""
+        self._check(lib().fkv_read_kv(self._h, _ptr(pts), pts.shape[0], n_rec, _rows(pts, 2), _ptr(req),
+                                      req.shape[0], _ptr(out), _DTYPE[out.dtype], _stream(stream)))
+        return out
+
+
+class Streams:
+    """An fkv_streams set: n_streams library-owned appendable streams."""
+
+    def __init__(self, ctx: Context, n_streams: int, capacity: int = 0, _handle=None):
+        self.ctx = ctx
+        self._h = ctypes.c_void_p()
+        if _handle is not None:
+            self._h = _handle
+        else:
+            ctx._check(lib().fkv_streams_create(ctx.handle, n_streams, capacity, ctypes.byref(self._h)))
+
+    @classmethod
+    def import_(cls, ctx: Context, length: int, host_pts: np.ndarray):
+        h = ctypes.c_void_p()
+        p = np.ascontiguousarray(host_pts, np.float64)
+        ctx._check(lib().fkv_streams_import(ctx.handle, p.shape[0], length, p.ctypes.data, ctypes.byref(h)))
+        return cls(ctx, p.shape[0], _handle=h)
+
+    def info(self):
+        ns, ln, st = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+        p = ctypes.c_void_p()
+        lib().fkv_streams_info(self._h, ctypes.byref(ns), ctypes.byref(ln), ctypes.byref(st), ctypes.byref(p))
+        return ns.value, ln.value, st.value, p.value
+
+    def points(self) -> torch.Tensor:
+        """A [n_streams, cap_spans, 2] float64 view of the library-owned point
+        buffer (valid until the next growing append)."""
+        ns, ln, st, p = self.info()
+        return _device_view(p, (ns, st, 2))
+
+    @property
+    def length(self) -> int:
+        return self.info()[1]
+
+    def reset(self):
+        lib().fkv_streams_reset(self._h)
+
+    def append(self, sym: torch.Tensor, stream=None):
+        """sym uint8 [n_streams, m]."""
+        self.ctx._check(lib().fkv_append(self.ctx.handle, self._h, _ptr(sym), sym.shape[1], _rows(sym),
+                                         _stream(stream)))
+
+    def export(self, stream=None) -> np.ndarray:
+        ns, ln, st, p = self.info()
+        out = np.empty((ns, self.ctx.n_spans(ln), 2), np.float64)
+        length = ctypes.c_int64()
+        self.ctx._check(lib().fkv_streams_export(self._h, ctypes.byref(length), out.ctypes.data, _stream(stream)))
+        return out
+
+    def close(self):
+        if self._h:
+            lib().fkv_streams_destroy(self._h)
+            self._h = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def _device_view(ptr: int, shape):
+    """Wrap a library-owned float64 device buffer as a torch tensor (no copy)."""
+    n = int(np.prod(shape))
+
+    class _Holder:
+        __cuda_array_interface__ = {"shape": tuple(shape), "typestr": "<f8", "data": (ptr, False),
+                                    "version": 3, "strides": None}
+    if n == 0:
+        return torch.empty(shape, dtype=torch.float64, device="cuda")
+    return torch.as_tensor(_Holder(), device="cuda")

@@ -1,0 +1,369 @@
+// Span codec kernels: the iterated-map code of Sec. 1 "The code", applied
+// span-parallel (one span per thread) for encoding, decoding, random reads
+// and tail appends (Sec. 2, Table 1).
+//
+// Encoding must reproduce the binary64 walk bit for bit, so it runs on the
+// FP64 pipe with explicit round-to-nearest intrinsics (no FMA contraction):
+// d = p - V(c); t = r * d; p = V(c) + t per coordinate.
+//
+// Decoding only has to recover the symbols, so it runs in exact 64-bit
+// fixed point (Q1.62) on the integer pipes: the nearest vertex is found from
+// exact dot products, and p <- (p - (1-r) V(c)) / r becomes a subtraction and
+// a 64x64->128-bit multiply by a fixed-point 1/r.
+#include "fkv_internal.h"
+
+namespace {
+
+constexpr int kThreads = 256;   // spans per block
+constexpr int kMaxSpan = 44;    // floor(44 / log2(1/r)) with r <= 1/2
+constexpr int kStageBytes = kThreads * kMaxSpan + 32;
+
+// Copy len bytes from global src into shared buf so that buf[off + i] =
+// src[i], off = src mod 16: aligned 16-byte vectors inside the range, single
+// bytes at the two ragged ends.  Never touches bytes outside [src, src+len).
+__device__ __forceinline__ int stage_in(uint8_t *buf, const uint8_t *src, int len)
+{
+    const int off = static_cast<int>(reinterpret_cast<uintptr_t>(src) & 15);
+    const uint8_t *a = src - off;
+    const int total = off + len;
+    const int nv = (total + 15) >> 4;
+    for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+        const int b0 = v << 4;
+        if (b0 >= off && b0 + 16 <= total) {
+            *reinterpret_cast<uint4 *>(buf + b0) = __ldg(reinterpret_cast<const uint4 *>(a + b0));
+        } else {
+            const int lo = b0 > off ? b0 : off;
+            const int hi = b0 + 16 < total ? b0 + 16 : total;
+            for (int q = lo; q < hi; ++q)
+                buf[q] = a[q];
+        }
+    }
+    return off;
+}
+
+// The mirror of stage_in: dst[i] = buf[off + i], off = dst mod 16.
+__device__ __forceinline__ void stage_out(uint8_t *dst, const uint8_t *buf, int len, int off)
+{
+    uint8_t *a = dst - off;
+    const int total = off + len;
+    const int nv = (total + 15) >> 4;
+    for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+        const int b0 = v << 4;
+        if (b0 >= off && b0 + 16 <= total) {
+            *reinterpret_cast<uint4 *>(a + b0) = *reinterpret_cast<const uint4 *>(buf + b0);
+        } else {
+            const int lo = b0 > off ? b0 : off;
+            const int hi = b0 + 16 < total ? b0 + 16 : total;
+            for (int q = lo; q < hi; ++q)
+                a[q] = buf[q];
+        }
+    }
+}
+
+// Sec. 1 forward map for one span from the anchor (0, 0), binary64, no FMA.
+__device__ __forceinline__ double2 encode_span(const uint8_t *s, int m, const double2 *sV, double r,
+                                               double x, double y)
+{
+    for (int k = 0; k < m; ++k) {
+        const double2 v = sV[s[k]];
+        const double dx = __dsub_rn(x, v.x);
+        const double dy = __dsub_rn(y, v.y);
+        const double tx = __dmul_rn(r, dx);
+        const double ty = __dmul_rn(r, dy);
+        x = __dadd_rn(v.x, tx);
+        y = __dadd_rn(v.y, ty);
+    }
+    return make_double2(x, y);
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_span_encode(const uint8_t *__restrict__ sym, int64_t n, int64_t sym_stride, int64_t spans, int bps,
+              double2 *__restrict__ pts, int64_t pt_stride, const double2 *__restrict__ V, double r, int L,
+              unsigned *status)
+{
+    __shared__ __align__(16) uint8_t sbuf[kStageBytes];
+    __shared__ double2 sV[256];
+    const int64_t stream = blockIdx.x / bps;
+    const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
+    sV[threadIdx.x] = V[threadIdx.x];
+    const int64_t b = s0 * L;
+    const int64_t e = min(n, (s0 + kThreads) * L);
+    const int off = stage_in(sbuf, sym + stream * sym_stride + b, static_cast<int>(e - b));
+    __syncthreads();
+    const int64_t s = s0 + threadIdx.x;
+    if (s < spans) {
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+        const double2 p = encode_span(sbuf + off + threadIdx.x * L, m, sV, r, 0.0, 0.0);
+        if (isnan(p.x))   // a symbol >= N reads a NaN vertex
+            atomicOr(status, FKV_ST_CORRUPT);
+        pts[stream * pt_stride + s] = p;
+    }
+}
+
+// ------------------------------------------------------------- decoding
+struct DecShared {
+    long long vx[256], vy[256], wx[256], wy[256], hn[256];
+};
+
+__device__ __forceinline__ void load_dec(DecShared &d, const fkv_decconst *__restrict__ g)
+{
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+        d.vx[i] = g->vx[i];
+        d.vy[i] = g->vy[i];
+        d.wx[i] = g->wx[i];
+        d.wy[i] = g->wy[i];
+        d.hn[i] = g->hn[i];
+    }
+}
+
+__device__ __forceinline__ long long to_q62(double v)
+{
+    return __double2ll_rn(v * 4611686018427387904.0);   // v * 2^62, exact scaling
+}
+
+// Nearest vertex of (X, Y): argmax of p.V(c) - |V(c)|^2 / 2 (units 2^-60).
+__device__ __forceinline__ long long vscore(const DecShared &d, long long X, long long Y, int c)
+{
+    return __mul64hi(X, d.vx[c]) + __mul64hi(Y, d.vy[c]) - d.hn[c];
+}
+
+__device__ __forceinline__ int classify(const DecShared &d, long long X, long long Y, int N)
+{
+    if (N <= 8) {
+        int best = 0;
+        long long bs = vscore(d, X, Y, 0);
+        for (int c = 1; c < N; ++c) {
+            const long long s = vscore(d, X, Y, c);
+            if (s > bs) {
+                bs = s;
+                best = c;
+            }
+        }
+        return best;
+    }
+    // Voronoi regions of the vertices are the angular sectors around them, so
+    // the angle picks the sector up to one neighbour; the exact dot products
+    // then decide between the three candidates.
+    const float xf = static_cast<float>(static_cast<int>(X >> 32));
+    const float yf = static_cast<float>(static_cast<int>(Y >> 32));
+    const float a = atan2f(yf, xf) * (static_cast<float>(N) * 0.15915494309189535f);
+    int c0 = __float2int_rn(a);
+    if (c0 < 0)
+        c0 += N;
+    if (c0 >= N)
+        c0 -= N;
+    const int cm = c0 == 0 ? N - 1 : c0 - 1;
+    const int cp = c0 == N - 1 ? 0 : c0 + 1;
+    int best = c0;
+    long long bs = vscore(d, X, Y, c0);
+    long long s = vscore(d, X, Y, cm);
+    if (s > bs) {
+        bs = s;
+        best = cm;
+    }
+    s = vscore(d, X, Y, cp);
+    if (s > bs)
+        best = cp;
+    return best;
+}
+
+// (v * rinv) >> k with a 128-bit intermediate product, 1 <= k <= 63.
+__device__ __forceinline__ long long mulshift(long long v, long long rinv, int k)
+{
+    const unsigned long long lo = static_cast<unsigned long long>(v) * static_cast<unsigned long long>(rinv);
+    const long long hi = __mul64hi(v, rinv);
+    return static_cast<long long>((lo >> k) | (static_cast<unsigned long long>(hi) << (64 - k)));
+}
+
+// One backward step of Sec. 1: classify, then p <- (p - (1-r) V(c)) / r.
+__device__ __forceinline__ int decode_step(const DecShared &d, long long &X, long long &Y, int N,
+                                           long long rinv, int rsh)
+{
+    const int c = classify(d, X, Y, N);
+    X = mulshift(static_cast<long long>(static_cast<unsigned long long>(X) - static_cast<unsigned long long>(d.wx[c])), rinv, rsh);
+    Y = mulshift(static_cast<long long>(static_cast<unsigned long long>(Y) - static_cast<unsigned long long>(d.wy[c])), rinv, rsh);
+    return c;
+}
+
+// Anchor check: after a span's first symbol the point is back at (0, 0);
+// a residual above 2^-4 (2^58 in Q62) flags a corrupt point.
+__device__ __forceinline__ bool anchor_ok(long long X, long long Y)
+{
+    const long long lim = 1ll << 58;
+    return X <= lim && X >= -lim && Y <= lim && Y >= -lim;
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
+              uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc, int N,
+              int L, unsigned *status)
+{
+    __shared__ __align__(16) uint8_t sbuf[kStageBytes];
+    __shared__ DecShared sd;
+    const int64_t stream = blockIdx.x / bps;
+    const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
+    load_dec(sd, dc);
+    const long long rinv = dc->rinv;
+    const int rsh = dc->rshift;
+    const int64_t b = s0 * L;
+    const int64_t e = min(n, (s0 + kThreads) * L);
+    uint8_t *dst = sym + stream * sym_stride + b;
+    const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
+    __syncthreads();
+    const int64_t s = s0 + threadIdx.x;
+    if (s < spans) {
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+        const double2 p = pts[stream * pt_stride + s];
+        long long X = to_q62(p.x), Y = to_q62(p.y);
+        uint8_t *my = sbuf + off + threadIdx.x * L;
+        for (int k = m - 1; k >= 0; --k)
+            my[k] = static_cast<uint8_t>(decode_step(sd, X, Y, N, rinv, rsh));
+        if (!anchor_ok(X, Y))
+            atomicOr(status, FKV_ST_CORRUPT);
+    }
+    __syncthreads();
+    stage_out(dst, sbuf, static_cast<int>(e - b), off);
+}
+
+// Sec. 2 random access: one request per thread, decoding only its span.
+__global__ void __launch_bounds__(kThreads)
+k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride,
+       const int64_t *__restrict__ req, int64_t n_req, uint8_t *__restrict__ out,
+       const fkv_decconst *__restrict__ dc, int N, int L, unsigned *status)
+{
+    __shared__ DecShared sd;
+    load_dec(sd, dc);
+    const long long rinv = dc->rinv;
+    const int rsh = dc->rshift;
+    __syncthreads();
+    const int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
+    if (q >= n_req)
+        return;
+    const int64_t st = req[2 * q], pos = req[2 * q + 1];
+    if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
+        out[q] = 0xFF;
+        atomicOr(status, FKV_ST_CORRUPT);
+        return;
+    }
+    const int64_t u = pos / L;
+    const int o = static_cast<int>(pos - u * L);
+    const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+    const double2 p = pts[st * pt_stride + u];
+    long long X = to_q62(p.x), Y = to_q62(p.y);
+    int c = 0;
+    for (int k = m - 1; k >= o; --k)
+        c = decode_step(sd, X, Y, N, rinv, rsh);
+    out[q] = static_cast<uint8_t>(c);
+}
+
+// Sec. 2 append: one thread per (stream, span touched by the new symbols).
+// The first touched span continues from the stored tail point when the old
+// length is not a multiple of L; every later span starts at the anchor.
+__global__ void __launch_bounds__(kThreads)
+k_append(double2 *__restrict__ pts, int64_t n_streams, int64_t pt_stride, int64_t n_old,
+         const uint8_t *__restrict__ sym, int64_t m, int64_t sym_stride, int64_t u_first, int64_t cnt,
+         const double2 *__restrict__ V, double r, int L, unsigned *status)
+{
+    __shared__ double2 sV[256];
+    sV[threadIdx.x] = V[threadIdx.x];
+    __syncthreads();
+    const int64_t t = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
+    if (t >= n_streams * cnt)
+        return;
+    const int64_t stream = t / cnt;
+    const int64_t u = u_first + (t - stream * cnt);
+    const int64_t n_new = n_old + m;
+    const int64_t b = max(u * L, n_old);
+    const int64_t e = min((u + 1) * L, n_new);
+    double2 p = make_double2(0.0, 0.0);
+    if (u * L < n_old)
+        p = pts[stream * pt_stride + u];
+    uint8_t s[kMaxSpan];
+    const uint8_t *src = sym + stream * sym_stride + (b - n_old);
+    const int len = static_cast<int>(e - b);
+    for (int k = 0; k < len; ++k)
+        s[k] = src[k];
+    p = encode_span(s, len, sV, r, p.x, p.y);
+    if (isnan(p.x))
+        atomicOr(status, FKV_ST_CORRUPT);
+    pts[stream * pt_stride + u] = p;
+}
+
+inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+}  // namespace
+
+cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_streams, int64_t n,
+                               int64_t sym_stride, double *pts, int64_t pt_stride, cudaStream_t st)
+{
+    const int64_t spans = cdiv(n, c->L);
+    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t blocks = n_streams * bps;
+    if (blocks == 0)
+        return cudaSuccess;
+    if (blocks > 0x7FFFFFFF)
+        return cudaErrorInvalidConfiguration;
+    k_span_encode<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+        sym, n, sym_stride, spans, static_cast<int>(bps), reinterpret_cast<double2 *>(pts), pt_stride,
+        c->d_V, c->r, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                               int64_t pt_stride, uint8_t *sym, int64_t sym_stride, cudaStream_t st)
+{
+    const int64_t spans = cdiv(n, c->L);
+    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t blocks = n_streams * bps;
+    if (blocks == 0)
+        return cudaSuccess;
+    if (blocks > 0x7FFFFFFF)
+        return cudaErrorInvalidConfiguration;
+    k_span_decode<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+        reinterpret_cast<const double2 *>(pts), n, pt_stride, spans, static_cast<int>(bps), sym,
+        sym_stride, c->d_dec, c->N, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                        int64_t pt_stride, const int64_t *req, int64_t n_req, uint8_t *out,
+                        cudaStream_t st)
+{
+    const int64_t blocks = cdiv(n_req, kThreads);
+    if (blocks == 0)
+        return cudaSuccess;
+    if (blocks > 0x7FFFFFFF)
+        return cudaErrorInvalidConfiguration;
+    k_read<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+        reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride, req, n_req, out, c->d_dec, c->N,
+        c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
+                          int64_t n_old, const uint8_t *sym, int64_t m, int64_t sym_stride,
+                          cudaStream_t st)
+{
+    if (m <= 0 || n_streams <= 0)
+        return cudaSuccess;
+    const int L = c->L;
+    int64_t head = 0;   // new symbols that finish the stored partial span
+    if (n_old % L) {
+        head = min(m, L - n_old % L);
+        const int64_t blocks = cdiv(n_streams, kThreads);
+        if (blocks > 0x7FFFFFFF)
+            return cudaErrorInvalidConfiguration;
+        k_append<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+            reinterpret_cast<double2 *>(pts), n_streams, pt_stride, n_old, sym, head, sym_stride, n_old / L, 1,
+            c->d_V, c->r, L, c->d_status);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess)
+            return e;
+    }
+    if (m == head)
+        return cudaSuccess;
+    // every later span starts at the anchor: the bulk span encoder on the
+    // remaining symbols, writing from span (n_old + head) / L on
+    return launch_span_encode(c, sym + head, n_streams, m - head, sym_stride,
+                              pts + 2 * ((n_old + head) / L), pt_stride, st);
+}

@@ -1,0 +1,618 @@
+// Host side of the C ABI declared in include/fkv.h: argument checks, the
+// context (vertex table, decoder constants, codebook copies), stream sets,
+// and the launches of the kernels in codec.cu, rvq.cu and gather.cu.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <cstdlib>
+#include <mutex>
+#include <vector>
+
+#include "fkv_internal.h"
+
+namespace {
+
+const char *kNoCtx = "no context";
+
+int fail(fkv_ctx *c, int code, const char *msg)
+{
+    if (c)
+        c->err = msg;
+    return code;
+}
+
+int cuda_fail(fkv_ctx *c, cudaError_t e, const char *where)
+{
+    if (c) {
+        c->err = std::string(where) + ": " + cudaGetErrorString(e);
+    }
+    return e == cudaErrorMemoryAllocation ? FKV_ENOMEM : FKV_ECUDA;
+}
+
+#define CK(call, where)                              \
+    do {                                             \
+        cudaError_t e_ = (call);                     \
+        if (e_ != cudaSuccess)                       \
+            return cuda_fail(ctx, e_, where);        \
+    } while (0)
+
+// Sec. 1 vertex table: unit circumradius, V(0) = (1, 0), counter-clockwise,
+// the angle 2*pi*c/N in binary64; quarter turns are exactly 0 and +-1.
+void vertex(int N, int c, double *x, double *y)
+{
+    if ((4 * c) % N == 0) {
+        const int q = (4 * c) / N;
+        *x = q == 0 ? 1.0 : (q == 2 ? -1.0 : 0.0);
+        *y = q == 1 ? 1.0 : (q == 3 ? -1.0 : 0.0);
+        return;
+    }
+    const double theta = 2.0 * M_PI * c / N;
+    *x = cos(theta);
+    *y = sin(theta);
+}
+
+long long q_round(long double v, int frac_bits)
+{
+    return llroundl(ldexpl(v, frac_bits));
+}
+
+void destroy_cbset(fkv_cbset &s)
+{
+    cudaFree(s.cb32);
+    cudaFree(s.cnorm);
+    cudaFree(s.cb16);
+    cudaFree(s.escale);
+    s = fkv_cbset();
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *,
+                                  CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// Upload one K-or-V half of the codebooks: float32 copy, squared norms, the
+// fp16 hi/lo split (scaled per (group, stage) by a power of two) and its TMA map.
+int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
+{
+    fkv_cbset &s = ctx->cb[kv];
+    s.stages = stages;
+    const int G = ctx->Ly * ctx->H, D = ctx->D;
+    const size_t ncode = static_cast<size_t>(G) * stages * 256;
+    std::vector<float> cn(ncode);
+    std::vector<int> es(static_cast<size_t>(G) * stages);
+    std::vector<__half> c16(ncode * 2 * D);
+    for (int gs = 0; gs < G * stages; ++gs) {
+        const float *cb = host + static_cast<size_t>(gs) * 256 * D;
+        float m = 0.0f;
+        for (int i = 0; i < 256 * D; ++i) {
+            if (!isfinite(cb[i]))
+                return fail(ctx, FKV_EINVAL, "codebook holds a non-finite value");
+            m = fmaxf(m, fabsf(cb[i]));
+        }
+        int E = 0;
+        if (m > 0.0f)
+            frexpf(m, &E);
+        const int e = m > 0.0f ? E - 15 : 0;
+        es[gs] = e;
+        for (int j = 0; j < 256; ++j) {
+            double nn = 0.0;
+            for (int d = 0; d < D; ++d) {
+                const double v = cb[j * D + d];
+                nn += v * v;
+                const float sv = ldexpf(cb[j * D + d], -e);
+                const __half hi = __float2half_rn(sv);
+                const __half lo = __float2half_rn(sv - __half2float(hi));
+                c16[((static_cast<size_t>(gs) * 2 + 0) * 256 + j) * D + d] = hi;
+                c16[((static_cast<size_t>(gs) * 2 + 1) * 256 + j) * D + d] = lo;
+            }
+            cn[static_cast<size_t>(gs) * 256 + j] = static_cast<float>(nn);
+        }
+    }
+    CK(cudaMalloc(&s.cb32, ncode * D * sizeof(float)), "codebook alloc");
+    CK(cudaMalloc(&s.cnorm, ncode * sizeof(float)), "codebook alloc");
+    CK(cudaMalloc(&s.cb16, ncode * 2 * D * sizeof(__half)), "codebook alloc");
+    CK(cudaMalloc(&s.escale, es.size() * sizeof(int)), "codebook alloc");
+    CK(cudaMemcpy(s.cb32, host, ncode * D * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
+    CK(cudaMemcpy(s.cnorm, cn.data(), ncode * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
+    CK(cudaMemcpy(s.cb16, c16.data(), c16.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
+    CK(cudaMemcpy(s.escale, es.data(), es.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
+    EncodeTiledFn enc = encode_tiled();
+    if (!enc)
+        return fail(ctx, FKV_ECUDA, "cuTensorMapEncodeTiled unavailable");
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(ncode * 2)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(D) * sizeof(__half)};
+    const cuuint32_t box[2] = {64, 256};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&s.tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, s.cb16, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(ctx, FKV_ECUDA, "cuTensorMapEncodeTiled failed");
+    return FKV_OK;
+}
+
+bool check_cache(const fkv_ctx *ctx, const fkv_cache *c)
+{
+    if (!c || !c->data || c->batch <= 0 || c->seq <= 0)
+        return false;
+    if (c->dtype != FKV_F32 && c->dtype != FKV_F16 && c->dtype != FKV_BF16)
+        return false;
+    const int64_t esz = c->dtype == FKV_F32 ? 4 : 2;
+    // head vectors start on 16-byte boundaries (vector loads and stores)
+    if (reinterpret_cast<uintptr_t>(c->data) % 16)
+        return false;
+    const int64_t s[4] = {c->stride_layer, c->stride_batch, c->stride_head, c->stride_pos};
+    for (int i = 0; i < 4; ++i)
+        if (s[i] < 0 || (s[i] * esz) % 16)
+            return false;
+    (void)ctx;
+    return true;
+}
+
+cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
+
+}  // namespace
+
+extern "C" {
+
+double fkv_packing_ratio(int N)
+{
+    if (N < 3 || N > 256)
+        return 0.0;
+    double s = 0.0;
+    for (int k = 1; k <= N / 4; ++k) {
+        double x, y;
+        vertex(N, k, &x, &y);
+        s += x;
+    }
+    return 1.0 / (2.0 * (1.0 + s));
+}
+
+int fkv_max_span_len(double r)
+{
+    if (!(r > 0.0 && r <= 0.5))
+        return 0;
+    return static_cast<int>(floor(44.0 / log2(1.0 / r)));
+}
+
+int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx **out)
+{
+    if (!out)
+        return FKV_EINVAL;
+    *out = nullptr;
+    fkv_ctx *ctx = new fkv_ctx();
+    auto bail = [&](int code) {
+        fkv_destroy(ctx);
+        return code;
+    };
+    if (N < 3 || N > 256)
+        return bail(FKV_EINVAL);
+    const double rN = fkv_packing_ratio(N);
+    if (!(r > 0.0) || r > rN * (1.0 + 1e-12))
+        return bail(FKV_EINVAL);
+    const int Lmax = fkv_max_span_len(r);
+    if (span_len < 1 || span_len > Lmax || span_len > 44)
+        return bail(FKV_EINVAL);
+    ctx->N = N;
+    ctx->r = r;
+    ctx->L = span_len;
+    if (cudaGetDevice(&ctx->device) != cudaSuccess)
+        return bail(FKV_ECUDA);
+
+    // vertex table, padded to 256 entries with NaN (a symbol >= N poisons its span)
+    std::vector<double2> V(256, make_double2(nan(""), nan("")));
+    for (int c = 0; c < N; ++c)
+        vertex(N, c, &V[c].x, &V[c].y);
+    // Q1.62 decoder constants
+    fkv_decconst dec;
+    memset(&dec, 0, sizeof(dec));
+    for (int c = 0; c < N; ++c) {
+        const long double vx = V[c].x, vy = V[c].y;
+        dec.vx[c] = q_round(vx, 62);
+        dec.vy[c] = q_round(vy, 62);
+        dec.wx[c] = q_round((1.0L - static_cast<long double>(r)) * vx, 62);
+        dec.wy[c] = q_round((1.0L - static_cast<long double>(r)) * vy, 62);
+        dec.hn[c] = q_round((vx * vx + vy * vy) / 2.0L, 60);
+    }
+    int k = 62;
+    while (k > 1 && ldexpl(1.0L, k) / static_cast<long double>(r) >= ldexpl(1.0L, 63))
+        --k;
+    dec.rshift = k;
+    dec.rinv = llroundl(ldexpl(1.0L, k) / static_cast<long double>(r));
+    CK(cudaMalloc(&ctx->d_V, 256 * sizeof(double2)), "vertex alloc");
+    CK(cudaMemcpy(ctx->d_V, V.data(), 256 * sizeof(double2), cudaMemcpyHostToDevice), "vertex copy");
+    CK(cudaMalloc(&ctx->d_dec, sizeof(fkv_decconst)), "decoder alloc");
+    CK(cudaMemcpy(ctx->d_dec, &dec, sizeof(dec), cudaMemcpyHostToDevice), "decoder copy");
+    CK(cudaMalloc(&ctx->d_status, sizeof(unsigned)), "status alloc");
+    CK(cudaMemset(ctx->d_status, 0, sizeof(unsigned)), "status init");
+
+    if (cb) {
+        if (N != 256 || cb->n_layers < 1 || cb->n_heads < 1 || (cb->dim != 64 && cb->dim != 128) ||
+            cb->stages_k < 1 || cb->stages_k > 8 || cb->stages_v < 1 || cb->stages_v > 8 || !cb->k || !cb->v)
+            return bail(FKV_EINVAL);
+        if (cb->n_heads * (cb->stages_k + cb->stages_v) > 1024)
+            return bail(FKV_EINVAL);
+        ctx->has_cb = true;
+        ctx->Ly = cb->n_layers;
+        ctx->H = cb->n_heads;
+        ctx->D = cb->dim;
+        int rc = upload_cbset(ctx, 0, cb->k, cb->stages_k);
+        if (rc == FKV_OK)
+            rc = upload_cbset(ctx, 1, cb->v, cb->stages_v);
+        if (rc != FKV_OK)
+            return bail(rc);
+    }
+    *out = ctx;
+    return FKV_OK;
+}
+
+int fkv_destroy(fkv_ctx *ctx)
+{
+    if (!ctx)
+        return FKV_OK;
+    cudaDeviceSynchronize();
+    cudaFree(ctx->d_V);
+    cudaFree(ctx->d_dec);
+    cudaFree(ctx->d_status);
+    cudaFree(ctx->d_scratch);
+    destroy_cbset(ctx->cb[0]);
+    destroy_cbset(ctx->cb[1]);
+    delete ctx;
+    return FKV_OK;
+}
+
+int fkv_vertices(const fkv_ctx *ctx, double *out)
+{
+    if (!ctx || !out)
+        return FKV_EINVAL;
+    for (int c = 0; c < ctx->N; ++c)
+        vertex(ctx->N, c, &out[2 * c], &out[2 * c + 1]);
+    return FKV_OK;
+}
+
+int fkv_params(const fkv_ctx *ctx, int *N, double *r, int *span_len)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (N)
+        *N = ctx->N;
+    if (r)
+        *r = ctx->r;
+    if (span_len)
+        *span_len = ctx->L;
+    return FKV_OK;
+}
+
+const char *fkv_last_error(const fkv_ctx *ctx)
+{
+    return ctx ? ctx->err.c_str() : kNoCtx;
+}
+
+int fkv_sync_status(fkv_ctx *ctx, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    unsigned st = 0;
+    CK(cudaStreamSynchronize(as_stream(stream)), "stream sync");
+    CK(cudaMemcpy(&st, ctx->d_status, sizeof(st), cudaMemcpyDeviceToHost), "status read");
+    CK(cudaMemset(ctx->d_status, 0, sizeof(unsigned)), "status clear");
+    if (st & FKV_ST_TIMEOUT)
+        return fail(ctx, FKV_ETIMEOUT, "a device wait timed out");
+    if (st & FKV_ST_CORRUPT)
+        return fail(ctx, FKV_ECORRUPT, "corrupt point or symbol (anchor check failed)");
+    return FKV_OK;
+}
+
+int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int64_t n,
+                    int64_t sym_stride, double *pts_dev, int64_t pt_stride, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_streams < 0 || n < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (n_streams == 0 || n == 0)
+        return FKV_OK;
+    if (!sym_dev || !pts_dev || sym_stride < n || pt_stride < (n + ctx->L - 1) / ctx->L)
+        return fail(ctx, FKV_EINVAL, "bad pointer or stride");
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16)
+        return fail(ctx, FKV_EINVAL, "points must be 16-byte aligned");
+    CK(launch_span_encode(ctx, sym_dev, n_streams, n, sym_stride, pts_dev, pt_stride, as_stream(stream)),
+       "span encode launch");
+    return FKV_OK;
+}
+
+int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n,
+                    int64_t pt_stride, uint8_t *sym_dev, int64_t sym_stride, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_streams < 0 || n < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (n_streams == 0 || n == 0)
+        return FKV_OK;
+    if (!sym_dev || !pts_dev || sym_stride < n || pt_stride < (n + ctx->L - 1) / ctx->L)
+        return fail(ctx, FKV_EINVAL, "bad pointer or stride");
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16)
+        return fail(ctx, FKV_EINVAL, "points must be 16-byte aligned");
+    CK(launch_span_decode(ctx, pts_dev, n_streams, n, pt_stride, sym_dev, sym_stride, as_stream(stream)),
+       "span decode launch");
+    return FKV_OK;
+}
+
+int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
+             const int64_t *req_dev, int64_t n_req, uint8_t *out_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_req < 0 || n_streams < 0 || n < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (n_req == 0)
+        return FKV_OK;
+    if (!pts_dev || !req_dev || !out_dev || pt_stride < (n + ctx->L - 1) / ctx->L)
+        return fail(ctx, FKV_EINVAL, "bad pointer or stride");
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16 || reinterpret_cast<uintptr_t>(req_dev) % 8)
+        return fail(ctx, FKV_EINVAL, "misaligned buffer");
+    CK(launch_read(ctx, pts_dev, n_streams, n, pt_stride, req_dev, n_req, out_dev, as_stream(stream)),
+       "read launch");
+    return FKV_OK;
+}
+
+int fkv_record_len(const fkv_ctx *ctx)
+{
+    if (!ctx || !ctx->has_cb)
+        return 0;
+    return ctx->H * (ctx->cb[0].stages + ctx->cb[1].stages);
+}
+
+int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t t1, uint8_t *sym_dev,
+                   int64_t stream_stride, int64_t rec0, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb)
+        return fail(ctx, FKV_EINVAL, "context has no codebooks");
+    if (kv != 0 && kv != 1)
+        return fail(ctx, FKV_EINVAL, "kv must be 0 (keys) or 1 (values)");
+    if (!check_cache(ctx, x))
+        return fail(ctx, FKV_EINVAL, "bad cache view (dtype, alignment or strides)");
+    if (t0 < 0 || t1 < t0 || t1 > x->seq || rec0 < 0 || !sym_dev)
+        return fail(ctx, FKV_EINVAL, "bad position range");
+    if (t1 == t0)
+        return FKV_OK;
+    const int64_t R = fkv_record_len(ctx);
+    if (stream_stride < (rec0 + (t1 - t0)) * R)
+        return fail(ctx, FKV_EINVAL, "stream stride too small for the records");
+    CK(launch_rvq_encode(ctx, kv, x, t0, t1, sym_dev, stream_stride, rec0, as_stream(stream)),
+       "rvq encode launch");
+    return FKV_OK;
+}
+
+int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, int64_t n_rec,
+                   fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb)
+        return fail(ctx, FKV_EINVAL, "context has no codebooks");
+    if (!sym_dev || n_rec < 0 || t0 < 0)
+        return fail(ctx, FKV_EINVAL, "bad arguments");
+    const int64_t R = fkv_record_len(ctx);
+    if (stream_stride < n_rec * R)
+        return fail(ctx, FKV_EINVAL, "stream stride too small for the records");
+    fkv_cache *outs[2] = {k_out, v_out};
+    for (int kv = 0; kv < 2; ++kv) {
+        if (!outs[kv])
+            continue;
+        if (!check_cache(ctx, outs[kv]) || t0 + n_rec > outs[kv]->seq)
+            return fail(ctx, FKV_EINVAL, "bad output cache view");
+    }
+    if (n_rec == 0)
+        return FKV_OK;
+    for (int kv = 0; kv < 2; ++kv)
+        if (outs[kv])
+            CK(launch_rvq_decode(ctx, kv, sym_dev, stream_stride, n_rec, outs[kv], t0, as_stream(stream)),
+               "gather launch");
+    return FKV_OK;
+}
+
+int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride, fkv_cache *k_out,
+                  fkv_cache *v_out, int64_t t0, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb)
+        return fail(ctx, FKV_EINVAL, "context has no codebooks");
+    const fkv_cache *ref = k_out ? k_out : v_out;
+    if (!ref || !pts_dev || n_rec < 0)
+        return fail(ctx, FKV_EINVAL, "bad arguments");
+    if (k_out && v_out && k_out->batch != v_out->batch)
+        return fail(ctx, FKV_EINVAL, "K and V batch differ");
+    if (n_rec == 0)
+        return FKV_OK;
+    const int64_t R = fkv_record_len(ctx);
+    const int64_t n_streams = ref->batch * ctx->Ly;
+    const int64_t n = n_rec * R;
+    const size_t need = static_cast<size_t>(n_streams) * static_cast<size_t>(n);
+    if (need > ctx->scratch_bytes) {
+        CK(cudaStreamSynchronize(as_stream(stream)), "scratch sync");
+        cudaFree(ctx->d_scratch);
+        ctx->d_scratch = nullptr;
+        ctx->scratch_bytes = 0;
+        CK(cudaMalloc(&ctx->d_scratch, need), "scratch alloc");
+        ctx->scratch_bytes = need;
+    }
+    int rc = fkv_span_decode(ctx, pts_dev, n_streams, n, pt_stride, ctx->d_scratch, n, stream);
+    if (rc != FKV_OK)
+        return rc;
+    return fkv_rvq_decode(ctx, ctx->d_scratch, n, n_rec, k_out, v_out, t0, stream);
+}
+
+int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
+                const int64_t *req_dev, int64_t n_req, void *out_dev, int dtype, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb)
+        return fail(ctx, FKV_EINVAL, "context has no codebooks");
+    if (n_req < 0 || n_streams < 0 || n_rec < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (n_req == 0)
+        return FKV_OK;
+    if (!pts_dev || !req_dev || !out_dev || (dtype != FKV_F32 && dtype != FKV_F16 && dtype != FKV_BF16))
+        return fail(ctx, FKV_EINVAL, "bad arguments");
+    const int64_t R = fkv_record_len(ctx);
+    if (pt_stride < (n_rec * R + ctx->L - 1) / ctx->L)
+        return fail(ctx, FKV_EINVAL, "point stride too small");
+    if (reinterpret_cast<uintptr_t>(out_dev) % 16 || reinterpret_cast<uintptr_t>(pts_dev) % 16)
+        return fail(ctx, FKV_EINVAL, "misaligned buffer");
+    CK(launch_read_kv(ctx, pts_dev, n_streams, n_rec, pt_stride, req_dev, n_req, out_dev, dtype,
+                      as_stream(stream)),
+       "read_kv launch");
+    return FKV_OK;
+}
+
+int fkv_streams_create(fkv_ctx *ctx, int64_t n_streams, int64_t capacity_symbols, fkv_streams **out)
+{
+    if (!ctx || !out)
+        return FKV_EINVAL;
+    *out = nullptr;
+    if (n_streams < 1 || capacity_symbols < 0)
+        return fail(ctx, FKV_EINVAL, "bad stream-set size");
+    fkv_streams *s = new fkv_streams();
+    s->ctx = ctx;
+    s->n_streams = n_streams;
+    s->cap_spans = capacity_symbols / ctx->L + 1;
+    cudaError_t e = cudaMalloc(&s->d_pts, static_cast<size_t>(n_streams) * s->cap_spans * 16);
+    if (e != cudaSuccess) {
+        delete s;
+        return cuda_fail(ctx, e, "stream alloc");
+    }
+    *out = s;
+    return FKV_OK;
+}
+
+int fkv_streams_destroy(fkv_streams *s)
+{
+    if (!s)
+        return FKV_OK;
+    cudaDeviceSynchronize();
+    cudaFree(s->d_pts);
+    delete s;
+    return FKV_OK;
+}
+
+int fkv_streams_reset(fkv_streams *s)
+{
+    if (!s)
+        return FKV_EINVAL;
+    s->length = 0;
+    return FKV_OK;
+}
+
+int fkv_streams_info(const fkv_streams *s, int64_t *n_streams, int64_t *length, int64_t *pt_stride,
+                     double **pts_dev)
+{
+    if (!s)
+        return FKV_EINVAL;
+    if (n_streams)
+        *n_streams = s->n_streams;
+    if (length)
+        *length = s->length;
+    if (pt_stride)
+        *pt_stride = s->cap_spans;
+    if (pts_dev)
+        *pts_dev = s->d_pts;
+    return FKV_OK;
+}
+
+int fkv_append(fkv_ctx *ctx, fkv_streams *s, const uint8_t *sym_dev, int64_t m, int64_t sym_stride,
+               void *stream)
+{
+    if (!ctx || !s || s->ctx != ctx)
+        return fail(ctx, FKV_EINVAL, "bad stream set");
+    if (m < 0 || (m > 0 && (!sym_dev || sym_stride < m)))
+        return fail(ctx, FKV_EINVAL, "bad symbols");
+    if (m == 0)
+        return FKV_OK;
+    const int64_t n_new = s->length + m;
+    const int64_t need = (n_new + ctx->L - 1) / ctx->L;
+    if (need > s->cap_spans) {
+        int64_t cap = s->cap_spans * 2;
+        if (cap < need)
+            cap = need;
+        double *np = nullptr;
+        CK(cudaMalloc(&np, static_cast<size_t>(s->n_streams) * cap * 16), "stream grow");
+        const int64_t used = (s->length + ctx->L - 1) / ctx->L;
+        if (used > 0)
+            CK(cudaMemcpy2DAsync(np, cap * 16, s->d_pts, s->cap_spans * 16, used * 16, s->n_streams,
+                                 cudaMemcpyDeviceToDevice, as_stream(stream)),
+               "stream grow copy");
+        CK(cudaStreamSynchronize(as_stream(stream)), "stream grow sync");
+        cudaFree(s->d_pts);
+        s->d_pts = np;
+        s->cap_spans = cap;
+    }
+    CK(launch_append(ctx, s->d_pts, s->n_streams, s->cap_spans, s->length, sym_dev, m, sym_stride,
+                     as_stream(stream)),
+       "append launch");
+    s->length = n_new;
+    return FKV_OK;
+}
+
+int fkv_streams_export(const fkv_streams *s, int64_t *length, double *host_pts, void *stream)
+{
+    if (!s)
+        return FKV_EINVAL;
+    fkv_ctx *ctx = s->ctx;
+    const int64_t used = (s->length + ctx->L - 1) / ctx->L;
+    if (length)
+        *length = s->length;
+    if (host_pts && used > 0) {
+        CK(cudaMemcpy2DAsync(host_pts, used * 16, s->d_pts, s->cap_spans * 16, used * 16, s->n_streams,
+                             cudaMemcpyDeviceToHost, as_stream(stream)),
+           "export copy");
+        CK(cudaStreamSynchronize(as_stream(stream)), "export sync");
+    }
+    return FKV_OK;
+}
+
+int fkv_streams_import(fkv_ctx *ctx, int64_t n_streams, int64_t length, const double *host_pts,
+                       fkv_streams **out)
+{
+    if (!ctx || !out || length < 0 || (length > 0 && !host_pts))
+        return fail(ctx, FKV_EINVAL, "bad import arguments");
+    int rc = fkv_streams_create(ctx, n_streams, length, out);
+    if (rc != FKV_OK)
+        return rc;
+    fkv_streams *s = *out;
+    const int64_t used = (length + ctx->L - 1) / ctx->L;
+    if (used > 0) {
+        cudaError_t e = cudaMemcpy2D(s->d_pts, s->cap_spans * 16, host_pts, used * 16, used * 16, n_streams,
+                                     cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            fkv_streams_destroy(s);
+            *out = nullptr;
+            return cuda_fail(ctx, e, "import copy");
+        }
+    }
+    s->length = length;
+    return FKV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,230 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "fkv.h"
+
+// Device status bits (ctx->d_status); mapped to FKV_E* by fkv_sync_status.
+#define FKV_ST_CORRUPT 1u
+#define FKV_ST_TIMEOUT 2u
+
+// Codebook-side constants of one K-or-V half of the archive.
+struct fkv_cbset {
+    int stages = 0;
+    float *cb32 = nullptr;    // [Ly*H][S][256][D] float32 (gather, residual update)
+    float *cnorm = nullptr;   // [Ly*H][S][256] float32 squared norms
+    __half *cb16 = nullptr;   // [Ly*H][S][2][256][D] fp16 hi/lo split, scaled by 2^-e
+    int *escale = nullptr;    // [Ly*H][S] exponent e of the fp16 split
+    CUtensorMap tmap;         // TMA map over cb16 as [rows][D], box {64, 256}, 128B swizzle
+};
+
+// Decoder constants: everything in Q1.62 fixed point (value * 2^62).
+struct fkv_decconst {
+    long long vx[256], vy[256];    // V(c)
+    long long wx[256], wy[256];    // (1 - r) V(c)
+    long long hn[256];             // |V(c)|^2 / 2 in units of 2^-60
+    long long rinv;                // round(2^rshift / r)
+    int rshift;
+};
+
+struct fkv_ctx {
+    int N = 0;
+    double r = 0.0;
+    int L = 0;
+    int device = 0;
+    double2 *d_V = nullptr;        // [256] vertices, entries >= N are NaN
+    fkv_decconst *d_dec = nullptr; // decoder constants (device copy)
+    unsigned *d_status = nullptr;
+    // archive geometry and codebooks
+    bool has_cb = false;
+    int Ly = 0, H = 0, D = 0;
+    fkv_cbset cb[2];
+    uint8_t *d_scratch = nullptr;
+    size_t scratch_bytes = 0;
+    std::string err;
+};
+
+struct fkv_streams {
+    fkv_ctx *ctx = nullptr;
+    int64_t n_streams = 0;
+    int64_t length = 0;          // symbols per stream
+    int64_t cap_spans = 0;       // point stride
+    double *d_pts = nullptr;     // [n_streams][cap_spans][2]
+};
+
+// ---------------------------------------------------------------- launches
+// codec.cu
+cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_streams, int64_t n,
+                               int64_t sym_stride, double *pts, int64_t pt_stride, cudaStream_t st);
+cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                               int64_t pt_stride, uint8_t *sym, int64_t sym_stride, cudaStream_t st);
+cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                        int64_t pt_stride, const int64_t *req, int64_t n_req, uint8_t *out,
+                        cudaStream_t st);
+cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
+                          int64_t n_old, const uint8_t *sym, int64_t m, int64_t sym_stride,
+                          cudaStream_t st);
+// rvq.cu
+cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
+                              uint8_t *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
+// gather.cu
+cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int64_t stream_stride,
+                              int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st);
+cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
+                           int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
+                           int dtype, cudaStream_t st);
+
+// ------------------------------------------------------- device helpers
+#ifdef __CUDACC__
+namespace fkvd {
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Every device wait in the library gives up after this long and records
+// FKV_ST_TIMEOUT instead of spinning forever.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait on an mbarrier phase; false (and a status bit) on timeout.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned *status)
+{
+    if (mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity))
+            return true;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            atomicOr(status, FKV_ST_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// 2-D TMA tile load into shared memory, completion counted on `bar`.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int c0, int c1,
+                                            uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap *map)
+{
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// ---- tcgen05 (5th-generation tensor core, accumulators in tensor memory)
+__device__ __forceinline__ void tmem_alloc(uint32_t slot_smem, uint32_t ncols)
+{
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot_smem),
+                 "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
+{
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (fp16 or bf16 in, fp32 accumulate).
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on `bar` once every previously issued tcgen05.mma of this thread is done.
+__device__ __forceinline__ void umma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
+// layout (rows of 64 16-bit elements, 8-row / 1024-byte swizzle atoms).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);   // start address
+    d |= static_cast<uint64_t>(1) << 16;                    // leading byte offset (unused here)
+    d |= static_cast<uint64_t>(1024 >> 4) << 32;            // stride byte offset: 8 rows x 128 B
+    d |= static_cast<uint64_t>(1) << 46;                    // descriptor version (sm_100 family)
+    d |= static_cast<uint64_t>(2) << 61;                    // swizzle mode: 128 B
+    return d;
+}
+
+// Instruction descriptor, kind::f16: fp16 A and B (K-major), fp32 D, M x N.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N)
+{
+    return (1u << 4)                                   // D format: f32
+           | (0u << 7) | (0u << 10)                    // A, B format: f16
+           | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
+           | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+}
+
+}  // namespace fkvd
+#endif

@@ -20,6 +20,7 @@ log-normal channel scales of each configuration.
 from __future__ import annotations
 
 import dataclasses
+import functools
 import math
 from typing import Tuple
 
@@ -225,8 +226,10 @@ def kv_cache(cfg: KVConfig, kv: int) -> np.ndarray:
     return kv_elements(cfg, kv, l, b, h, t)
 
 
+@functools.lru_cache(maxsize=8)
 def codebooks(cfg: KVConfig, kv: int) -> np.ndarray:
-    """Synthetic per-head RVQ codebooks, float32 [Ly, H, S, 256, D].
+    """Synthetic per-head RVQ codebooks, float32 [Ly, H, S, 256, D] (memoised,
+    returned read-only).
 
     The paper trains them by k-means on KV from a disjoint span of the same
     text; here stage s draws 256 codewords from the data's own per-channel
@@ -241,7 +244,9 @@ def codebooks(cfg: KVConfig, kv: int) -> np.ndarray:
     z = irwin_hall(flat, TID_CB_K if kv == 0 else TID_CB_V, cfg.cfg_id)
     sig = channel_sigma(cfg, kv)[l, h, d] * (STAGE_SHRINK ** s)
     sc = (sig / IRWIN_HALL_STD).astype(np.float32)
-    return (z.astype(np.float32) * sc).astype(np.float32)
+    out = (z.astype(np.float32) * sc).astype(np.float32)
+    out.flags.writeable = False
+    return out
 
 
 # ----------------------------------------------------------- symbol streams --
@@ -270,3 +275,89 @@ def positions(n: int, count: int, stream: int, cfg_id: int = 2, salt: int = 0) -
     e = np.arange(count, dtype=np.uint64) + (np.uint64(stream) << np.uint64(40))
     w = uniform_u32(e, TID_POS + 64 * salt, cfg_id).astype(np.uint64)
     return ((w * np.uint64(n)) >> np.uint64(32)).astype(np.int64)
+
+
+# ------------------------------------------------- device-side generation --
+import ctypes as _ct
+import os as _os
+import subprocess as _sp
+import threading as _th
+
+_SYN_DIR = _os.path.dirname(_os.path.abspath(__file__))
+_SYN_SRC = _os.path.join(_SYN_DIR, "csrc", "synth_gen.cu")
+_SYN_LIB = _os.path.join(_SYN_DIR, "_build", "libsynth.so")
+_syn_lock = _th.Lock()
+_syn = None
+
+
+def build(force: bool = False) -> str:
+    """Compile csrc/synth_gen.cu into _build/libsynth.so (nvcc, sm_103a)."""
+    _os.makedirs(_os.path.dirname(_SYN_LIB), exist_ok=True)
+    if (not force and _os.path.exists(_SYN_LIB)
+            and _os.path.getmtime(_SYN_LIB) >= _os.path.getmtime(_SYN_SRC)):
+        return _SYN_LIB
+    tmp = _SYN_LIB + ".tmp%d" % _os.getpid()
+    nvcc = "/usr/local/cuda/bin/nvcc" if _os.path.exists("/usr/local/cuda/bin/nvcc") else "nvcc"
+    _sp.run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-Xcompiler", "-fPIC", "-shared",
+             _SYN_SRC, "-o", tmp], check=True)
+    _os.replace(tmp, _SYN_LIB)
+    return _SYN_LIB
+
+
+def _gpu():
+    global _syn
+    with _syn_lock:
+        if _syn is None:
+            L = _ct.CDLL(build())
+            i64, u32, u64, p = _ct.c_int64, _ct.c_uint32, _ct.c_uint64, _ct.c_void_p
+            L.synth_gen_kv.argtypes = [p, _ct.c_int, i64, i64, i64, i64, i64, u32, u32, u32, p, p]
+            L.synth_gen_symbols.argtypes = [p, i64, u64, u32, u32, _ct.c_int, p, u32, u32, p]
+            L.synth_gen_positions.argtypes = [p, i64, u64, u32, u64, u32, u32, i64, i64, p]
+            _syn = L
+        return _syn
+
+
+def gpu_kv_cache(cfg: KVConfig, kv: int, device="cuda", out=None):
+    """The cache [Ly, B, H, T, D] generated on the device (torch tensor),
+    element for element equal to kv_cache()/kv_elements()."""
+    import torch
+    tdt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[cfg.dtype]
+    if out is None:
+        out = torch.empty(cfg.cache_shape(), dtype=tdt, device=device)
+    scale = torch.from_numpy(channel_scale32(cfg, kv)).to(device)
+    k0, k1 = seed_key(cfg.cfg_id)
+    Ly, B, H, T, D = cfg.cache_shape()
+    rc = _gpu().synth_gen_kv(out.data_ptr(), {"f32": 0, "f16": 1, "bf16": 2}[cfg.dtype], Ly, B, H, T, D,
+                             TID_K if kv == 0 else TID_V, k0, k1, scale.data_ptr(),
+                             torch.cuda.current_stream().cuda_stream)
+    if rc != 0:
+        raise RuntimeError("synth_gen_kv failed (%d)" % rc)
+    torch.cuda.current_stream().synchronize()
+    return out
+
+
+def gpu_symbols(N: int, dist: str, n_streams: int, n: int, device="cuda", cfg_id: int = 2, first_stream: int = 0):
+    """uint8 [n_streams, n] symbol streams on the device, equal to symbols()."""
+    import torch
+    out = torch.empty((n_streams, n), dtype=torch.uint8, device=device)
+    thr = torch.from_numpy(zipf_thresholds(N).astype(np.uint32)).to(device)
+    k0, k1 = seed_key(cfg_id)
+    tid = TID_SYM + (0 if dist == "uniform" else 16) + 32 * N
+    for s in range(n_streams):
+        rc = _gpu().synth_gen_symbols(out[s].data_ptr(), n, first_stream + s, tid, N, int(dist == "zipf"),
+                                      thr.data_ptr(), k0, k1, torch.cuda.current_stream().cuda_stream)
+        if rc != 0:
+            raise RuntimeError("synth_gen_symbols failed (%d)" % rc)
+    return out
+
+
+def gpu_positions(n: int, count: int, stream: int, device="cuda", cfg_id: int = 2, salt: int = 0):
+    """int64 [count] positions on the device, equal to positions()."""
+    import torch
+    out = torch.empty(count, dtype=torch.int64, device=device)
+    k0, k1 = seed_key(cfg_id)
+    rc = _gpu().synth_gen_positions(out.data_ptr(), count, stream, TID_POS + 64 * salt, n, k0, k1, 1, 0,
+                                    torch.cuda.current_stream().cuda_stream)
+    if rc != 0:
+        raise RuntimeError("synth_gen_positions failed (%d)" % rc)
+    return out

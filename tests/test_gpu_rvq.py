@@ -1,0 +1,264 @@
+"""GPU parity of per-head residual VQ and the codebook gather (Sec. 3 "Setup").
+
+Criterion: every index must equal the oracle's wherever the oracle's top-2
+distance gap exceeds 1e-4 * ||residual||^2 (stage s compared only where the
+earlier stages agreed); closer ties are counted and reported.  Rebuilt K/V:
+float32 sums within 1e-3 of the oracle's float64 sums, and fp16/bf16 outputs
+equal to the oracle sum rounded to nearest-even except where the float32
+summation error bound straddles a rounding boundary."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+
+pytestmark = pytest.mark.gpu
+GAP = 1e-4
+TORCH_DT = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}
+
+
+@pytest.fixture(scope="module")
+def fkv():
+    import paper_2607_07144_gb300 as m
+    m.lib()
+    return m
+
+
+def compare_rvq(gpu, ora, gap):
+    """-> (hard mismatches, near-tie mismatches, compared entries)."""
+    n, S = ora.shape
+    prefix = np.ones(n, bool)
+    hard = near = seen = 0
+    for s in range(S):
+        diff = (gpu[:, s] != ora[:, s]) & prefix
+        h = diff & (gap[:, s] > GAP)
+        hard += int(h.sum())
+        near += int((diff & ~h).sum())
+        seen += int(prefix.sum())
+        prefix &= ~diff
+    return hard, near, seen
+
+
+def host_cache(cfg, kv):
+    a = synth.kv_cache(cfg, kv)
+    return synth.storage_to_f64(a, cfg.dtype)
+
+
+def to_device(cfg, a64):
+    t = torch.from_numpy(a64).to(TORCH_DT[cfg.dtype])
+    return t.cuda()
+
+
+def run_rvq(fkv, cfg, K, V, cbk, cbv, t0=None, t1=None):
+    ctx = fkv.Context(256, codebooks=(cbk, cbv))
+    t0 = cfg.t0 if t0 is None else t0
+    t1 = cfg.t1 if t1 is None else t1
+    R = ctx.record_len()
+    sym = torch.zeros((cfg.batch * cfg.n_layers, (t1 - t0) * R), dtype=torch.uint8, device="cuda")
+    ctx.rvq_encode(0, K, t0, t1, sym)
+    ctx.rvq_encode(1, V, t0, t1, sym)
+    assert ctx.sync_status() == 0
+    return ctx, sym
+
+
+def gpu_indices(oracle_mod, sym, cfg, P):
+    s = sym.cpu().numpy().reshape(cfg.batch, cfg.n_layers, P * cfg.record_len)
+    out = {}
+    for b in range(cfg.batch):
+        for l in range(cfg.n_layers):
+            out[b, l] = oracle_mod.indices_from_records(s[b, l], cfg.n_heads, cfg.stages_k, cfg.stages_v)
+    return out
+
+
+def check_config_full(fkv, oracle_mod, cfg):
+    K64, V64 = host_cache(cfg, 0), host_cache(cfg, 1)
+    cbk, cbv = synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)
+    ctx, sym = run_rvq(fkv, cfg, to_device(cfg, K64), to_device(cfg, V64), cbk, cbv)
+    P = cfg.n_archived
+    gi = gpu_indices(oracle_mod, sym, cfg, P)
+    tot_hard = tot_near = tot_seen = 0
+    for b in range(cfg.batch):
+        for l in range(cfg.n_layers):
+            ik, iv = gi[b, l]
+            for h in range(cfg.n_heads):
+                for kv, X, cb, gidx in ((0, K64, cbk, ik), (1, V64, cbv, iv)):
+                    x = X[l, b, h, cfg.t0:cfg.t1]
+                    oi, gap = oracle_mod.rvq_encode(x, cb[l, h])
+                    hard, near, seen = compare_rvq(gidx[h], oi, gap)
+                    tot_hard += hard
+                    tot_near += near
+                    tot_seen += seen
+    print("rvq %s: compared %d, near-tie mismatches %d" % (cfg.name, tot_seen, tot_near))
+    assert tot_hard == 0
+    return ctx, sym, gi, K64, V64, cbk, cbv
+
+
+def test_config0_full(fkv, oracle_mod):
+    cfg = synth.CFG0
+    ctx, sym, gi, K64, V64, cbk, cbv = check_config_full(fkv, oracle_mod, cfg)
+    # reconstruction in float32: within 1e-3 of the oracle's float64 sum
+    P = cfg.n_archived
+    Kr = torch.zeros(cfg.cache_shape(), dtype=torch.float32, device="cuda")
+    Vr = torch.zeros(cfg.cache_shape(), dtype=torch.float32, device="cuda")
+    ctx.rvq_decode(sym, P, Kr, Vr, t0=cfg.t0)
+    assert ctx.sync_status() == 0
+    Kr, Vr = Kr.cpu().numpy(), Vr.cpu().numpy()
+    ik, iv = gi[0, 0]
+    worst = 0.0
+    for h in range(cfg.n_heads):
+        yk = oracle_mod.rvq_decode(ik[h], cbk[0, h])
+        yv = oracle_mod.rvq_decode(iv[h], cbv[0, h])
+        worst = max(worst, np.abs(Kr[0, 0, h, cfg.t0:cfg.t1] - yk).max(), np.abs(Vr[0, 0, h, cfg.t0:cfg.t1] - yv).max())
+    assert worst <= 1e-3
+    assert np.all(Kr[0, 0, :, :cfg.t0] == 0) and np.all(Kr[0, 0, :, cfg.t1:] == 0)   # exact window untouched
+
+
+def _check_rounded(got, ref64, dtype, absum):
+    """got (rounded on the GPU from a float32 sum) must equal the oracle's
+    float64 sum rounded to nearest-even, except where the float32 summation
+    error bound (4 * 2^-24 * sum |c_s|, plus 1e-6 relative) straddles a
+    rounding boundary.  Returns the number of such borderline differences."""
+    want = synth_round(ref64, dtype)
+    ok = got == want
+    if ok.all():
+        return 0
+    eps = 4 * 2.0 ** -24 * absum + 1e-6 * np.abs(ref64)
+    borderline = synth_round(ref64 - eps, dtype) != synth_round(ref64 + eps, dtype)
+    bad = ~(ok | borderline)
+    assert not bad.any(), (int(bad.sum()), got[bad][:5], ref64[bad][:5])
+    return int((~ok).sum())
+
+
+def synth_round(y, dtype):
+    import oracle
+    return oracle.round_to(y, dtype)
+
+
+def test_small_gpt2_fp16_full(fkv, oracle_mod):
+    cfg = synth.small_config(synth.CFG1, 201, n_layers=2, batch=3, seq=36 + 300)
+    ctx, sym, gi, K64, V64, cbk, cbv = check_config_full(fkv, oracle_mod, cfg)
+    P = cfg.n_archived
+    Kr = torch.zeros(cfg.cache_shape(), dtype=torch.float16, device="cuda")
+    Vr = torch.zeros(cfg.cache_shape(), dtype=torch.float16, device="cuda")
+    ctx.rvq_decode(sym, P, Kr, Vr, t0=cfg.t0)
+    Kr = Kr.cpu().numpy().astype(np.float64)
+    Vr = Vr.cpu().numpy().astype(np.float64)
+    mid = 0
+    for (b, l), (ik, iv) in gi.items():
+        for h in range(cfg.n_heads):
+            mid += _check_rounded(Kr[l, b, h, cfg.t0:cfg.t1], oracle_mod.rvq_decode(ik[h], cbk[l, h]), "f16",
+                                  oracle_mod.rvq_decode(ik[h], np.abs(cbk[l, h])))
+            mid += _check_rounded(Vr[l, b, h, cfg.t0:cfg.t1], oracle_mod.rvq_decode(iv[h], cbv[l, h]), "f16",
+                                  oracle_mod.rvq_decode(iv[h], np.abs(cbv[l, h])))
+    print("fp16 midpoint cases:", mid)
+
+
+def test_small_llama_bf16_d128(fkv, oracle_mod):
+    cfg = synth.small_config(synth.CFG3, 203, n_layers=2, batch=2, seq=36 + 260)
+    ctx, sym, gi, K64, V64, cbk, cbv = check_config_full(fkv, oracle_mod, cfg)
+    P = cfg.n_archived
+    Kr = torch.zeros(cfg.cache_shape(), dtype=torch.bfloat16, device="cuda")
+    ctx.rvq_decode(sym, P, Kr, None, t0=cfg.t0)
+    Kr = Kr.float().cpu().numpy().astype(np.float64)
+    for (b, l), (ik, iv) in gi.items():
+        for h in range(cfg.n_heads):
+            _check_rounded(Kr[l, b, h, cfg.t0:cfg.t1], oracle_mod.rvq_decode(ik[h], cbk[l, h]), "bf16",
+                           oracle_mod.rvq_decode(ik[h], np.abs(cbk[l, h])))
+
+
+def _one_group_cfg(dim, dtype, seq):
+    return synth.KVConfig(900 + dim, "edge", 1, 1, 1, dim, seq, dtype, 2, 1, 0, 1.0, 0.0)
+
+
+@pytest.mark.parametrize("dim", [64, 128])
+def test_edge_vectors(fkv, oracle_mod, dim):
+    """Codeword-equal inputs, duplicate codewords (ties -> lowest index),
+    huge, tiny and zero vectors, partial tiles."""
+    rng = np.random.default_rng(dim)
+    cbk = rng.normal(size=(1, 1, 2, 256, dim)).astype(np.float32)
+    cbk[0, 0, 1] *= 0.5
+    cbk[0, 0, 0, 200] = cbk[0, 0, 0, 9]                  # duplicate codeword
+    cbv = rng.normal(size=(1, 1, 1, 256, dim)).astype(np.float32)
+    for n in [1, 127, 129, 300]:
+        x = rng.normal(size=(n, dim))
+        x[0] = cbk[0, 0, 0, 9]                            # equal to a (duplicated) codeword
+        if n > 5:
+            x[1] = cbk[0, 0, 0, 77]
+            x[2] *= 1e4
+            x[3] *= 1e-6
+            x[4] = 0.0
+            x[5] = cbk[0, 0, 0, 3] + cbk[0, 0, 1, 5]
+        cfg = _one_group_cfg(dim, "f32", n)
+        X = torch.from_numpy(x.astype(np.float32)).reshape(1, 1, 1, n, dim).cuda()
+        ctx, sym = run_rvq(fkv, cfg, X, X, cbk, cbv, t0=0, t1=n)
+        idx = sym.cpu().numpy().reshape(n, 3)
+        oi, gap = oracle_mod.rvq_encode(x.astype(np.float32).astype(np.float64), cbk[0, 0])
+        hard, near, seen = compare_rvq(idx[:, :2].astype(np.int32), oi, gap)
+        assert hard == 0, (n, hard)
+        assert idx[0, 0] == 9
+        if n > 5:
+            assert idx[1, 0] == 77 and idx[5, 0] == 3
+
+
+def test_strided_cache_view(fkv, oracle_mod):
+    """A non-contiguous view (layer dimension interleaved with an unused
+    buffer) gives the same symbols as the contiguous copy."""
+    cfg = synth.small_config(synth.CFG1, 205, n_layers=2, batch=2, seq=36 + 140)
+    K = to_device(cfg, host_cache(cfg, 0))
+    V = to_device(cfg, host_cache(cfg, 1))
+    big = torch.zeros((cfg.n_layers, 2) + cfg.cache_shape()[1:], dtype=K.dtype, device="cuda")
+    big[:, 1] = K
+    Ks = big[:, 1]
+    cbk, cbv = synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)
+    _, s1 = run_rvq(fkv, cfg, K, V, cbk, cbv)
+    _, s2 = run_rvq(fkv, cfg, Ks, V, cbk, cbv)
+    assert torch.equal(s1, s2)
+
+
+def _sampled_check(fkv, oracle_mod, cfg, n_sample):
+    K = synth.gpu_kv_cache(cfg, 0)
+    V = synth.gpu_kv_cache(cfg, 1)
+    cbk, cbv = synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)
+    ctx, sym = run_rvq(fkv, cfg, K, V, cbk, cbv)
+    R, P = cfg.record_len, cfg.n_archived
+    rng = np.random.default_rng(cfg.cfg_id)
+    l = rng.integers(0, cfg.n_layers, n_sample)
+    b = rng.integers(0, cfg.batch, n_sample)
+    h = rng.integers(0, cfg.n_heads, n_sample)
+    t = rng.integers(cfg.t0, cfg.t1, n_sample)
+    symh = sym.view(cfg.batch, cfg.n_layers, P, R)
+    hard_total = near_total = 0
+    for kv, X, cb, S, off in ((0, K, cbk, cfg.stages_k, 0), (1, V, cbv, cfg.stages_v, cfg.n_heads * cfg.stages_k)):
+        xs = synth.storage_to_f64(synth.kv_elements(cfg, kv, l, b, h, t), cfg.dtype)
+        dev = X[torch.from_numpy(l).cuda(), torch.from_numpy(b).cuda(), torch.from_numpy(h).cuda(),
+                torch.from_numpy(t).cuda()].float().cpu().numpy().astype(np.float64)
+        assert np.array_equal(xs, dev)                  # device generator == host twin
+        g = np.empty((n_sample, S), np.int32)
+        sl = symh[torch.from_numpy(b).cuda(), torch.from_numpy(l).cuda(), torch.from_numpy(t - cfg.t0).cuda()]
+        sl = sl.cpu().numpy()
+        for i in range(n_sample):
+            g[i] = sl[i, off + h[i] * S: off + (h[i] + 1) * S]
+        oi = np.empty((n_sample, S), np.int32)
+        gap = np.empty((n_sample, S))
+        for grp in set(zip(l.tolist(), h.tolist())):
+            sel = (l == grp[0]) & (h == grp[1])
+            oi[sel], gap[sel] = oracle_mod.rvq_encode(xs[sel], cb[grp[0], grp[1]])
+        hard, near, seen = compare_rvq(g, oi, gap)
+        hard_total += hard
+        near_total += near
+    print("%s sampled %d vectors: near-tie mismatches %d" % (cfg.name, n_sample, near_total))
+    assert hard_total == 0
+    return ctx, sym, K, V
+
+
+def test_config1_full_size_sampled(fkv, oracle_mod):
+    _sampled_check(fkv, oracle_mod, synth.CFG1, 4000)
+
+
+def test_config3_full_size_sampled(fkv, oracle_mod):
+    free, total = torch.cuda.mem_get_info()
+    if free < 48e9:
+        pytest.skip("needs ~40 GB of device memory")
+    ctx, sym, K, V = _sampled_check(fkv, oracle_mod, synth.CFG3, 3000)
+    del K, V, sym
+    torch.cuda.empty_cache()
