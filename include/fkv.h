@@ -198,6 +198,23 @@ int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, 
 int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
                   fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
 
+/* Allocation-free variant of fkv_decode_kv (the paper has no counterpart;
+ * it exists for callers that must not allocate device memory, such as a
+ * serving loop whose device memory belongs to its own pool allocator, or a
+ * decode step that cannot take the implicit synchronisation of cudaMalloc).
+ * Same arguments, layouts and results as fkv_decode_kv, but the decoded
+ * symbols go through a 16 MiB scratch array compiled into the library
+ * instead of a context-owned buffer: it calls no cudaMalloc or cudaFree.
+ * Limit: batch * n_layers * n_rec * fkv_record_len(ctx) <= 16 MiB, else
+ * FKV_EINVAL with nothing launched (decode fewer sequences per call).  The
+ * first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture.  All calls share the array and it keeps the previous call's
+ * contents, so calls that can overlap on the GPU race and must be ordered by
+ * the caller. */
+int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
+                         fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
+
 /* Sec. 2 random access at record granularity: for each request q,
  * req_dev[2q] = stream (b * n_layers + l), req_dev[2q + 1] = record index,
  * decode only the spans of that record and write its K and V head vectors to

@@ -60,6 +60,7 @@ SIGNATURES = {
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
     "fkv_decode_kv": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
+    "fkv_decode_kv_static": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
     "fkv_read_kv": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _I, _P]),
     "fkv_streams_create": (_I, [_P, _I64, _I64, ctypes.POINTER(_P)]),
     "fkv_streams_destroy": (_I, [_P]),
@@ -236,6 +237,17 @@ class Context:
         self._check(lib().fkv_decode_kv(self._h, _ptr(pts), n_rec, _rows(pts, 2),
                                         ctypes.byref(ck) if ck else None, ctypes.byref(cv) if cv else None,
                                         t0, _stream(stream)))
+
+    def decode_kv_static(self, pts: torch.Tensor, n_rec: int, k_out: torch.Tensor = None,
+                         v_out: torch.Tensor = None, t0: int = 0, stream=None):
+        """decode_kv without any device allocation: the decoded symbols go
+        through the library's fixed 16 MiB scratch array (for callers whose
+        device memory must all come from their own allocator)."""
+        ck = cache_view(k_out) if k_out is not None else None
+        cv = cache_view(v_out) if v_out is not None else None
+        self._check(lib().fkv_decode_kv_static(self._h, _ptr(pts), n_rec, _rows(pts, 2),
+                                               ctypes.byref(ck) if ck else None, ctypes.byref(cv) if cv else None,
+                                               t0, _stream(stream)))
 
     def read_kv(self, pts: torch.Tensor, n_rec: int, req: torch.Tensor, out: torch.Tensor, stream=None):
         """req int64 [n_req, 2] = (stream, record) -> out [n_req, 2, heads, dim]."""

@@ -1,0 +1,131 @@
+// fkv_decode_kv_static: the full archive read of fkv_decode_kv, for callers
+// that must not allocate device memory.
+//
+// fkv_decode_kv keeps the decoded symbols between its two kernels in a
+// context-owned buffer that it (re)allocates with cudaMalloc when an archive
+// is larger than any seen before -- a call that also synchronises the stream.
+// Some callers cannot accept that: a serving loop whose device memory all
+// belongs to its own pool allocator (memory taken behind the pool's back can
+// make the pool's later requests fail), or a latency-critical decode step that
+// may not stall on an implicit device-wide synchronisation.  This entry point
+// uses instead a fixed scratch array compiled into the library, so it never
+// calls cudaMalloc, cudaFree or any allocating routine.
+//
+// The array lives for the life of the process on every GPU that loads this
+// library and holds kStaticScratchBytes (16 MiB) of decoded symbols: at most
+// batch * n_layers * n_rec * R bytes per call (R = fkv_record_len).  Every
+// call shares it, so calls whose kernels overlap on the GPU (different
+// streams without ordering) race on it and must be serialised by the caller.
+// It keeps whatever the previous call left; nothing here needs it zeroed,
+// because the decode kernel overwrites every byte the gather then reads.
+#include <mutex>
+
+#include "fkv_internal.h"
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = 16u << 20;
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_lock;
+void *g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device (looked up once
+// per device with that device current).  In host code the symbol itself is a
+// host-side stand-in and must never be handed to a kernel.
+int scratch_address(fkv_ctx *ctx, uint8_t **out)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        ctx->err = std::string("static scratch: cudaGetDevice: ") + cudaGetErrorString(e);
+        return FKV_ECUDA;
+    }
+    if (dev < 0 || dev >= kMaxDevices) {
+        ctx->err = "static scratch: device index out of range";
+        return FKV_EINVAL;
+    }
+    std::lock_guard<std::mutex> g(g_lock);
+    if (!g_scratch_addr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_scratch);
+        if (e != cudaSuccess || !p) {
+            ctx->err = std::string("static scratch: cudaGetSymbolAddress: ") + cudaGetErrorString(e);
+            return FKV_ECUDA;
+        }
+        g_scratch_addr[dev] = p;
+    }
+    *out = static_cast<uint8_t *>(g_scratch_addr[dev]);
+    return FKV_OK;
+}
+
+}  // namespace
+
+extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
+                                    fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb) {
+        ctx->err = "context has no codebooks";
+        return FKV_EINVAL;
+    }
+    const fkv_cache *ref = k_out ? k_out : v_out;
+    if (!ref || !pts_dev || n_rec < 0 || t0 < 0) {
+        ctx->err = "bad arguments";
+        return FKV_EINVAL;
+    }
+    if (k_out && v_out && k_out->batch != v_out->batch) {
+        ctx->err = "K and V batch differ";
+        return FKV_EINVAL;
+    }
+    if (n_rec == 0)
+        return FKV_OK;
+    const int64_t R = fkv_record_len(ctx);
+    const int64_t n_streams = ref->batch * ctx->Ly;
+    const int64_t n = n_rec * R;
+    if (n_streams <= 0 || n > static_cast<int64_t>(kStaticScratchBytes) / n_streams) {
+        ctx->err = "fkv_decode_kv_static: batch * n_layers * n_rec * record_len exceeds the 16 MiB static "
+                   "scratch; decode fewer sequences per call";
+        return FKV_EINVAL;
+    }
+    if (pt_stride < (n + ctx->L - 1) / ctx->L) {
+        ctx->err = "point stride too small";
+        return FKV_EINVAL;
+    }
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16) {
+        ctx->err = "points must be 16-byte aligned";
+        return FKV_EINVAL;
+    }
+    // output views are checked before anything is launched
+    const fkv_cache *outs[2] = {k_out, v_out};
+    for (const fkv_cache *c : outs) {
+        if (!c)
+            continue;
+        const bool dt = c->dtype == FKV_F32 || c->dtype == FKV_F16 || c->dtype == FKV_BF16;
+        const int64_t esz = c->dtype == FKV_F32 ? 4 : 2;
+        const int64_t s4[4] = {c->stride_layer, c->stride_batch, c->stride_head, c->stride_pos};
+        bool ok = dt && c->data && c->batch > 0 && t0 + n_rec <= c->seq &&
+                  reinterpret_cast<uintptr_t>(c->data) % 16 == 0;
+        for (int i = 0; i < 4 && ok; ++i)
+            ok = s4[i] >= 0 && (s4[i] * esz) % 16 == 0;
+        if (!ok) {
+            ctx->err = "bad output cache view";
+            return FKV_EINVAL;
+        }
+    }
+    uint8_t *scratch = nullptr;
+    int rc = scratch_address(ctx, &scratch);
+    if (rc != FKV_OK)
+        return rc;
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_span_decode(ctx, pts_dev, n_streams, n, pt_stride, scratch, n, st);
+    if (e != cudaSuccess) {
+        ctx->err = std::string("static decode launch: ") + cudaGetErrorString(e);
+        return FKV_ECUDA;
+    }
+    // the gather with the same checks as fkv_rvq_decode, reading the static scratch
+    return fkv_rvq_decode(ctx, scratch, n, n_rec, k_out, v_out, t0, stream);
+}
