@@ -7,10 +7,9 @@
 // d = p - V(c); t = r * d; p = V(c) + t per coordinate.
 //
 // Decoding only has to recover the symbols, so it runs in exact 64-bit
-// fixed point (Q1.62) on the integer pipes: the nearest vertex is found from
-// exact dot products, and p <- (p - (1-r) V(c)) / r becomes a subtraction and
-// a 64x64->128-bit multiply by a fixed-point 1/r.
-#include "fkv_internal.h"
+// fixed point (Q1.62) on the integer pipes with no division at all (see
+// decode_core.cuh).
+#include "decode_core.cuh"
 
 namespace {
 
@@ -101,110 +100,23 @@ k_span_encode(const uint8_t *__restrict__ sym, int64_t n, int64_t sym_stride, in
 }
 
 // ------------------------------------------------------------- decoding
-struct DecShared {
-    long long vx[256], vy[256], wx[256], wy[256], hn[256];
-};
+// (arithmetic in decode_core.cuh: exact Q1.62 walk, no division)
 
-__device__ __forceinline__ void load_dec(DecShared &d, const fkv_decconst *__restrict__ g)
+__host__ __device__ inline int tables_bytes(int N, int L)
 {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
-        d.vx[i] = g->vx[i];
-        d.vy[i] = g->vy[i];
-        d.wx[i] = g->wx[i];
-        d.wy[i] = g->wy[i];
-        d.hn[i] = g->hn[i];
-    }
-}
-
-__device__ __forceinline__ long long to_q62(double v)
-{
-    return __double2ll_rn(v * 4611686018427387904.0);   // v * 2^62, exact scaling
-}
-
-// Nearest vertex of (X, Y): argmax of p.V(c) - |V(c)|^2 / 2 (units 2^-60).
-__device__ __forceinline__ long long vscore(const DecShared &d, long long X, long long Y, int c)
-{
-    return __mul64hi(X, d.vx[c]) + __mul64hi(Y, d.vy[c]) - d.hn[c];
-}
-
-__device__ __forceinline__ int classify(const DecShared &d, long long X, long long Y, int N)
-{
-    if (N <= 8) {
-        int best = 0;
-        long long bs = vscore(d, X, Y, 0);
-        for (int c = 1; c < N; ++c) {
-            const long long s = vscore(d, X, Y, c);
-            if (s > bs) {
-                bs = s;
-                best = c;
-            }
-        }
-        return best;
-    }
-    // Voronoi regions of the vertices are the angular sectors around them, so
-    // the angle picks the sector up to one neighbour; the exact dot products
-    // then decide between the three candidates.
-    const float xf = static_cast<float>(static_cast<int>(X >> 32));
-    const float yf = static_cast<float>(static_cast<int>(Y >> 32));
-    const float a = atan2f(yf, xf) * (static_cast<float>(N) * 0.15915494309189535f);
-    int c0 = __float2int_rn(a);
-    if (c0 < 0)
-        c0 += N;
-    if (c0 >= N)
-        c0 -= N;
-    const int cm = c0 == 0 ? N - 1 : c0 - 1;
-    const int cp = c0 == N - 1 ? 0 : c0 + 1;
-    int best = c0;
-    long long bs = vscore(d, X, Y, c0);
-    long long s = vscore(d, X, Y, cm);
-    if (s > bs) {
-        bs = s;
-        best = cm;
-    }
-    s = vscore(d, X, Y, cp);
-    if (s > bs)
-        best = cp;
-    return best;
-}
-
-// (v * rinv) >> k with a 128-bit intermediate product, 1 <= k <= 63.
-__device__ __forceinline__ long long mulshift(long long v, long long rinv, int k)
-{
-    const unsigned long long lo = static_cast<unsigned long long>(v) * static_cast<unsigned long long>(rinv);
-    const long long hi = __mul64hi(v, rinv);
-    return static_cast<long long>((lo >> k) | (static_cast<unsigned long long>(hi) << (64 - k)));
-}
-
-// One backward step of Sec. 1: classify, then p <- (p - (1-r) V(c)) / r.
-__device__ __forceinline__ int decode_step(const DecShared &d, long long &X, long long &Y, int N,
-                                           long long rinv, int rsh)
-{
-    const int c = classify(d, X, Y, N);
-    X = mulshift(static_cast<long long>(static_cast<unsigned long long>(X) - static_cast<unsigned long long>(d.wx[c])), rinv, rsh);
-    Y = mulshift(static_cast<long long>(static_cast<unsigned long long>(Y) - static_cast<unsigned long long>(d.wy[c])), rinv, rsh);
-    return c;
-}
-
-// Anchor check: after a span's first symbol the point is back at (0, 0);
-// a residual above 2^-4 (2^58 in Q62) flags a corrupt point.
-__device__ __forceinline__ bool anchor_ok(long long X, long long Y)
-{
-    const long long lim = 1ll << 58;
-    return X <= lim && X >= -lim && Y <= lim && Y >= -lim;
+    return (fkvdec::smem_bytes(N, L) + 15) & ~15;
 }
 
 __global__ void __launch_bounds__(kThreads)
 k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
-              uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc, int N,
-              int L, unsigned *status)
+              uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
+              const longlong2 *__restrict__ T, int N, int L, unsigned *status)
 {
-    __shared__ __align__(16) uint8_t sbuf[kStageBytes];
-    __shared__ DecShared sd;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    uint8_t *sbuf = dsm + tables_bytes(N, L);
     const int64_t stream = blockIdx.x / bps;
     const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
-    load_dec(sd, dc);
-    const long long rinv = dc->rinv;
-    const int rsh = dc->rshift;
     const int64_t b = s0 * L;
     const int64_t e = min(n, (s0 + kThreads) * L);
     uint8_t *dst = sym + stream * sym_stride + b;
@@ -214,27 +126,26 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
     if (s < spans) {
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
         const double2 p = pts[stream * pt_stride + s];
-        long long X = to_q62(p.x), Y = to_q62(p.y);
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
         uint8_t *my = sbuf + off + threadIdx.x * L;
-        for (int k = m - 1; k >= 0; --k)
-            my[k] = static_cast<uint8_t>(decode_step(sd, X, Y, N, rinv, rsh));
-        if (!anchor_ok(X, Y))
+        fkvdec::walk(t, X, Y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<uint8_t>(c); });
+        const long long lim = __ldg(&dc->alim[m]);
+        if (X > lim || X < -lim || Y > lim || Y < -lim)
             atomicOr(status, FKV_ST_CORRUPT);
     }
     __syncthreads();
     stage_out(dst, sbuf, static_cast<int>(e - b), off);
 }
 
-// Sec. 2 random access: one request per thread, decoding only its span.
+// Sec. 2 random access: one request per thread, decoding only its span down
+// to the requested offset.
 __global__ void __launch_bounds__(kThreads)
 k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride,
        const int64_t *__restrict__ req, int64_t n_req, uint8_t *__restrict__ out,
-       const fkv_decconst *__restrict__ dc, int N, int L, unsigned *status)
+       const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L, unsigned *status)
 {
-    __shared__ DecShared sd;
-    load_dec(sd, dc);
-    const long long rinv = dc->rinv;
-    const int rsh = dc->rshift;
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
     __syncthreads();
     const int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
     if (q >= n_req)
@@ -249,11 +160,10 @@ k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt
     const int o = static_cast<int>(pos - u * L);
     const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
     const double2 p = pts[st * pt_stride + u];
-    long long X = to_q62(p.x), Y = to_q62(p.y);
-    int c = 0;
-    for (int k = m - 1; k >= o; --k)
-        c = decode_step(sd, X, Y, N, rinv, rsh);
-    out[q] = static_cast<uint8_t>(c);
+    long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+    int sym = 0;
+    fkvdec::walk(t, X, Y, m - o, [&](int j, int c) { sym = c; });
+    out[q] = static_cast<uint8_t>(sym);
 }
 
 // Sec. 2 append: one thread per (stream, span touched by the new symbols).
@@ -319,9 +229,13 @@ cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_st
         return cudaSuccess;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    k_span_decode<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+    const int smem = tables_bytes(c->N, c->L) + kStageBytes;
+    cudaError_t e = cudaFuncSetAttribute(k_span_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    k_span_decode<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
         reinterpret_cast<const double2 *>(pts), n, pt_stride, spans, static_cast<int>(bps), sym,
-        sym_stride, c->d_dec, c->N, c->L, c->d_status);
+        sym_stride, c->d_dec, c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 
@@ -334,9 +248,13 @@ cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, 
         return cudaSuccess;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    k_read<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
-        reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride, req, n_req, out, c->d_dec, c->N,
-        c->L, c->d_status);
+    const int smem = tables_bytes(c->N, c->L);
+    cudaError_t e = cudaFuncSetAttribute(k_read, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    k_read<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
+        reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride, req, n_req, out, c->d_dec, c->d_T,
+        c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 

@@ -1,0 +1,151 @@
+// Span decoding core shared by the bulk decoder, the random reads and the
+// record reads (Sec. 1 "The code": the symbol is the cell holding the point,
+// then p_{k-1} = (p_k - (1-r) V(c_k)) / r).
+//
+// The decoder never divides.  With m the span length and Q_k = r^(m-k) p_k,
+//     Q_m = stored point,   Q_{k-1} = Q_k - (1-r) r^(m-k) V(c_k),
+// and Q_0 = r^m p_0 must be back at the anchor (the origin).  Nearest-vertex
+// classification of p_k (= cell containment for r <= r_N) is the argmax over
+// c of p_k . V(c) because every vertex lies on the unit circle, and that is
+// scale-free: argmax_c Q_k . V(c).  The margin of the true point to a cell
+// boundary is about r^m in Q space at every step, so Q is kept in exact
+// Q1.62 fixed point (int64, units of 2^-62) and the step is one table load
+// of T[j][c] = round((1-r) r^j V(c) 2^62), j = m - k, and two subtractions.
+//
+// Classification takes an fp32 fast path with a certified margin and falls
+// back to exact 64x64->128-bit dot products in the rare near-boundary case:
+//   * N = 4: the vertices are the axis directions, exact integer compares;
+//   * N <= 8: fp32 scores q . V(c); exact scores when the best two are closer
+//     than a bound far above the fp32 error;
+//   * N > 8: Voronoi regions of the vertices are angular sectors, so the fp32
+//     angle picks the sector; within 1e-3 sector widths of a boundary the two
+//     neighbouring sectors are decided by the exact sign of Q . (V(a) - V(b)).
+#pragma once
+
+#include "fkv_internal.h"
+
+namespace fkvdec {
+
+struct Tables {
+    const longlong2 *T;   // [L][N] (x, y), shared memory
+    const long long *vx;  // [N] V(c) in Q1.62, shared memory
+    const long long *vy;
+    const float2 *vf;     // [N] V(c) as float, shared memory
+    int N;
+};
+
+// Shared-memory footprint of the tables for (N, L).
+__host__ __device__ inline int smem_bytes(int N, int L)
+{
+    return L * N * 16 + N * 16 + N * 8;
+}
+
+// Block-cooperative copy of the tables into `sm` (16-byte aligned).
+__device__ inline Tables load(const fkv_decconst *__restrict__ g, const longlong2 *__restrict__ Tg, int N, int L,
+                              uint8_t *sm)
+{
+    longlong2 *T = reinterpret_cast<longlong2 *>(sm);
+    long long *vx = reinterpret_cast<long long *>(sm + L * N * 16);
+    long long *vy = vx + N;
+    float2 *vf = reinterpret_cast<float2 *>(sm + L * N * 16 + N * 16);
+    for (int i = threadIdx.x; i < L * N; i += blockDim.x)
+        T[i] = Tg[i];
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        vx[i] = g->vx[i];
+        vy[i] = g->vy[i];
+        vf[i] = make_float2(g->vfx[i], g->vfy[i]);
+    }
+    return Tables{T, vx, vy, vf, N};
+}
+
+__device__ __forceinline__ long long exact_dot(const Tables &t, long long X, long long Y, int c)
+{
+    return __mul64hi(X, t.vx[c]) + __mul64hi(Y, t.vy[c]);
+}
+
+static __device__ __noinline__ int classify_exact_all(const Tables &t, long long X, long long Y)
+{
+    int best = 0;
+    long long bs = exact_dot(t, X, Y, 0);
+    for (int c = 1; c < t.N; ++c) {
+        const long long s = exact_dot(t, X, Y, c);
+        if (s > bs) {
+            bs = s;
+            best = c;
+        }
+    }
+    return best;
+}
+
+__device__ __forceinline__ int classify(const Tables &t, long long X, long long Y)
+{
+    const int N = t.N;
+    if (N == 4) {
+        const long long ax = X < 0 ? -X : X, ay = Y < 0 ? -Y : Y;
+        if (ax >= ay)
+            return X >= 0 ? 0 : 2;
+        return Y >= 0 ? 1 : 3;
+    }
+    const float qx = __ll2float_rn(X), qy = __ll2float_rn(Y);
+    if (N <= 8) {
+        float b1 = -INFINITY, b2 = -INFINITY;
+        int bi = 0;
+        for (int c = 0; c < N; ++c) {
+            const float s = fmaf(qx, t.vf[c].x, qy * t.vf[c].y);
+            if (s > b1) {
+                b2 = b1;
+                b1 = s;
+                bi = c;
+            } else if (s > b2) {
+                b2 = s;
+            }
+        }
+        if (b1 - b2 > 0x1p-18f * (fabsf(qx) + fabsf(qy)))
+            return bi;
+        return classify_exact_all(t, X, Y);
+    }
+    const float a = atan2f(qy, qx) * (static_cast<float>(N) * 0.15915494309189535f);
+    const float ar = rintf(a);
+    const float f = a - ar;                        // in [-0.5, 0.5]
+    int c0 = static_cast<int>(ar);
+    if (c0 < 0)
+        c0 += N;
+    if (c0 >= N)
+        c0 -= N;
+    if (fabsf(f) < 0.499f)
+        return c0;
+    int c1 = f > 0.0f ? c0 + 1 : c0 - 1;           // the neighbour across the near boundary
+    if (c1 < 0)
+        c1 += N;
+    if (c1 >= N)
+        c1 -= N;
+    const long long d = exact_dot(t, X, Y, c0) - exact_dot(t, X, Y, c1);
+    if (d > 0)
+        return c0;
+    if (d < 0)
+        return c1;
+    return c0 < c1 ? c0 : c1;
+}
+
+__device__ __forceinline__ long long to_q62(double v)
+{
+    return __double2ll_rn(v * 4611686018427387904.0);   // v * 2^62, exact scaling
+}
+
+// Decode `steps` symbols backward from Q (the span's stored point in Q1.62):
+// step j = 0 .. steps-1 emits the symbol at offset m-1-j of the span.
+// `emit(j, c)` receives each symbol.
+template <class Emit>
+__device__ __forceinline__ void walk(const Tables &t, long long &X, long long &Y, int steps, Emit emit)
+{
+    const int N = t.N;
+    for (int j = 0; j < steps; ++j) {
+        const int c = classify(t, X, Y);
+        emit(j, c);
+        const longlong2 w = t.T[j * N + c];
+        X = static_cast<long long>(static_cast<unsigned long long>(X) - static_cast<unsigned long long>(w.x));
+        Y = static_cast<long long>(static_cast<unsigned long long>(Y) - static_cast<unsigned long long>(w.y));
+    }
+}
+
+}  // namespace fkvdec

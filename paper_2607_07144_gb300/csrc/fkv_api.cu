@@ -219,26 +219,37 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
     std::vector<double2> V(256, make_double2(nan(""), nan("")));
     for (int c = 0; c < N; ++c)
         vertex(N, c, &V[c].x, &V[c].y);
-    // Q1.62 decoder constants
+    // decoder constants: vertices in Q1.62 and float, the step table
+    // T[j][c] = (1 - r) r^j V(c) in Q1.62, and the anchor limits 2^-4 r^m
     fkv_decconst dec;
     memset(&dec, 0, sizeof(dec));
+    std::vector<longlong2> T(static_cast<size_t>(span_len) * N);
     for (int c = 0; c < N; ++c) {
-        const long double vx = V[c].x, vy = V[c].y;
-        dec.vx[c] = q_round(vx, 62);
-        dec.vy[c] = q_round(vy, 62);
-        dec.wx[c] = q_round((1.0L - static_cast<long double>(r)) * vx, 62);
-        dec.wy[c] = q_round((1.0L - static_cast<long double>(r)) * vy, 62);
-        dec.hn[c] = q_round((vx * vx + vy * vy) / 2.0L, 60);
+        dec.vx[c] = q_round(V[c].x, 62);
+        dec.vy[c] = q_round(V[c].y, 62);
+        dec.vfx[c] = static_cast<float>(V[c].x);
+        dec.vfy[c] = static_cast<float>(V[c].y);
     }
-    int k = 62;
-    while (k > 1 && ldexpl(1.0L, k) / static_cast<long double>(r) >= ldexpl(1.0L, 63))
-        --k;
-    dec.rshift = k;
-    dec.rinv = llroundl(ldexpl(1.0L, k) / static_cast<long double>(r));
+    long double rj = 1.0L;
+    for (int j = 0; j < span_len; ++j) {
+        const long double coef = (1.0L - static_cast<long double>(r)) * rj;
+        for (int c = 0; c < N; ++c) {
+            T[static_cast<size_t>(j) * N + c].x = q_round(coef * V[c].x, 62);
+            T[static_cast<size_t>(j) * N + c].y = q_round(coef * V[c].y, 62);
+        }
+        rj *= static_cast<long double>(r);
+    }
+    rj = 1.0L;
+    for (int m = 0; m < 48; ++m) {
+        dec.alim[m] = q_round(0.0625L * rj, 62);
+        rj *= static_cast<long double>(r);
+    }
     CK(cudaMalloc(&ctx->d_V, 256 * sizeof(double2)), "vertex alloc");
     CK(cudaMemcpy(ctx->d_V, V.data(), 256 * sizeof(double2), cudaMemcpyHostToDevice), "vertex copy");
     CK(cudaMalloc(&ctx->d_dec, sizeof(fkv_decconst)), "decoder alloc");
     CK(cudaMemcpy(ctx->d_dec, &dec, sizeof(dec), cudaMemcpyHostToDevice), "decoder copy");
+    CK(cudaMalloc(&ctx->d_T, T.size() * sizeof(longlong2)), "decoder alloc");
+    CK(cudaMemcpy(ctx->d_T, T.data(), T.size() * sizeof(longlong2), cudaMemcpyHostToDevice), "decoder copy");
     CK(cudaMalloc(&ctx->d_status, sizeof(unsigned)), "status alloc");
     CK(cudaMemset(ctx->d_status, 0, sizeof(unsigned)), "status init");
 
@@ -269,6 +280,7 @@ int fkv_destroy(fkv_ctx *ctx)
     cudaDeviceSynchronize();
     cudaFree(ctx->d_V);
     cudaFree(ctx->d_dec);
+    cudaFree(ctx->d_T);
     cudaFree(ctx->d_status);
     cudaFree(ctx->d_scratch);
     destroy_cbset(ctx->cb[0]);

@@ -25,13 +25,11 @@ struct fkv_cbset {
     CUtensorMap tmap;         // TMA map over cb16 as [rows][D], box {64, 256}, 128B swizzle
 };
 
-// Decoder constants: everything in Q1.62 fixed point (value * 2^62).
+// Decoder constants (see decode_core.cuh).  Fixed point is Q1.62 (value * 2^62).
 struct fkv_decconst {
     long long vx[256], vy[256];    // V(c)
-    long long wx[256], wy[256];    // (1 - r) V(c)
-    long long hn[256];             // |V(c)|^2 / 2 in units of 2^-60
-    long long rinv;                // round(2^rshift / r)
-    int rshift;
+    float vfx[256], vfy[256];      // V(c) rounded to float
+    long long alim[48];            // anchor limit 2^-4 r^m in Q1.62, per span length m
 };
 
 struct fkv_ctx {
@@ -41,6 +39,7 @@ struct fkv_ctx {
     int device = 0;
     double2 *d_V = nullptr;        // [256] vertices, entries >= N are NaN
     fkv_decconst *d_dec = nullptr; // decoder constants (device copy)
+    longlong2 *d_T = nullptr;      // [L][N] (1-r) r^j V(c) in Q1.62
     unsigned *d_status = nullptr;
     // archive geometry and codebooks
     bool has_cb = false;

@@ -7,7 +7,7 @@
 // that slice sit in shared memory, so HBM sees only the index bytes in and
 // the rebuilt K/V out.  Sums run in float32, stage order, then round to
 // nearest-even into the cache dtype.
-#include "fkv_internal.h"
+#include "decode_core.cuh"
 
 namespace {
 
@@ -40,7 +40,7 @@ __device__ __forceinline__ void store2(void *out, int dtype, int64_t elem, float
 
 __global__ void __launch_bounds__(kThreads) k_gather(const GatherArgs a)
 {
-    extern __shared__ __align__(16) float scb[];   // [S][256][Dp]
+    extern __shared__ __align__(16) float scb[];   // [S][256][Dp] floats, then offsets and indices
     const int chunk = blockIdx.x % a.chunks;
     const int part = (blockIdx.x / a.chunks) % a.parts;
     const int g = blockIdx.x / (a.chunks * a.parts);
@@ -54,81 +54,41 @@ __global__ void __launch_bounds__(kThreads) k_gather(const GatherArgs a)
         const int row = i / q4, q = i - row * q4;
         reinterpret_cast<float4 *>(scb)[i] = __ldg(reinterpret_cast<const float4 *>(src + static_cast<int64_t>(row) * D + d0) + q);
     }
+    // this block's indices and output offsets -> shared memory (independent
+    // loads, many in flight; 32-bit index arithmetic, checked on the host)
+    int64_t *soff = reinterpret_cast<int64_t *>(scb + S * 256 * Dp);
+    uint8_t *sids = reinterpret_cast<uint8_t *>(soff + kChunk);
+    const int nvec = static_cast<int>(a.batch * a.n_rec);
+    const int v_beg = chunk * static_cast<int>(kChunk);
+    const int nv = min(nvec - v_beg, static_cast<int>(kChunk));
+    const unsigned n_rec = static_cast<unsigned>(a.n_rec);
+    for (int vi = threadIdx.x; vi < nv; vi += kThreads) {
+        const unsigned v = static_cast<unsigned>(v_beg + vi);
+        const unsigned b = v / n_rec;
+        const unsigned rec = v - b * n_rec;
+        const uint8_t *ids = a.sym + (static_cast<int64_t>(b) * a.n_layers + l) * a.stream_stride +
+                             static_cast<int64_t>(rec) * a.R + a.kv_off + h * S;
+        for (int s = 0; s < S; ++s)
+            sids[vi * S + s] = __ldg(ids + s);
+        soff[vi] = l * a.s_layer + b * a.s_batch + h * a.s_head + (a.t0 + rec) * a.s_pos + d0;
+    }
     __syncthreads();
     const int tpv = Dp / 2;                  // threads per vector (two dims each)
     const int vpi = kThreads / tpv;          // vectors per pass
     const int dd = (threadIdx.x % tpv) * 2;
-    const int64_t nvec = a.batch * a.n_rec;
-    const int64_t v_beg = static_cast<int64_t>(chunk) * kChunk;
-    const int64_t v_end = min(nvec, v_beg + kChunk);
-    for (int64_t v = v_beg + threadIdx.x / tpv; v < v_end; v += vpi) {
-        const int64_t b = v / a.n_rec;
-        const int64_t rec = v - b * a.n_rec;
-        const uint8_t *ids = a.sym + (b * a.n_layers + l) * a.stream_stride + rec * a.R + a.kv_off + h * S;
+#pragma unroll 2
+    for (int vi = threadIdx.x / tpv; vi < nv; vi += vpi) {
         float x = 0.0f, y = 0.0f;
         for (int s = 0; s < S; ++s) {
-            const float2 c = *reinterpret_cast<const float2 *>(scb + (s * 256 + ids[s]) * Dp + dd);
+            const float2 c = *reinterpret_cast<const float2 *>(scb + (s * 256 + sids[vi * S + s]) * Dp + dd);
             x += c.x;
             y += c.y;
         }
-        const int64_t e = l * a.s_layer + b * a.s_batch + h * a.s_head + (a.t0 + rec) * a.s_pos + d0 + dd;
-        store2(a.out, a.dtype, e, x, y);
+        store2(a.out, a.dtype, soff[vi] + dd, x, y);
     }
 }
 
 // ------------------------------------------------------- random reads ---
-struct DecTables {
-    long long vx[256], vy[256], wx[256], wy[256], hn[256];
-};
-
-__device__ __forceinline__ long long vscore(const DecTables &d, long long X, long long Y, int c)
-{
-    return __mul64hi(X, d.vx[c]) + __mul64hi(Y, d.vy[c]) - d.hn[c];
-}
-
-__device__ __forceinline__ int classify(const DecTables &d, long long X, long long Y, int N)
-{
-    if (N <= 8) {
-        int best = 0;
-        long long bs = vscore(d, X, Y, 0);
-        for (int c = 1; c < N; ++c) {
-            const long long s = vscore(d, X, Y, c);
-            if (s > bs) {
-                bs = s;
-                best = c;
-            }
-        }
-        return best;
-    }
-    const float xf = static_cast<float>(static_cast<int>(X >> 32));
-    const float yf = static_cast<float>(static_cast<int>(Y >> 32));
-    int c0 = __float2int_rn(atan2f(yf, xf) * (static_cast<float>(N) * 0.15915494309189535f));
-    if (c0 < 0)
-        c0 += N;
-    if (c0 >= N)
-        c0 -= N;
-    const int cm = c0 == 0 ? N - 1 : c0 - 1;
-    const int cp = c0 == N - 1 ? 0 : c0 + 1;
-    int best = c0;
-    long long bs = vscore(d, X, Y, c0);
-    long long s = vscore(d, X, Y, cm);
-    if (s > bs) {
-        bs = s;
-        best = cm;
-    }
-    s = vscore(d, X, Y, cp);
-    if (s > bs)
-        best = cp;
-    return best;
-}
-
-__device__ __forceinline__ long long mulshift(long long v, long long rinv, int k)
-{
-    const unsigned long long lo = static_cast<unsigned long long>(v) * static_cast<unsigned long long>(rinv);
-    const long long hi = __mul64hi(v, rinv);
-    return static_cast<long long>((lo >> k) | (static_cast<unsigned long long>(hi) << (64 - k)));
-}
-
 constexpr int kReadWarps = 8;
 constexpr int kMaxRecord = 1024;
 
@@ -142,29 +102,27 @@ struct ReadArgs {
     int n_layers, n_heads, D, SK, SV, R, N, L;
     const float *cbk, *cbv;
     const fkv_decconst *dec;
+    const longlong2 *T;
     unsigned *status;
 };
+
+__host__ __device__ inline int read_tables_bytes(int N, int L)
+{
+    return (fkvdec::smem_bytes(N, L) + 15) & ~15;
+}
 
 // One warp per request: its lanes decode the spans covering the record into
 // shared memory, then gather the record's 2 * H head vectors.
 __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
 {
-    __shared__ DecTables sd;
-    __shared__ uint8_t srec[kReadWarps][kMaxRecord];
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
-        sd.vx[i] = a.dec->vx[i];
-        sd.vy[i] = a.dec->vy[i];
-        sd.wx[i] = a.dec->wx[i];
-        sd.wy[i] = a.dec->wy[i];
-        sd.hn[i] = a.dec->hn[i];
-    }
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(a.dec, a.T, a.N, a.L, dsm);
+    uint8_t *srec = dsm + read_tables_bytes(a.N, a.L);
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t q = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp;
     if (q >= a.n_req)
         return;
-    const long long rinv = a.dec->rinv;
-    const int rsh = a.dec->rshift;
     const int64_t st = a.req[2 * q], rec = a.req[2 * q + 1];
     const int H = a.n_heads, D = a.D, R = a.R, L = a.L;
     const int64_t out_vec = static_cast<int64_t>(2) * H * D;
@@ -178,22 +136,19 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
     const int64_t n = a.n_rec * R;
     const int64_t sym0 = rec * R;
     const int64_t u0 = sym0 / L, u1 = (sym0 + R - 1) / L;
-    uint8_t *my = srec[warp];
+    uint8_t *my = srec + warp * kMaxRecord;
     bool bad = false;
     for (int64_t u = u0 + lane; u <= u1; u += 32) {
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
         const double2 p = a.pts[st * a.pt_stride + u];
-        long long X = __double2ll_rn(p.x * 4611686018427387904.0);
-        long long Y = __double2ll_rn(p.y * 4611686018427387904.0);
-        for (int k = m - 1; k >= 0; --k) {
-            const int c = classify(sd, X, Y, a.N);
-            const int64_t pos = u * L + k - sym0;
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        const int64_t base = u * L - sym0;
+        fkvdec::walk(t, X, Y, m, [&](int j, int c) {
+            const int64_t pos = base + m - 1 - j;
             if (pos >= 0 && pos < R)
                 my[pos] = static_cast<uint8_t>(c);
-            X = mulshift(static_cast<long long>(static_cast<unsigned long long>(X) - static_cast<unsigned long long>(sd.wx[c])), rinv, rsh);
-            Y = mulshift(static_cast<long long>(static_cast<unsigned long long>(Y) - static_cast<unsigned long long>(sd.wy[c])), rinv, rsh);
-        }
-        const long long lim = 1ll << 58;
+        });
+        const long long lim = __ldg(&a.dec->alim[m]);
         bad |= X > lim || X < -lim || Y > lim || Y < -lim;
     }
     if (bad)
@@ -254,12 +209,14 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int6
     const int64_t nvec = a.batch * n_rec;
     if (nvec <= 0)
         return cudaSuccess;
+    if (nvec > 0x7FFFFFFF)
+        return cudaErrorInvalidValue;   // vector indices are 32-bit in the kernel
     const int64_t chunks = (nvec + kChunk - 1) / kChunk;
     const int64_t blocks = chunks * parts * c->Ly * c->H;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
     a.chunks = static_cast<int>(chunks);
-    const size_t smem = static_cast<size_t>(a.S) * 256 * a.Dp * 4;
+    const size_t smem = static_cast<size_t>(a.S) * 256 * a.Dp * 4 + static_cast<size_t>(kChunk) * (8 + a.S);
     cudaError_t e = cudaFuncSetAttribute(k_gather, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem > 48 * 1024 ? smem : 48 * 1024));
     if (e != cudaSuccess)
@@ -292,12 +249,17 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     a.cbk = c->cb[0].cb32;
     a.cbv = c->cb[1].cb32;
     a.dec = c->d_dec;
+    a.T = c->d_T;
     a.status = c->d_status;
     if (n_req <= 0)
         return cudaSuccess;
     const int64_t blocks = (n_req + kReadWarps - 1) / kReadWarps;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    k_read_kv<<<static_cast<unsigned>(blocks), kReadWarps * 32, 0, st>>>(a);
+    const int smem = read_tables_bytes(a.N, a.L) + kReadWarps * kMaxRecord;
+    cudaError_t e = cudaFuncSetAttribute(k_read_kv, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    k_read_kv<<<static_cast<unsigned>(blocks), kReadWarps * 32, smem, st>>>(a);
     return cudaGetLastError();
 }
