@@ -63,6 +63,7 @@ void destroy_cbset(fkv_cbset &s)
     cudaFree(s.cnorm);
     cudaFree(s.cb16);
     cudaFree(s.escale);
+    cudaFree(s.cbaug);
     s = fkv_cbset();
 }
 
@@ -86,17 +87,41 @@ EncodeTiledFn encode_tiled()
     return fn;
 }
 
-// Upload one K-or-V half of the codebooks: float32 copy, squared norms, the
-// fp16 hi/lo split (scaled per (group, stage) by a power of two) and its TMA map.
+// Byte offset of element (row, k) of a [rows x 16] fp16 operand in the
+// no-swizzle K-major core-matrix layout (8 x 16-byte core matrices; 128 B
+// between the two along K, 256 B between 8-row groups).
+size_t core16_offset(int row, int k)
+{
+    return static_cast<size_t>(row / 8) * 256 + (k / 8) * 128 + (row % 8) * 16 + (k % 8) * 2;
+}
+
+// Three fp16 parts whose sum is v to about 33 bits.
+void split3(double v, __half *out)
+{
+    double rest = v;
+    for (int i = 0; i < 3; ++i) {
+        out[i] = __double2half(rest);
+        rest -= static_cast<double>(__half2float(out[i]));
+    }
+}
+
+// Upload one K-or-V half of the codebooks: float32 copy, squared norms and
+// the fp16 operands of the tensor-core RVQ kernels with their TMA map.
+//   D = 128 (k_rvq<128>): hi/lo split of c 2^-e, max |c 2^-e| in [2^14, 2^15).
+//   D = 64 (k_rvq64): hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^8, 2^9),
+//   and a 256 x 16 norm operand per (group, stage): columns 0-2 hold three
+//   fp16 parts of ||c 2^-e||^2 2^-10, columns 3-5 hold 2^14, the rest zero.
 int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
 {
     fkv_cbset &s = ctx->cb[kv];
     s.stages = stages;
     const int G = ctx->Ly * ctx->H, D = ctx->D;
+    const bool d64 = D == 64;
     const size_t ncode = static_cast<size_t>(G) * stages * 256;
     std::vector<float> cn(ncode);
     std::vector<int> es(static_cast<size_t>(G) * stages);
     std::vector<__half> c16(ncode * 2 * D);
+    std::vector<__half> caug(d64 ? ncode * 16 : 0, __float2half(0.0f));
     for (int gs = 0; gs < G * stages; ++gs) {
         const float *cb = host + static_cast<size_t>(gs) * 256 * D;
         float m = 0.0f;
@@ -108,20 +133,32 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         int E = 0;
         if (m > 0.0f)
             frexpf(m, &E);
-        const int e = m > 0.0f ? E - 15 : 0;
+        const int e = m > 0.0f ? (d64 ? E - 9 : E - 15) : 0;
         es[gs] = e;
+        const float mul = d64 ? -2.0f : 1.0f;
         for (int j = 0; j < 256; ++j) {
-            double nn = 0.0;
+            double nn = 0.0, ns = 0.0;
             for (int d = 0; d < D; ++d) {
                 const double v = cb[j * D + d];
                 nn += v * v;
-                const float sv = ldexpf(cb[j * D + d], -e);
+                const double vs = ldexp(v, -e);
+                ns += vs * vs;
+                const float sv = mul * ldexpf(cb[j * D + d], -e);
                 const __half hi = __float2half_rn(sv);
                 const __half lo = __float2half_rn(sv - __half2float(hi));
                 c16[((static_cast<size_t>(gs) * 2 + 0) * 256 + j) * D + d] = hi;
                 c16[((static_cast<size_t>(gs) * 2 + 1) * 256 + j) * D + d] = lo;
             }
             cn[static_cast<size_t>(gs) * 256 + j] = static_cast<float>(nn);
+            if (d64) {
+                __half *blk = caug.data() + static_cast<size_t>(gs) * 256 * 16;
+                __half parts[3];
+                split3(ldexp(ns, -10), parts);
+                for (int k = 0; k < 16; ++k) {
+                    const __half val = k < 3 ? parts[k] : (k < 6 ? __float2half(16384.0f) : __float2half(0.0f));
+                    blk[core16_offset(j, k) / 2] = val;
+                }
+            }
         }
     }
     CK(cudaMalloc(&s.cb32, ncode * D * sizeof(float)), "codebook alloc");
@@ -132,6 +169,10 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
     CK(cudaMemcpy(s.cnorm, cn.data(), ncode * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.cb16, c16.data(), c16.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.escale, es.data(), es.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
+    if (d64) {
+        CK(cudaMalloc(&s.cbaug, caug.size() * sizeof(__half)), "codebook alloc");
+        CK(cudaMemcpy(s.cbaug, caug.data(), caug.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
+    }
     EncodeTiledFn enc = encode_tiled();
     if (!enc)
         return fail(ctx, FKV_ECUDA, "cuTensorMapEncodeTiled unavailable");

@@ -23,6 +23,9 @@ struct fkv_cbset {
     __half *cb16 = nullptr;   // [Ly*H][S][2][256][D] fp16 hi/lo split, scaled by 2^-e
     int *escale = nullptr;    // [Ly*H][S] exponent e of the fp16 split
     CUtensorMap tmap;         // TMA map over cb16 as [rows][D], box {64, 256}, 128B swizzle
+    // 64-dimensional heads only (rvq.cu k_rvq64): cb16 holds the hi/lo split of
+    // -2 c 2^-e with max |c 2^-e| in [2^8, 2^9), and cbaug the norm operand.
+    __half *cbaug = nullptr;  // [Ly*H][S] blocks of 256 x 16 fp16 in core-matrix layout (8 KB)
 };
 
 // Decoder constants (see decode_core.cuh).  Fixed point is Q1.62 (value * 2^62).

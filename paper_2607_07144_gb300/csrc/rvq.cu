@@ -39,6 +39,7 @@ struct RvqArgs {
     const float *cb32;
     const float *cnorm;
     const int *escale;
+    const __half *cbaug;
     uint8_t *sym;
     int64_t stream_stride, rec0;
     int R, kv_off;
@@ -92,6 +93,13 @@ __device__ __forceinline__ void load8(const uint8_t *p, int dtype, float *o)
             o[2 * i + 1] = f.y;
         }
     }
+}
+
+// 2^e as a float for e in [-126, 127] (clamped), built from its exponent bits.
+__device__ __forceinline__ float pow2f(int e)
+{
+    e = e < -126 ? -126 : (e > 127 ? 127 : e);
+    return __int_as_float((e + 127) << 23);
 }
 
 // Power-of-two exponent e such that m * 2^-e lies in [2^14, 2^15) (0 for m = 0).
@@ -374,6 +382,549 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
         tmem_dealloc(tmem, kTmemCols);
 }
 
+// ===================================================================
+// Persistent, warp-specialised kernel for 64-dimensional heads.
+//
+// One CTA per SM walks pairs of tiles (2 x 128 vectors of one codebook
+// group) through all stages.  Warp 0 streams the stage operands into a double
+// buffer (fp16 hi/lo of -2 c' by TMA, the 256 x 16 norm operand by a bulk
+// copy); warp 1 issues the MMAs; two 4-warp epilogue groups each own one tile:
+// a 128 x 256 fp32 accumulator in tensor memory (2 x 256 of the 512 columns),
+// a hi/lo operand tile of the scaled residual r' and its 128 x 16 norm operand.
+//
+// Every quantity of a (group, stage) is scaled by one power of two 2^-e (set
+// by the codebook: max |c'| in [2^8, 2^9)), so with the extra K = 16 MMA
+//     acc_j = sum (r'_hi,lo) (-2 c'_hi,lo) + 2^10 sum_3 parts(||c'_j||^2 2^-10)
+//             + 2^14 sum_3 parts(||r'||^2 2^-14) = ||r' - c'_j||^2
+// (hi*hi + hi*lo + lo*hi, ~22-bit operands; norms to ~33 bits) is the squared
+// distance itself, non-negative, so the argmin keys are its float bits read as
+// integers with the column index packed into the low 8 bits: one integer min
+// per column.  The packed keys resolve distances to 2^-15 relative, which is
+// inside the 1e-4 ||r||^2 tie band while the best distance is below 3 ||r'||^2;
+// otherwise the row is rescanned with exact float compares.  A row whose
+// scaled residual reaches 2^11 (|r| above 4x the largest codeword element) is
+// scored exactly in fp32 instead.  The fp32 residual lives in registers; the
+// chosen codeword comes from the buffer; the next pair's 16-bit input rows are
+// prefetched into registers during the last stage.  Both tiles of a pair share
+// each stage's operands, so one tile's epilogue overlaps the other's MMAs.
+namespace v2 {
+constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups
+constexpr int kThreads = kWarps * 32;
+constexpr int A_TILE = kRows * 128;          // 16 KB: 128 rows x 64 fp16 (128-byte swizzle)
+constexpr int A_SLOT = 2 * A_TILE;           // hi + lo
+constexpr int A_AUG = kRows * 32;            // 4 KB: 128 rows x 16 fp16 (core-matrix layout)
+constexpr int B_TILE = kCodes * 128;         // 32 KB
+constexpr int B_AUG = kCodes * 32;           // 8 KB
+constexpr int B_BUF = 2 * B_TILE + B_AUG;    // 72 KB
+constexpr int OFF_A = 0;
+constexpr int OFF_AAUG = 2 * A_SLOT;
+constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 72 KB: 1024-aligned
+constexpr int OFF_BAR = OFF_B + 2 * B_BUF;   // b_full[2], b_empty[2], a_ready[2], acc_full[2], drain
+constexpr int OFF_SLOT = OFF_BAR + 80;
+constexpr int OFF_LO = OFF_SLOT + 16;        // lo-operand use stamps, one per slot
+constexpr int OFF_ABORT = OFF_LO + 16;
+constexpr int END = OFF_ABORT + 16;
+constexpr int SMEM = END + 1024;
+constexpr float kFastLimit = 2048.0f;        // |r'| below 2^11: operands and norms in range
+}  // namespace v2
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// 1-D bulk copy global -> shared, completion counted on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+// Shared-memory descriptor of a K-major operand in the no-swizzle
+// core-matrix layout: 128 B between the two 8x16 B core matrices along K,
+// 256 B between 8-row groups.
+__device__ __forceinline__ uint64_t sdesc_core16(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+    d |= static_cast<uint64_t>(128 >> 4) << 16;     // leading byte offset: along K
+    d |= static_cast<uint64_t>(256 >> 4) << 32;     // stride byte offset: 8-row groups
+    d |= static_cast<uint64_t>(1) << 46;            // descriptor version (sm_100 family)
+    return d;                                       // swizzle mode 0: none
+}
+
+// 16-byte word of row `row`, columns 8h .. 8h+7, of a [rows x 16] operand.
+__device__ __forceinline__ uint32_t core16_off(int row, int h)
+{
+    return static_cast<uint32_t>((row >> 3) * 256 + h * 128 + (row & 7) * 16);
+}
+
+__device__ __forceinline__ uint32_t pack_half2(float a, float b)
+{
+    const __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t *r)
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// tcgen05.ld of 16 columns without waiting; pair with tmem_wait16 on the
+// same registers before using them.
+__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t *r)
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+// tcgen05.wait::ld with the in-flight registers as read-write operands, so no
+// use of them can be scheduled above the wait.
+__device__ __forceinline__ void tmem_wait16(uint32_t *r)
+{
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+                   "+r"(r[14]), "+r"(r[15])
+                 :
+                 : "memory");
+}
+
+// Scale the fp32 residual by `sc`, store its hi/lo split into this row of
+// the operand tile and its squared norm (three fp16 parts of ||r'||^2 2^-14)
+// into the row's norm operand.  Returns whether any lo is nonzero; *fast
+// tells whether every |r'| stays below the fast-path limit, *norm2 = ||r'||^2.
+__device__ __forceinline__ bool write_operands(uint8_t *ahi, uint8_t *alo, uint8_t *aaug, int row, const float *r,
+                                               float sc, bool *fast, float *norm2)
+{
+    uint32_t nz = 0;
+    float nrm = 0.0f, mx = 0.0f;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        uint4 hv, lv;
+        uint32_t *hw = &hv.x, *lw = &lv.x;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float a0 = r[c * 8 + 2 * i] * sc, a1 = r[c * 8 + 2 * i + 1] * sc;
+            nrm = fmaf(a0, a0, nrm);
+            nrm = fmaf(a1, a1, nrm);
+            mx = fmaxf(mx, fmaxf(fabsf(a0), fabsf(a1)));
+            const __half2 h2 = __floats2half2_rn(a0, a1);
+            const float2 hf = __half22float2(h2);
+            hw[i] = *reinterpret_cast<const uint32_t *>(&h2);
+            lw[i] = pack_half2(a0 - hf.x, a1 - hf.y);
+            nz |= lw[i] & 0x7FFF7FFFu;   // any nonzero lo (either sign of zero counts as zero)
+        }
+        const uint32_t off = swz(row, c);
+        *reinterpret_cast<uint4 *>(ahi + off) = hv;
+        *reinterpret_cast<uint4 *>(alo + off) = lv;
+    }
+    // norm parts: ||r'||^2 2^-14 = p0 + p1 + p2
+    const float q = nrm * 0x1p-14f;
+    const float p0 = __half2float(__float2half_rn(q));
+    const float p1 = __half2float(__float2half_rn(q - p0));
+    const float p2 = q - p0 - p1;
+    uint4 w;
+    w.x = pack_half2(1024.0f, 1024.0f);
+    w.y = pack_half2(1024.0f, p0);
+    w.z = pack_half2(p1, p2);
+    w.w = 0u;
+    *reinterpret_cast<uint4 *>(aaug + core16_off(row, 0)) = w;
+    *fast = mx < v2::kFastLimit;
+    *norm2 = nrm;
+    return nz != 0;
+}
+
+template <int ESZ>
+__device__ __forceinline__ void unpack_row64(const uint4 *xr, int dtype, float *r)
+{
+    if (ESZ == 4) {
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            r[4 * c] = __uint_as_float(xr[c].x);
+            r[4 * c + 1] = __uint_as_float(xr[c].y);
+            r[4 * c + 2] = __uint_as_float(xr[c].z);
+            r[4 * c + 3] = __uint_as_float(xr[c].w);
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const uint32_t w[4] = {xr[c].x, xr[c].y, xr[c].z, xr[c].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                float2 f;
+                if (dtype == FKV_F16)
+                    f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+                else
+                    f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
+                r[8 * c + 2 * i] = f.x;
+                r[8 * c + 2 * i + 1] = f.y;
+            }
+        }
+    }
+}
+
+// Exact fp32 scoring of one row against the 256 codewords of a buffer
+// (c' = -(hi + lo) / 2), for rows outside the fast path.  Lowest index on ties.
+__device__ __forceinline__ int slow_argmin(const float *r, float sc, const uint8_t *bb)
+{
+    float best = INFINITY;
+    int bidx = 0;
+#pragma unroll 1
+    for (int j = 0; j < kCodes; ++j) {
+        float d = 0.0f;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const uint32_t off = swz(j, c);
+            const uint4 hv = *reinterpret_cast<const uint4 *>(bb + off);
+            const uint4 lv = *reinterpret_cast<const uint4 *>(bb + v2::B_TILE + off);
+            const __half2 *hh = reinterpret_cast<const __half2 *>(&hv);
+            const __half2 *ll = reinterpret_cast<const __half2 *>(&lv);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 h = __half22float2(hh[i]), l = __half22float2(ll[i]);
+                const float t0 = fmaf(r[c * 8 + 2 * i], sc, 0.5f * (h.x + l.x));
+                const float t1 = fmaf(r[c * 8 + 2 * i + 1], sc, 0.5f * (h.y + l.y));
+                d = fmaf(t0, t0, d);
+                d = fmaf(t1, t1, d);
+            }
+        }
+        if (d < best) {
+            best = d;
+            bidx = j;
+        }
+    }
+    return bidx;
+}
+
+// Packed keys: the distance's float bits with the column index in the low 8
+// bits; non-negative floats order as signed integers (a rounding-negative
+// distance sorts first, as the smallest), so one integer min per column finds
+// the smallest distance and its column, the lower column on equal keys.
+// Four independent chains (column j % 4).
+__device__ __forceinline__ void min_keys16(const uint32_t *acc, int col0, int *m)
+{
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        const int key = static_cast<int>((acc[j] & 0xFFFFFF00u) | static_cast<uint32_t>(col0 + j));
+        m[j & 3] = min(m[j & 3], key);
+    }
+}
+
+// Exact argmin of an accumulator row (float compare, lowest index on ties).
+__device__ __forceinline__ int exact_argmin_tmem(uint32_t trow)
+{
+    float best = INFINITY;
+    int bidx = 0;
+#pragma unroll 1
+    for (int ch = 0; ch < kCodes / 16; ++ch) {
+        uint32_t acc[16];
+        tmem_ld16(trow + ch * 16, acc);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const float d = __uint_as_float(acc[j]);
+            if (d < best) {
+                best = d;
+                bidx = ch * 16 + j;
+            }
+        }
+    }
+    return bidx;
+}
+
+template <int ESZ>
+__global__ void __launch_bounds__(v2::kThreads, 1)
+k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per_group, int n_pairs)
+{
+    using namespace v2;
+    constexpr int XN = 64 * ESZ / 16;            // 16-byte chunks per input row
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t sbase = smem_u32(base);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(base + OFF_ABORT);
+    volatile int *lo_stamp = reinterpret_cast<volatile int *>(base + OFF_LO);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // barrier i: 0,1 b_full; 2,3 b_empty; 4,5 a_ready; 6,7 acc_full; 8 drain (MMA completion at exit)
+    auto bar = [&](int i) { return sbase + OFF_BAR + 8u * i; };
+    if (tid == 0) {
+        mbar_init(bar(0), 1);
+        mbar_init(bar(1), 1);
+        mbar_init(bar(2), 256);
+        mbar_init(bar(3), 256);
+        mbar_init(bar(4), 128);
+        mbar_init(bar(5), 128);
+        mbar_init(bar(6), 1);
+        mbar_init(bar(7), 1);
+        mbar_init(bar(8), 1);
+        lo_stamp[0] = 0;
+        lo_stamp[1] = 0;
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap);
+    }
+    // the norm operands' columns 8..15 are zero for good
+    for (int i = tid; i < 2 * kRows; i += v2::kThreads)
+        *reinterpret_cast<uint4 *>(base + OFF_AAUG + (i / kRows) * A_AUG + core16_off(i % kRows, 1)) =
+            make_uint4(0, 0, 0, 0);
+    fence_proxy_async_smem();
+    if (warp == 1)
+        tmem_alloc(sbase + OFF_SLOT, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(base + OFF_SLOT);
+    const int S = a.S;
+    const int64_t nvec = a.batch * a.n_pos;
+    const int tiles = a.tiles_per_group;
+
+    if (warp == 0) {
+        // ---------------------------------------------------- TMA producer
+        if (lane == 0) {
+            int it = 0;
+            int last[2] = {-1, -1};               // last iteration that loaded each buffer
+            for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
+                const int g = p / pairs_per_group;
+                bool ok = true;
+                for (int s = 0; s < S; ++s, ++it) {
+                    const int bi = it & 1;
+                    const uint32_t ph = (it >> 1) & 1;
+                    if (!wait_or_abort(bar(2 + bi), ph ^ 1, a.status, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t bb = sbase + OFF_B + bi * B_BUF;
+                    const int row0 = (g * S + s) * 2 * kCodes;
+                    mbar_arrive_expect_tx(bar(bi), 2u * B_TILE + B_AUG);
+                    tma_load_2d(bb, &tmap, 0, row0, bar(bi));
+                    tma_load_2d(bb + B_TILE, &tmap, 0, row0 + kCodes, bar(bi));
+                    bulk_load(bb + 2 * B_TILE, a.cbaug + static_cast<int64_t>(g * S + s) * kCodes * 16, B_AUG, bar(bi));
+                    last[bi] = it;
+                }
+                if (!ok)
+                    break;
+            }
+            // no copy may still be landing in shared memory when the CTA exits
+            // (after an abort the consumers may not have waited for them)
+            for (int bi = 0; bi < 2; ++bi)
+                if (last[bi] >= 0)
+                    mbar_wait(bar(bi), (last[bi] >> 1) & 1, a.status);
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
+            int it = 0;
+            uint32_t aph[2] = {0, 0};
+            int use[2] = {0, 0};
+            bool ok = true;
+            for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
+                for (int s = 0; s < S && ok; ++s, ++it) {
+                    const int bi = it & 1;
+                    const uint32_t ph = (it >> 1) & 1;
+                    ok = wait_or_abort(bar(bi), ph, a.status, abort_flag);
+                    if (!ok)
+                        break;
+                    const uint32_t bb = sbase + OFF_B + bi * B_BUF;
+                    for (int k = 0; k < 2; ++k) {
+                        ok = wait_or_abort(bar(4 + k), aph[k], a.status, abort_flag);
+                        if (!ok)
+                            break;
+                        aph[k] ^= 1;
+                        tc_fence_after();
+                        const bool lo = lo_stamp[k] == ++use[k];
+                        const uint32_t ab = sbase + OFF_A + k * A_SLOT;
+                        const uint32_t acc = tmem + k * 256;
+                        // squared norms first (K = 16, no swizzle), then the split dot products
+                        umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(bb + 2 * B_TILE),
+                                 idesc, 0);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t dah = sdesc_sw128(ab + kk * 32);
+                            const uint64_t dal = sdesc_sw128(ab + A_TILE + kk * 32);
+                            const uint64_t dbh = sdesc_sw128(bb + kk * 32);
+                            const uint64_t dbl = sdesc_sw128(bb + B_TILE + kk * 32);
+                            umma_f16(acc, dah, dbh, idesc, 1);
+                            umma_f16(acc, dah, dbl, idesc, 1);
+                            if (lo)
+                                umma_f16(acc, dal, dbh, idesc, 1);
+                        }
+                        umma_commit(bar(6 + k));
+                    }
+                }
+            }
+            // every MMA has completed before tensor memory is released
+            umma_commit(bar(8));
+            mbar_wait(bar(8), 0, a.status);
+        }
+    } else {
+        // ---------------------------------------------------- epilogue groups
+        const int k = (warp - 2) >> 2;           // tile slot 0 or 1
+        const int quad = warp & 3;                // TMEM lane quadrant of this warp
+        const int row = quad * 32 + lane;
+        const uint32_t trow = tmem + k * 256 + (static_cast<uint32_t>(quad * 32) << 16);
+        uint8_t *ahi = base + OFF_A + k * A_SLOT;
+        uint8_t *alo = ahi + A_TILE;
+        uint8_t *aaug = base + OFF_AAUG + k * A_AUG;
+        uint4 xr[XN];
+        auto load_row = [&](int p) {
+            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
+            const int tile = 2 * q + k;
+            const int64_t v = static_cast<int64_t>(tile) * kRows + row;
+            if (tile < tiles && v < nvec) {
+                const int l = g / a.n_heads, h = g - l * a.n_heads;
+                const int64_t b = v / a.n_pos;
+                const int64_t t = a.t0 + (v - b * a.n_pos);
+                const uint4 *src = reinterpret_cast<const uint4 *>(
+                    static_cast<const uint8_t *>(a.x) + (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * ESZ);
+#pragma unroll
+                for (int c = 0; c < XN; ++c)
+                    xr[c] = __ldg(src + c);
+            } else {
+#pragma unroll
+                for (int c = 0; c < XN; ++c)
+                    xr[c] = make_uint4(0, 0, 0, 0);
+            }
+        };
+        int it = 0;
+        uint32_t fph = 0;
+        int use = 0;
+        constexpr bool kPrefetch = ESZ == 2;      // 16-bit rows: 32 registers of prefetch
+        if (kPrefetch && static_cast<int>(blockIdx.x) < n_pairs)
+            load_row(blockIdx.x);
+        for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
+            if (!kPrefetch)
+                load_row(p);
+            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
+            const int l = g / a.n_heads, h = g - l * a.n_heads;
+            const int tile = 2 * q + k;
+            const int64_t v = static_cast<int64_t>(tile) * kRows + row;
+            const bool valid = tile < tiles && v < nvec;
+            float r[64];
+            unpack_row64<ESZ>(xr, a.dtype, r);
+            int e = __ldg(&a.escale[g * S]);
+            bool fast;
+            float rn2;
+            bool lo_nz = write_operands(ahi, alo, aaug, row, r, pow2f(-e), &fast, &rn2);
+            ++use;
+            if (lo_nz)
+                lo_stamp[k] = use;
+            fence_proxy_async_smem();
+            mbar_arrive(bar(4 + k));
+            uint8_t idx[8];
+            bool ok = true;
+            for (int s = 0; s < S; ++s, ++it) {
+                const int bi = it & 1;
+                const int e_next = s + 1 < S ? __ldg(&a.escale[g * S + s + 1]) : 0;   // in flight during the waits
+                ok = wait_or_abort(bar(6 + k), fph, a.status, abort_flag) &&
+                     wait_or_abort(bar(bi), (it >> 1) & 1, a.status, abort_flag);
+                // the tensor-memory loads below are warp-collective: the warp
+                // goes on, or leaves, as one
+                ok = __all_sync(0xFFFFFFFFu, ok);
+                if (!ok)
+                    break;
+                fph ^= 1;
+                tc_fence_after();
+                if (kPrefetch && s == S - 1 && p + static_cast<int>(gridDim.x) < n_pairs)
+                    load_row(p + gridDim.x);      // next pair's input, in flight during the epilogue
+                const uint8_t *bb = base + OFF_B + bi * B_BUF;
+                int mk[4] = {0x7FFFFFFF, 0x7FFFFFFF, 0x7FFFFFFF, 0x7FFFFFFF};
+                __syncwarp();
+                {
+                    // double-buffered TMEM reads: chunk c + 1 in flight while chunk c is keyed
+                    uint32_t acc0[16], acc1[16];
+                    tmem_ld16_async(trow, acc0);
+                    tmem_wait16(acc0);
+#pragma unroll
+                    for (int ch = 0; ch < kCodes / 16; ch += 2) {
+                        tmem_ld16_async(trow + (ch + 1) * 16, acc1);
+                        min_keys16(acc0, ch * 16, mk);
+                        tmem_wait16(acc1);
+                        if (ch + 2 < kCodes / 16)
+                            tmem_ld16_async(trow + (ch + 2) * 16, acc0);
+                        min_keys16(acc1, (ch + 1) * 16, mk);
+                        if (ch + 2 < kCodes / 16)
+                            tmem_wait16(acc0);
+                    }
+                }
+                const int key = min(min(mk[0], mk[1]), min(mk[2], mk[3]));
+                int bidx = key & 0xFF;
+                // the packed keys only resolve ties within 2^-15 d_min; that is
+                // inside the 1e-4 ||r||^2 tie band while d_min < 3 ||r'||^2
+                const bool rescan = fast && !(__int_as_float(key & 0xFFFFFF00) < 3.0f * rn2);
+                if (__any_sync(0xFFFFFFFFu, rescan)) {   // warp-collective loads: every lane takes part
+                    const int b = exact_argmin_tmem(trow);
+                    if (rescan)
+                        bidx = b;
+                }
+                tc_fence_before();
+                if (!fast)
+                    bidx = slow_argmin(r, pow2f(-e), bb);
+                idx[s] = static_cast<uint8_t>(bidx);
+                if (s + 1 < S) {
+                    // r <- r - c_bidx  (c = -(hi + lo) 2^(e-1))
+                    const float cs = pow2f(e - 1);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint32_t bo = swz(bidx, c);
+                        const uint4 hv = *reinterpret_cast<const uint4 *>(bb + bo);
+                        const uint4 lv = *reinterpret_cast<const uint4 *>(bb + B_TILE + bo);
+                        const __half2 *hh = reinterpret_cast<const __half2 *>(&hv);
+                        const __half2 *ll = reinterpret_cast<const __half2 *>(&lv);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const float2 ca = __half22float2(hh[i]), cb = __half22float2(ll[i]);
+                            r[8 * c + 2 * i] = fmaf(cs, ca.x + cb.x, r[8 * c + 2 * i]);
+                            r[8 * c + 2 * i + 1] = fmaf(cs, ca.y + cb.y, r[8 * c + 2 * i + 1]);
+                        }
+                    }
+                    if (!valid) {
+#pragma unroll
+                        for (int i = 0; i < 64; ++i)
+                            r[i] = 0.0f;
+                    }
+                    e = e_next;
+                    lo_nz = write_operands(ahi, alo, aaug, row, r, pow2f(-e), &fast, &rn2);
+                    ++use;
+                    if (lo_nz)
+                        lo_stamp[k] = use;
+                    fence_proxy_async_smem();
+                    mbar_arrive(bar(4 + k));
+                }
+                mbar_arrive(bar(2 + bi));
+            }
+            if (!ok)
+                break;
+            if (valid) {
+                const int64_t b = v / a.n_pos;
+                const int64_t t = a.t0 + (v - b * a.n_pos);
+                uint8_t *dst = a.sym + (b * a.n_layers + l) * a.stream_stride + (a.rec0 + (t - a.t0)) * a.R +
+                               a.kv_off + h * S;
+                for (int s = 0; s < S; ++s)
+                    dst[s] = idx[s];
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
@@ -396,6 +947,7 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
     a.cb32 = cb.cb32;
     a.cnorm = cb.cnorm;
     a.escale = cb.escale;
+    a.cbaug = cb.cbaug;
     a.sym = sym;
     a.stream_stride = stream_stride;
     a.rec0 = rec0;
@@ -411,15 +963,28 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
         return cudaErrorInvalidConfiguration;
     a.tiles_per_group = static_cast<int>(tiles);
     if (c->D == 64) {
-        static bool attr = false;
-        if (!attr) {
-            cudaError_t e = cudaFuncSetAttribute(k_rvq<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 Layout<64>::SMEM);
+        const int64_t ppg = (tiles + 1) / 2;
+        const int64_t n_pairs = ppg * c->Ly * c->H;
+        if (n_pairs > 0x7FFFFFFF)
+            return cudaErrorInvalidConfiguration;
+        int sms = 0;
+        cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+        if (e != cudaSuccess)
+            return e;
+        const unsigned grid = static_cast<unsigned>(n_pairs < sms ? n_pairs : sms);
+        if (x->dtype == FKV_F32) {
+            e = cudaFuncSetAttribute(k_rvq64<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, v2::SMEM);
             if (e != cudaSuccess)
                 return e;
-            attr = true;
+            k_rvq64<4><<<grid, v2::kThreads, v2::SMEM, st>>>(cb.tmap, a, static_cast<int>(ppg),
+                                                               static_cast<int>(n_pairs));
+        } else {
+            e = cudaFuncSetAttribute(k_rvq64<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, v2::SMEM);
+            if (e != cudaSuccess)
+                return e;
+            k_rvq64<2><<<grid, v2::kThreads, v2::SMEM, st>>>(cb.tmap, a, static_cast<int>(ppg),
+                                                               static_cast<int>(n_pairs));
         }
-        k_rvq<64><<<static_cast<unsigned>(blocks), kThreads, Layout<64>::SMEM, st>>>(cb.tmap, a);
     } else {
         static bool attr = false;
         if (!attr) {
