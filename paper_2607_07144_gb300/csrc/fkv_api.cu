@@ -108,9 +108,10 @@ void split3(double v, __half *out)
 // Upload one K-or-V half of the codebooks: float32 copy, squared norms and
 // the fp16 operands of the tensor-core RVQ kernels with their TMA map.
 //   D = 128 (k_rvq<128>): hi/lo split of c 2^-e, max |c 2^-e| in [2^14, 2^15).
-//   D = 64 (k_rvq64): hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^8, 2^9),
-//   and a 256 x 16 norm operand per (group, stage): columns 0-2 hold three
-//   fp16 parts of ||c 2^-e||^2 2^-10, columns 3-5 hold 2^14, the rest zero.
+//   D = 64 (k_rvq64): hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^3, 2^9)
+//   (in [2^8, 2^9) at a group's first stage; later stages keep the previous
+//   e while they can), and a 256 x 16 norm operand per (group, stage):
+//   columns 0-2 hold three fp16 parts of ||c 2^-e||^2 2^-10, the rest zero.
 int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
 {
     fkv_cbset &s = ctx->cb[kv];
@@ -133,7 +134,16 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         int E = 0;
         if (m > 0.0f)
             frexpf(m, &E);
-        const int e = m > 0.0f ? (d64 ? E - 9 : E - 15) : 0;
+        int e = m > 0.0f ? (d64 ? E - 9 : E - 15) : 0;
+        if (d64 && gs % stages != 0) {
+            // 64-dim heads: keep the previous stage's scale while this stage's
+            // max |c| 2^-e stays in [2^3, 2^9), so the kernel rescales the
+            // residual only between stages of very different magnitude
+            const int prev = es[gs - 1];
+            const float q = ldexpf(m, -prev);
+            if (q >= 8.0f && q < 512.0f)
+                e = prev;
+        }
         es[gs] = e;
         const float mul = d64 ? -2.0f : 1.0f;
         for (int j = 0; j < 256; ++j) {
@@ -155,7 +165,7 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
                 __half parts[3];
                 split3(ldexp(ns, -10), parts);
                 for (int k = 0; k < 16; ++k) {
-                    const __half val = k < 3 ? parts[k] : (k < 6 ? __float2half(16384.0f) : __float2half(0.0f));
+                    const __half val = k < 3 ? parts[k] : __float2half(0.0f);
                     blk[core16_offset(j, k) / 2] = val;
                 }
             }

@@ -24,7 +24,7 @@ struct fkv_cbset {
     int *escale = nullptr;    // [Ly*H][S] exponent e of the fp16 split
     CUtensorMap tmap;         // TMA map over cb16 as [rows][D], box {64, 256}, 128B swizzle
     // 64-dimensional heads only (rvq.cu k_rvq64): cb16 holds the hi/lo split of
-    // -2 c 2^-e with max |c 2^-e| in [2^8, 2^9), and cbaug the norm operand.
+    // -2 c 2^-e with max |c 2^-e| in [2^3, 2^9), and cbaug the norm operand.
     __half *cbaug = nullptr;  // [Ly*H][S] blocks of 256 x 16 fp16 in core-matrix layout (8 KB)
 };
 

@@ -389,43 +389,45 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
 // group) through all stages.  Warp 0 streams the stage operands into a double
 // buffer (fp16 hi/lo of -2 c' by TMA, the 256 x 16 norm operand by a bulk
 // copy); warp 1 issues the MMAs; two 4-warp epilogue groups each own one tile:
-// a 128 x 256 fp32 accumulator in tensor memory (2 x 256 of the 512 columns),
-// a hi/lo operand tile of the scaled residual r' and its 128 x 16 norm operand.
+// a 128 x 256 fp32 accumulator in tensor memory (2 x 256 of the 512 columns)
+// and a hi/lo operand tile of the scaled residual r'.
 //
-// Every quantity of a (group, stage) is scaled by one power of two 2^-e (set
-// by the codebook: max |c'| in [2^8, 2^9)), so with the extra K = 16 MMA
+// A (group, stage) is scaled by a power of two 2^-e (max |c'| in [2^3, 2^9),
+// usually one e for all stages of a group), and an extra K = 16 MMA against a
+// constant operand adds the codeword norms, so
 //     acc_j = sum (r'_hi,lo) (-2 c'_hi,lo) + 2^10 sum_3 parts(||c'_j||^2 2^-10)
-//             + 2^14 sum_3 parts(||r'||^2 2^-14) = ||r' - c'_j||^2
-// (hi*hi + hi*lo + lo*hi, ~22-bit operands; norms to ~33 bits) is the squared
-// distance itself, non-negative, so the argmin keys are its float bits read as
-// integers with the column index packed into the low 8 bits: one integer min
-// per column.  The packed keys resolve distances to 2^-15 relative, which is
-// inside the 1e-4 ||r||^2 tie band while the best distance is below 3 ||r'||^2;
-// otherwise the row is rescanned with exact float compares.  A row whose
-// scaled residual reaches 2^11 (|r| above 4x the largest codeword element) is
-// scored exactly in fp32 instead.  The fp32 residual lives in registers; the
-// chosen codeword comes from the buffer; the next pair's 16-bit input rows are
-// prefetched into registers during the last stage.  Both tiles of a pair share
-// each stage's operands, so one tile's epilogue overlaps the other's MMAs.
+//           = ||r' - c'_j||^2 - ||r'||^2
+// (hi*hi + hi*lo + lo*hi, ~22-bit operands; norms to ~33 bits).  The argmin
+// over the 256 columns is exact on the fp32 accumulators: tcgen05.ld.red
+// returns the minimum of every 16 columns with the load, which gives the
+// best value and its 16-column chunk, and an elementwise minimum across the
+// chunks gives its position inside the chunk; an exact tie (the minimum in two
+// chunks or two positions) is rescanned column by column.  A row whose scaled
+// residual reaches 2^14 (far outside the codebook) is scored exactly in fp32
+// from the stage buffer instead.  The fp32 residual r' lives in registers and
+// is updated with mixed-precision FMAs straight from the fp16 hi/lo codeword in
+// the buffer; the next pair's 16-bit input rows are prefetched into registers
+// during the last stage.  Both tiles of a pair share each stage's operands, so
+// one tile's epilogue overlaps the other's MMAs.
 namespace v2 {
 constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups
 constexpr int kThreads = kWarps * 32;
 constexpr int A_TILE = kRows * 128;          // 16 KB: 128 rows x 64 fp16 (128-byte swizzle)
 constexpr int A_SLOT = 2 * A_TILE;           // hi + lo
-constexpr int A_AUG = kRows * 32;            // 4 KB: 128 rows x 16 fp16 (core-matrix layout)
+constexpr int A_AUG = kRows * 32;            // 4 KB: 128 rows x 16 fp16 (core-matrix layout), constant
 constexpr int B_TILE = kCodes * 128;         // 32 KB
 constexpr int B_AUG = kCodes * 32;           // 8 KB
 constexpr int B_BUF = 2 * B_TILE + B_AUG;    // 72 KB
 constexpr int OFF_A = 0;
 constexpr int OFF_AAUG = 2 * A_SLOT;
-constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 72 KB: 1024-aligned
+constexpr int OFF_B = OFF_AAUG + A_AUG;      // 68 KB: 1024-aligned
 constexpr int OFF_BAR = OFF_B + 2 * B_BUF;   // b_full[2], b_empty[2], a_ready[2], acc_full[2], drain
 constexpr int OFF_SLOT = OFF_BAR + 80;
-constexpr int OFF_LO = OFF_SLOT + 16;        // lo-operand use stamps, one per slot
+constexpr int OFF_LO = OFF_SLOT + 16;        // per slot: the pair whose first-stage lo operand is nonzero
 constexpr int OFF_ABORT = OFF_LO + 16;
 constexpr int END = OFF_ABORT + 16;
 constexpr int SMEM = END + 1024;
-constexpr float kFastLimit = 2048.0f;        // |r'| below 2^11: operands and norms in range
+constexpr float kFastLimit = 16384.0f;       // |r'| below 2^14: fp16 operands in range
 }  // namespace v2
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar)
@@ -466,85 +468,107 @@ __device__ __forceinline__ uint32_t pack_half2(float a, float b)
     return *reinterpret_cast<const uint32_t *>(&h);
 }
 
+__device__ __forceinline__ float min3f(float a, float b, float c)
+{
+    float d;
+    asm volatile("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// x0 += w.lo / 2, x1 += w.hi / 2 for the two fp16 halves of w, each one
+// mixed-precision FMA (exact product, one rounding).
+__device__ __forceinline__ void add_half2_halved(uint32_t w, float &x0, float &x1)
+{
+    asm("{\n\t.reg .b16 l, h, c;\n\t"
+        "mov.b32 {l, h}, %2;\n\t"
+        "mov.b16 c, 0x3800;\n\t"
+        "fma.rn.f32.f16 %0, l, c, %0;\n\t"
+        "fma.rn.f32.f16 %1, h, c, %1;\n\t}"
+        : "+f"(x0), "+f"(x1)
+        : "r"(w));
+}
+
+// hi = fp16(a) (packed pair), lo = fp16(a - hi); a - hi is exact in fp32.
+__device__ __forceinline__ void split_half2(float a0, float a1, uint32_t &hi, uint32_t &lo)
+{
+    asm("{\n\t.reg .b16 x, y, m;\n\t.reg .f32 d0, d1;\n\t"
+        "cvt.rn.f16x2.f32 %0, %3, %2;\n\t"
+        "mov.b32 {x, y}, %0;\n\t"
+        "mov.b16 m, 0xBC00;\n\t"
+        "fma.rn.f32.f16 d0, x, m, %2;\n\t"
+        "fma.rn.f32.f16 d1, y, m, %3;\n\t"
+        "cvt.rn.f16x2.f32 %1, d1, d0;\n\t}"
+        : "=r"(hi), "=r"(lo)
+        : "f"(a0), "f"(a1));
+}
+
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t *r)
 {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
           "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        : "r"(taddr)
+        : "memory");
 }
 
-// tcgen05.ld of 16 columns without waiting; pair with tmem_wait16 on the
-// same registers before using them.
-__device__ __forceinline__ void tmem_ld16_async(uint32_t taddr, uint32_t *r)
+// Columns [c, c + 32) of this thread's accumulator row as two 16-column
+// chunks a and b, with their minima ra and rb (tcgen05.ld.red), loads and
+// wait in one statement.
+__device__ __forceinline__ void tmem_red2x16(uint32_t taddr, float *a, float *b, float &ra, float &rb)
 {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-          "=r"(r[14]), "=r"(r[15])
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, %32, [%34];\n\t"
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %33, [%34+16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=f"(a[0]), "=f"(a[1]), "=f"(a[2]), "=f"(a[3]), "=f"(a[4]), "=f"(a[5]), "=f"(a[6]), "=f"(a[7]), "=f"(a[8]), "=f"(a[9]), "=f"(a[10]), "=f"(a[11]), "=f"(a[12]), "=f"(a[13]), "=f"(a[14]), "=f"(a[15]), "=f"(b[0]), "=f"(b[1]), "=f"(b[2]), "=f"(b[3]), "=f"(b[4]), "=f"(b[5]), "=f"(b[6]), "=f"(b[7]), "=f"(b[8]), "=f"(b[9]), "=f"(b[10]), "=f"(b[11]), "=f"(b[12]), "=f"(b[13]), "=f"(b[14]), "=f"(b[15]),
+          "=f"(ra), "=f"(rb)
         : "r"(taddr));
 }
 
-// tcgen05.wait::ld with the in-flight registers as read-write operands, so no
-// use of them can be scheduled above the wait.
-__device__ __forceinline__ void tmem_wait16(uint32_t *r)
+// Scale the residual row by a power of two.
+__device__ __forceinline__ void scale_row(float *r, float f)
 {
-    asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
-                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
-                   "+r"(r[14]), "+r"(r[15])
-                 :
-                 : "memory");
+#pragma unroll
+    for (int i = 0; i < 64; ++i)
+        r[i] *= f;
 }
 
-// Scale the fp32 residual by `sc`, store its hi/lo split into this row of
-// the operand tile and its squared norm (three fp16 parts of ||r'||^2 2^-14)
-// into the row's norm operand.  Returns whether any lo is nonzero; *fast
-// tells whether every |r'| stays below the fast-path limit, *norm2 = ||r'||^2.
-__device__ __forceinline__ bool write_operands(uint8_t *ahi, uint8_t *alo, uint8_t *aaug, int row, const float *r,
-                                               float sc, bool *fast, float *norm2)
+// Store the hi/lo split of the scaled residual r' into this row of the
+// operand tile.  *fast tells whether every |r'| stays below the fast-path
+// limit; with NZ the return value tells whether any lo is nonzero.
+template <bool NZ>
+__device__ __forceinline__ bool write_operands(uint8_t *ahi, uint8_t *alo, int row, const float *r, bool *fast)
 {
     uint32_t nz = 0;
-    float nrm = 0.0f, mx = 0.0f;
+    float mx = 0.0f;
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
         uint4 hv, lv;
         uint32_t *hw = &hv.x, *lw = &lv.x;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            const float a0 = r[c * 8 + 2 * i] * sc, a1 = r[c * 8 + 2 * i + 1] * sc;
-            nrm = fmaf(a0, a0, nrm);
-            nrm = fmaf(a1, a1, nrm);
-            mx = fmaxf(mx, fmaxf(fabsf(a0), fabsf(a1)));
-            const __half2 h2 = __floats2half2_rn(a0, a1);
-            const float2 hf = __half22float2(h2);
-            hw[i] = *reinterpret_cast<const uint32_t *>(&h2);
-            lw[i] = pack_half2(a0 - hf.x, a1 - hf.y);
-            nz |= lw[i] & 0x7FFF7FFFu;   // any nonzero lo (either sign of zero counts as zero)
+            const float a0 = r[c * 8 + 2 * i], a1 = r[c * 8 + 2 * i + 1];
+            split_half2(a0, a1, hw[i], lw[i]);
+            mx = max3f(mx, fabsf(a0), fabsf(a1));
+            if (NZ)
+                nz |= lw[i] & 0x7FFF7FFFu;   // either sign of zero counts as zero
         }
         const uint32_t off = swz(row, c);
         *reinterpret_cast<uint4 *>(ahi + off) = hv;
         *reinterpret_cast<uint4 *>(alo + off) = lv;
     }
-    // norm parts: ||r'||^2 2^-14 = p0 + p1 + p2
-    const float q = nrm * 0x1p-14f;
-    const float p0 = __half2float(__float2half_rn(q));
-    const float p1 = __half2float(__float2half_rn(q - p0));
-    const float p2 = q - p0 - p1;
-    uint4 w;
-    w.x = pack_half2(1024.0f, 1024.0f);
-    w.y = pack_half2(1024.0f, p0);
-    w.z = pack_half2(p1, p2);
-    w.w = 0u;
-    *reinterpret_cast<uint4 *>(aaug + core16_off(row, 0)) = w;
     *fast = mx < v2::kFastLimit;
-    *norm2 = nrm;
     return nz != 0;
 }
 
@@ -577,9 +601,9 @@ __device__ __forceinline__ void unpack_row64(const uint4 *xr, int dtype, float *
     }
 }
 
-// Exact fp32 scoring of one row against the 256 codewords of a buffer
+// Exact fp32 scoring of one scaled row against the 256 codewords of a buffer
 // (c' = -(hi + lo) / 2), for rows outside the fast path.  Lowest index on ties.
-__device__ __forceinline__ int slow_argmin(const float *r, float sc, const uint8_t *bb)
+__device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb)
 {
     float best = INFINITY;
     int bidx = 0;
@@ -596,8 +620,8 @@ __device__ __forceinline__ int slow_argmin(const float *r, float sc, const uint8
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const float2 h = __half22float2(hh[i]), l = __half22float2(ll[i]);
-                const float t0 = fmaf(r[c * 8 + 2 * i], sc, 0.5f * (h.x + l.x));
-                const float t1 = fmaf(r[c * 8 + 2 * i + 1], sc, 0.5f * (h.y + l.y));
+                const float t0 = r[c * 8 + 2 * i] + 0.5f * (h.x + l.x);
+                const float t1 = r[c * 8 + 2 * i + 1] + 0.5f * (h.y + l.y);
                 d = fmaf(t0, t0, d);
                 d = fmaf(t1, t1, d);
             }
@@ -610,18 +634,47 @@ __device__ __forceinline__ int slow_argmin(const float *r, float sc, const uint8
     return bidx;
 }
 
-// Packed keys: the distance's float bits with the column index in the low 8
-// bits; non-negative floats order as signed integers (a rounding-negative
-// distance sorts first, as the smallest), so one integer min per column finds
-// the smallest distance and its column, the lower column on equal keys.
-// Four independent chains (column j % 4).
-__device__ __forceinline__ void min_keys16(const uint32_t *acc, int col0, int *m)
+// Argmin of one accumulator row (warp-collective: every lane of the warp
+// calls it).  Returns bc * 16 + p, where bc is the first 16-column chunk whose
+// minimum (from tcgen05.ld.red) equals the row minimum and p the position at
+// which the elementwise minimum across chunks equals it.  When the row minimum
+// is held by exactly one chunk and one position, that column is the unique
+// argmin; otherwise (an exact tie, or no finite value) *amb is set and the
+// caller rescans.
+__device__ __forceinline__ int argmin_row(uint32_t trow, bool *amb)
 {
+    float m[16];
+    float best = INFINITY;
+    int bc = 0;
+    bool tie = false;
+#pragma unroll 1
+    for (int c = 0; c < kCodes / 16; c += 2) {
+        float a[16], b[16], ra, rb;
+        tmem_red2x16(trow + c * 16, a, b, ra, rb);
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-        const int key = static_cast<int>((acc[j] & 0xFFFFFF00u) | static_cast<uint32_t>(col0 + j));
-        m[j & 3] = min(m[j & 3], key);
+        for (int p = 0; p < 16; ++p)
+            m[p] = c == 0 ? fminf(a[p], b[p]) : min3f(m[p], a[p], b[p]);
+        if (ra < best) {
+            best = ra;
+            bc = c;
+            tie = false;
+        } else if (ra == best) {
+            tie = true;
+        }
+        if (rb < best) {
+            best = rb;
+            bc = c + 1;
+            tie = false;
+        } else if (rb == best) {
+            tie = true;
+        }
     }
+    uint32_t pm = 0;
+#pragma unroll
+    for (int p = 0; p < 16; ++p)
+        pm |= (m[p] == best ? 1u : 0u) << p;
+    *amb = tie || pm == 0 || (pm & (pm - 1)) != 0;
+    return bc * 16 + (__ffs(pm) - 1);
 }
 
 // Exact argmin of an accumulator row (float compare, lowest index on ties).
@@ -675,10 +728,13 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         fence_mbar_init();
         prefetch_tmap(&tmap);
     }
-    // the norm operands' columns 8..15 are zero for good
-    for (int i = tid; i < 2 * kRows; i += v2::kThreads)
-        *reinterpret_cast<uint4 *>(base + OFF_AAUG + (i / kRows) * A_AUG + core16_off(i % kRows, 1)) =
-            make_uint4(0, 0, 0, 0);
+    // the norm operand of A: columns 0..2 hold 2^10 (times the three parts of
+    // ||c'||^2 2^-10 in B), the rest zero
+    for (int i = tid; i < kRows; i += v2::kThreads) {
+        *reinterpret_cast<uint4 *>(base + OFF_AAUG + core16_off(i, 0)) =
+            make_uint4(pack_half2(1024.0f, 1024.0f), pack_half2(1024.0f, 0.0f), 0u, 0u);
+        *reinterpret_cast<uint4 *>(base + OFF_AAUG + core16_off(i, 1)) = make_uint4(0u, 0u, 0u, 0u);
+    }
     fence_proxy_async_smem();
     if (warp == 1)
         tmem_alloc(sbase + OFF_SLOT, 512);
@@ -726,11 +782,13 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
+            const uint64_t daug = sdesc_core16(sbase + OFF_AAUG);
             int it = 0;
             uint32_t aph[2] = {0, 0};
-            int use[2] = {0, 0};
+            int pc = 0;
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
+                ++pc;
                 for (int s = 0; s < S && ok; ++s, ++it) {
                     const int bi = it & 1;
                     const uint32_t ph = (it >> 1) & 1;
@@ -744,12 +802,13 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                             break;
                         aph[k] ^= 1;
                         tc_fence_after();
-                        const bool lo = lo_stamp[k] == ++use[k];
+                        // the lo operand is nonzero after the first stage; at the
+                        // first stage only if a row's input needs it
+                        const bool lo = s > 0 || lo_stamp[k] == pc;
                         const uint32_t ab = sbase + OFF_A + k * A_SLOT;
                         const uint32_t acc = tmem + k * 256;
-                        // squared norms first (K = 16, no swizzle), then the split dot products
-                        umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(bb + 2 * B_TILE),
-                                 idesc, 0);
+                        // codeword norms first (K = 16, no swizzle), then the split dot products
+                        umma_f16(acc, daug, sdesc_core16(bb + 2 * B_TILE), idesc, 0);
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk) {
                             const uint64_t dah = sdesc_sw128(ab + kk * 32);
@@ -777,18 +836,24 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         const uint32_t trow = tmem + k * 256 + (static_cast<uint32_t>(quad * 32) << 16);
         uint8_t *ahi = base + OFF_A + k * A_SLOT;
         uint8_t *alo = ahi + A_TILE;
-        uint8_t *aaug = base + OFF_AAUG + k * A_AUG;
         uint4 xr[XN];
-        auto load_row = [&](int p) {
+        auto row_src = [&](int p, bool *in) -> const uint4 * {
             const int g = p / pairs_per_group, q = p - g * pairs_per_group;
             const int tile = 2 * q + k;
             const int64_t v = static_cast<int64_t>(tile) * kRows + row;
-            if (tile < tiles && v < nvec) {
-                const int l = g / a.n_heads, h = g - l * a.n_heads;
-                const int64_t b = v / a.n_pos;
-                const int64_t t = a.t0 + (v - b * a.n_pos);
-                const uint4 *src = reinterpret_cast<const uint4 *>(
-                    static_cast<const uint8_t *>(a.x) + (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * ESZ);
+            *in = tile < tiles && v < nvec;
+            if (!*in)
+                return nullptr;
+            const int l = g / a.n_heads, h = g - l * a.n_heads;
+            const int64_t b = v / a.n_pos;
+            const int64_t t = a.t0 + (v - b * a.n_pos);
+            return reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(a.x) +
+                                                   (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * ESZ);
+        };
+        auto load_row = [&](int p) {
+            bool in;
+            const uint4 *src = row_src(p, &in);
+            if (in) {
 #pragma unroll
                 for (int c = 0; c < XN; ++c)
                     xr[c] = __ldg(src + c);
@@ -800,13 +865,22 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         };
         int it = 0;
         uint32_t fph = 0;
-        int use = 0;
-        constexpr bool kPrefetch = ESZ == 2;      // 16-bit rows: 32 registers of prefetch
-        if (kPrefetch && static_cast<int>(blockIdx.x) < n_pairs)
+        int pc = 0;
+        if (static_cast<int>(blockIdx.x) < n_pairs)
             load_row(blockIdx.x);
         for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
-            if (!kPrefetch)
-                load_row(p);
+            const bool has_next = p + static_cast<int>(gridDim.x) < n_pairs;
+            if (has_next) {
+                // pull the next pair's input row into L2 now; it is loaded into
+                // registers once this pair's last argmin no longer needs them
+                bool in;
+                const uint4 *src = row_src(p + gridDim.x, &in);
+                if (in) {
+#pragma unroll
+                    for (int c = 0; c < XN; c += 8)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(src + c));
+                }
+            }
             const int g = p / pairs_per_group, q = p - g * pairs_per_group;
             const int l = g / a.n_heads, h = g - l * a.n_heads;
             const int tile = 2 * q + k;
@@ -815,19 +889,18 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             float r[64];
             unpack_row64<ESZ>(xr, a.dtype, r);
             int e = __ldg(&a.escale[g * S]);
+            scale_row(r, pow2f(-e));
             bool fast;
-            float rn2;
-            bool lo_nz = write_operands(ahi, alo, aaug, row, r, pow2f(-e), &fast, &rn2);
-            ++use;
-            if (lo_nz)
-                lo_stamp[k] = use;
+            ++pc;
+            if (write_operands<true>(ahi, alo, row, r, &fast))
+                lo_stamp[k] = pc;
             fence_proxy_async_smem();
             mbar_arrive(bar(4 + k));
             uint8_t idx[8];
             bool ok = true;
             for (int s = 0; s < S; ++s, ++it) {
                 const int bi = it & 1;
-                const int e_next = s + 1 < S ? __ldg(&a.escale[g * S + s + 1]) : 0;   // in flight during the waits
+                const int e_next = s + 1 < S ? __ldg(&a.escale[g * S + s + 1]) : e;   // in flight during the waits
                 ok = wait_or_abort(bar(6 + k), fph, a.status, abort_flag) &&
                      wait_or_abort(bar(bi), (it >> 1) & 1, a.status, abort_flag);
                 // the tensor-memory loads below are warp-collective: the warp
@@ -837,73 +910,52 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                     break;
                 fph ^= 1;
                 tc_fence_after();
-                if (kPrefetch && s == S - 1 && p + static_cast<int>(gridDim.x) < n_pairs)
-                    load_row(p + gridDim.x);      // next pair's input, in flight during the epilogue
                 const uint8_t *bb = base + OFF_B + bi * B_BUF;
-                int mk[4] = {0x7FFFFFFF, 0x7FFFFFFF, 0x7FFFFFFF, 0x7FFFFFFF};
                 __syncwarp();
-                {
-                    // double-buffered TMEM reads: chunk c + 1 in flight while chunk c is keyed
-                    uint32_t acc0[16], acc1[16];
-                    tmem_ld16_async(trow, acc0);
-                    tmem_wait16(acc0);
-#pragma unroll
-                    for (int ch = 0; ch < kCodes / 16; ch += 2) {
-                        tmem_ld16_async(trow + (ch + 1) * 16, acc1);
-                        min_keys16(acc0, ch * 16, mk);
-                        tmem_wait16(acc1);
-                        if (ch + 2 < kCodes / 16)
-                            tmem_ld16_async(trow + (ch + 2) * 16, acc0);
-                        min_keys16(acc1, (ch + 1) * 16, mk);
-                        if (ch + 2 < kCodes / 16)
-                            tmem_wait16(acc0);
-                    }
-                }
-                const int key = min(min(mk[0], mk[1]), min(mk[2], mk[3]));
-                int bidx = key & 0xFF;
-                // the packed keys only resolve ties within 2^-15 d_min; that is
-                // inside the 1e-4 ||r||^2 tie band while d_min < 3 ||r'||^2
-                const bool rescan = fast && !(__int_as_float(key & 0xFFFFFF00) < 3.0f * rn2);
-                if (__any_sync(0xFFFFFFFFu, rescan)) {   // warp-collective loads: every lane takes part
+                bool amb;
+                int bidx = argmin_row(trow, &amb);
+                if (__any_sync(0xFFFFFFFFu, fast && amb)) {   // warp-collective loads: every lane takes part
                     const int b = exact_argmin_tmem(trow);
-                    if (rescan)
+                    if (amb)
                         bidx = b;
                 }
                 tc_fence_before();
                 if (!fast)
-                    bidx = slow_argmin(r, pow2f(-e), bb);
+                    bidx = slow_argmin(r, bb);
                 idx[s] = static_cast<uint8_t>(bidx);
+                if (s == S - 1 && has_next)
+                    load_row(p + gridDim.x);      // r is dead from here: the next input takes its registers
                 if (s + 1 < S) {
-                    // r <- r - c_bidx  (c = -(hi + lo) 2^(e-1))
-                    const float cs = pow2f(e - 1);
+                    // r' <- r' - c'_bidx = r' + (hi + lo) / 2
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
                         const uint32_t bo = swz(bidx, c);
                         const uint4 hv = *reinterpret_cast<const uint4 *>(bb + bo);
                         const uint4 lv = *reinterpret_cast<const uint4 *>(bb + B_TILE + bo);
-                        const __half2 *hh = reinterpret_cast<const __half2 *>(&hv);
-                        const __half2 *ll = reinterpret_cast<const __half2 *>(&lv);
+                        const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+                        const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
-                            const float2 ca = __half22float2(hh[i]), cb = __half22float2(ll[i]);
-                            r[8 * c + 2 * i] = fmaf(cs, ca.x + cb.x, r[8 * c + 2 * i]);
-                            r[8 * c + 2 * i + 1] = fmaf(cs, ca.y + cb.y, r[8 * c + 2 * i + 1]);
+                            add_half2_halved(hw[i], r[8 * c + 2 * i], r[8 * c + 2 * i + 1]);
+                            add_half2_halved(lw[i], r[8 * c + 2 * i], r[8 * c + 2 * i + 1]);
                         }
+                    }
+                }
+                mbar_arrive(bar(2 + bi));         // this thread is done with the stage buffer
+                if (s + 1 < S) {
+                    if (e_next != e) {            // uniform: one group per CTA at a time
+                        scale_row(r, pow2f(e - e_next));
+                        e = e_next;
                     }
                     if (!valid) {
 #pragma unroll
                         for (int i = 0; i < 64; ++i)
                             r[i] = 0.0f;
                     }
-                    e = e_next;
-                    lo_nz = write_operands(ahi, alo, aaug, row, r, pow2f(-e), &fast, &rn2);
-                    ++use;
-                    if (lo_nz)
-                        lo_stamp[k] = use;
+                    write_operands<false>(ahi, alo, row, r, &fast);
                     fence_proxy_async_smem();
                     mbar_arrive(bar(4 + k));
                 }
-                mbar_arrive(bar(2 + bi));
             }
             if (!ok)
                 break;
