@@ -261,7 +261,7 @@ def roofline(res, peaks, launches_traffic=None):
     dominant = {
         "bound": "tensor", "achieved": rvq_tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
         "frac": rvq_tf / peaks["bf16_tflops"], "traffic": launches_traffic,
-        "kernel": "k_rvq<64> (RVQ assignment), algorithmic 2*64*256 flop per vector-stage, %s peak (fp16 dense = bf16 rate)"
+        "kernel": "k_rvq64 (RVQ assignment), algorithmic 2*64*256 flop per vector-stage, %s peak (fp16 dense = bf16 rate)"
                   % ("of measured" if peaks["source"] == "measured" else "of fallback"),
     }
     return dominant, kernels, dec_bytes, out_bytes

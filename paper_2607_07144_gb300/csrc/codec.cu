@@ -137,6 +137,70 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
     stage_out(dst, sbuf, static_cast<int>(e - b), off);
 }
 
+// The same decode for a whole archive of token records, written out in the
+// planar layout the archive gather reads: per stream, the H key planes
+// (n_rec x S_K indices each, one plane per head) and then the H value planes
+// (n_rec x S_V).  A block decodes 256 spans into shared memory and writes
+// every plane's run of its records with consecutive threads on consecutive
+// bytes; a record cut by the block boundary is completed by the neighbour.
+__global__ void __launch_bounds__(kThreads)
+k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
+                     uint8_t *__restrict__ out, int H, int SK, int SV, const fkv_decconst *__restrict__ dc,
+                     const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    uint8_t *sbuf = dsm + tables_bytes(N, L);
+    const int R = H * (SK + SV);
+    const int64_t n = n_rec * R;
+    const int64_t stream = blockIdx.x / bps;
+    const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
+    const int64_t q0 = s0 * L;
+    const int64_t q1 = min(n, (s0 + kThreads) * L);
+    __syncthreads();
+    const int64_t s = s0 + threadIdx.x;
+    if (s < spans) {
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+        const double2 p = pts[stream * pt_stride + s];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        uint8_t *my = sbuf + threadIdx.x * L;
+        fkvdec::walk(t, X, Y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<uint8_t>(c); });
+        const long long lim = __ldg(&dc->alim[m]);
+        if (X > lim || X < -lim || Y > lim || Y < -lim)
+            atomicOr(status, FKV_ST_CORRUPT);
+    }
+    __syncthreads();
+    // records [rec_lo, rec_lo + nrb) overlap this block's symbols [q0, q1)
+    const int64_t rec_lo = q0 / R;
+    const int nrb = static_cast<int>((q1 - 1) / R - rec_lo + 1);
+    const int nk = H * SK;                       // key indices per record
+    const int runk = nrb * SK, runv = nrb * SV;  // one plane's run of this block's records
+    uint8_t *base = out + stream * n;
+    for (int i = threadIdx.x; i < nrb * R; i += kThreads) {
+        int h, j, st, o;
+        int64_t plane;
+        if (i < H * runk) {
+            h = i / runk;
+            const int w = i - h * runk;
+            j = w / SK;
+            st = w - j * SK;
+            o = h * SK + st;
+            plane = static_cast<int64_t>(h) * n_rec * SK + (rec_lo + j) * SK + st;
+        } else {
+            const int i2 = i - H * runk;
+            h = i2 / runv;
+            const int w = i2 - h * runv;
+            j = w / SV;
+            st = w - j * SV;
+            o = nk + h * SV + st;
+            plane = static_cast<int64_t>(nk) * n_rec + static_cast<int64_t>(h) * n_rec * SV + (rec_lo + j) * SV + st;
+        }
+        const int64_t q = (rec_lo + j) * R + o;
+        if (q >= q0 && q < q1)
+            base[plane] = sbuf[q - q0];
+    }
+}
+
 // Sec. 2 random access: one request per thread, decoding only its span down
 // to the requested offset.
 __global__ void __launch_bounds__(kThreads)
@@ -236,6 +300,28 @@ cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_st
     k_span_decode<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
         reinterpret_cast<const double2 *>(pts), n, pt_stride, spans, static_cast<int>(bps), sym,
         sym_stride, c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
+                                      int64_t pt_stride, uint8_t *out, cudaStream_t st)
+{
+    const int SK = c->cb[0].stages, SV = c->cb[1].stages;
+    const int64_t n = n_rec * c->H * (SK + SV);
+    const int64_t spans = cdiv(n, c->L);
+    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t blocks = n_streams * bps;
+    if (blocks == 0)
+        return cudaSuccess;
+    if (blocks > 0x7FFFFFFF)
+        return cudaErrorInvalidConfiguration;
+    const int smem = tables_bytes(c->N, c->L) + kStageBytes;
+    cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    k_span_decode_planar<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
+        reinterpret_cast<const double2 *>(pts), n_rec, pt_stride, spans, static_cast<int>(bps), out, c->H, SK, SV,
+        c->d_dec, c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 

@@ -100,32 +100,15 @@ extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t
         return FKV_EINVAL;
     }
     // output views are checked before anything is launched
-    const fkv_cache *outs[2] = {k_out, v_out};
-    for (const fkv_cache *c : outs) {
-        if (!c)
-            continue;
-        const bool dt = c->dtype == FKV_F32 || c->dtype == FKV_F16 || c->dtype == FKV_BF16;
-        const int64_t esz = c->dtype == FKV_F32 ? 4 : 2;
-        const int64_t s4[4] = {c->stride_layer, c->stride_batch, c->stride_head, c->stride_pos};
-        bool ok = dt && c->data && c->batch > 0 && t0 + n_rec <= c->seq &&
-                  reinterpret_cast<uintptr_t>(c->data) % 16 == 0;
-        for (int i = 0; i < 4 && ok; ++i)
-            ok = s4[i] >= 0 && (s4[i] * esz) % 16 == 0;
-        if (!ok) {
-            ctx->err = "bad output cache view";
-            return FKV_EINVAL;
-        }
+    if (!check_outputs(ctx, k_out, v_out, n_rec, t0)) {
+        ctx->err = "bad output cache view";
+        return FKV_EINVAL;
     }
     uint8_t *scratch = nullptr;
     int rc = scratch_address(ctx, &scratch);
     if (rc != FKV_OK)
         return rc;
-    const cudaStream_t st = static_cast<cudaStream_t>(stream);
-    cudaError_t e = launch_span_decode(ctx, pts_dev, n_streams, n, pt_stride, scratch, n, st);
-    if (e != cudaSuccess) {
-        ctx->err = std::string("static decode launch: ") + cudaGetErrorString(e);
-        return FKV_ECUDA;
-    }
-    // the gather with the same checks as fkv_rvq_decode, reading the static scratch
-    return fkv_rvq_decode(ctx, scratch, n, n_rec, k_out, v_out, t0, stream);
+    // the same planar decode and gathers as fkv_decode_kv, through the static scratch
+    return decode_archive(ctx, pts_dev, n_streams, n_rec, pt_stride, scratch, k_out, v_out, t0,
+                          static_cast<cudaStream_t>(stream));
 }

@@ -220,6 +220,28 @@ cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 
 }  // namespace
 
+// Both output views (either may be null) hold [t0, t0 + n_rec).
+bool check_outputs(const fkv_ctx *ctx, const fkv_cache *k_out, const fkv_cache *v_out, int64_t n_rec, int64_t t0)
+{
+    const fkv_cache *outs[2] = {k_out, v_out};
+    for (const fkv_cache *c : outs)
+        if (c && (!check_cache(ctx, c) || t0 < 0 || t0 + n_rec > c->seq))
+            return false;
+    return true;
+}
+
+int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
+                   uint8_t *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st)
+{
+    const int64_t stride = n_rec * fkv_record_len(ctx);
+    CK(launch_span_decode_planar(ctx, pts, n_streams, n_rec, pt_stride, scratch, st), "span decode launch");
+    const fkv_cache *outs[2] = {k_out, v_out};
+    for (int kv = 0; kv < 2; ++kv)
+        if (outs[kv])
+            CK(launch_rvq_decode(ctx, kv, scratch, FKV_SYM_PLANAR, stride, n_rec, outs[kv], t0, st), "gather launch");
+    return FKV_OK;
+}
+
 extern "C" {
 
 double fkv_packing_ratio(int N)
@@ -478,18 +500,15 @@ int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, 
     const int64_t R = fkv_record_len(ctx);
     if (stream_stride < n_rec * R)
         return fail(ctx, FKV_EINVAL, "stream stride too small for the records");
-    fkv_cache *outs[2] = {k_out, v_out};
-    for (int kv = 0; kv < 2; ++kv) {
-        if (!outs[kv])
-            continue;
-        if (!check_cache(ctx, outs[kv]) || t0 + n_rec > outs[kv]->seq)
-            return fail(ctx, FKV_EINVAL, "bad output cache view");
-    }
+    if (!check_outputs(ctx, k_out, v_out, n_rec, t0))
+        return fail(ctx, FKV_EINVAL, "bad output cache view");
     if (n_rec == 0)
         return FKV_OK;
+    fkv_cache *outs[2] = {k_out, v_out};
     for (int kv = 0; kv < 2; ++kv)
         if (outs[kv])
-            CK(launch_rvq_decode(ctx, kv, sym_dev, stream_stride, n_rec, outs[kv], t0, as_stream(stream)),
+            CK(launch_rvq_decode(ctx, kv, sym_dev, FKV_SYM_RECORDS, stream_stride, n_rec, outs[kv], t0,
+                                 as_stream(stream)),
                "gather launch");
     return FKV_OK;
 }
@@ -506,11 +525,16 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
         return fail(ctx, FKV_EINVAL, "bad arguments");
     if (k_out && v_out && k_out->batch != v_out->batch)
         return fail(ctx, FKV_EINVAL, "K and V batch differ");
+    // every view is checked before anything is launched
+    if (!check_outputs(ctx, k_out, v_out, n_rec, t0))
+        return fail(ctx, FKV_EINVAL, "bad output cache view");
     if (n_rec == 0)
         return FKV_OK;
     const int64_t R = fkv_record_len(ctx);
     const int64_t n_streams = ref->batch * ctx->Ly;
     const int64_t n = n_rec * R;
+    if (pt_stride < (n + ctx->L - 1) / ctx->L || reinterpret_cast<uintptr_t>(pts_dev) % 16)
+        return fail(ctx, FKV_EINVAL, "bad point stride or alignment");
     const size_t need = static_cast<size_t>(n_streams) * static_cast<size_t>(n);
     if (need > ctx->scratch_bytes) {
         CK(cudaStreamSynchronize(as_stream(stream)), "scratch sync");
@@ -520,10 +544,8 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
         CK(cudaMalloc(&ctx->d_scratch, need), "scratch alloc");
         ctx->scratch_bytes = need;
     }
-    int rc = fkv_span_decode(ctx, pts_dev, n_streams, n, pt_stride, ctx->d_scratch, n, stream);
-    if (rc != FKV_OK)
-        return rc;
-    return fkv_rvq_decode(ctx, ctx->d_scratch, n, n_rec, k_out, v_out, t0, stream);
+    return decode_archive(ctx, pts_dev, n_streams, n_rec, pt_stride, ctx->d_scratch, k_out, v_out, t0,
+                          as_stream(stream));
 }
 
 int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec, int64_t pt_stride,

@@ -76,8 +76,21 @@ cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int6
 // rvq.cu
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
                               uint8_t *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
+// Decoded archive symbols in one of two layouts: the token records of the
+// stream itself (stream_stride bytes per stream), or planar (per stream of
+// n_rec * R bytes: H key planes of n_rec x S_K, then H value planes of
+// n_rec x S_V), which launch_span_decode_planar writes for the gather.
+enum { FKV_SYM_RECORDS = 0, FKV_SYM_PLANAR = 1 };
+cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
+                                      int64_t pt_stride, uint8_t *out, cudaStream_t st);
+// fkv_api.cu: both output views (either may be null) hold [t0, t0 + n_rec);
+// the planar decode of a whole archive into `scratch` (n_streams * n_rec * R
+// bytes) and the K/V gathers from it, once every argument has been checked.
+bool check_outputs(const fkv_ctx *ctx, const fkv_cache *k_out, const fkv_cache *v_out, int64_t n_rec, int64_t t0);
+int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
+                   uint8_t *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st);
 // gather.cu
-cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int64_t stream_stride,
+cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st);
 cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
                            int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,

@@ -2,28 +2,36 @@
 // reconstruction is the sum of the selected centroids), for whole archives
 // and for random record reads (Sec. 2).
 //
-// Whole archive: a block owns one codebook group (layer, head), a slice of
-// the head dimension and a run of vectors; the group's float32 codebooks for
-// that slice sit in shared memory, so HBM sees only the index bytes in and
-// the rebuilt K/V out.  Sums run in float32, stage order, then round to
-// nearest-even into the cache dtype.
+// Whole archive: persistent blocks, each taking an equal share of the
+// (codebook group, dimension slice, vector) work.  A block holds the float32
+// codebooks of one group and one slice of the head dimension (all stages) in
+// shared memory while it works on that slice, so HBM sees only the index
+// bytes in and the rebuilt K/V out.  A thread rebuilds four dimensions (one
+// 16-byte granule of a slice row) of a vector.  Sums run in float32, stage
+// order, then round to nearest-even into the cache dtype.
+//
+// Shared-memory reads are conflict-free for any indices: a slice row spans a
+// multiple of 128 bytes, so its granule g lies in bank group g % 8, and the
+// eight threads of a quarter warp read the eight consecutive granules of one
+// row.  A 16-float slice (two rows per bank line, for more than four stages)
+// permutes its granules by an XOR of the row instead.
 #include "decode_core.cuh"
 
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kSmemBudget = 64 * 1024;   // codebook slice per block
-constexpr int64_t kChunk = 4096;         // vectors per block
+constexpr int kThreads = 512;
+constexpr int kDT = 4;                   // dimensions a thread rebuilds
 
 struct GatherArgs {
-    const uint8_t *sym;
-    int64_t stream_stride, n_rec, batch, t0;
-    int n_layers, n_heads, D, S, R, kv_off;
+    const uint8_t *sym;    // the S indices of (b, l, h, rec) at sym + b ib + l il + h ih + rec ir + ioff
+    int64_t ib, il, ih, ir, ioff;
+    int64_t n_rec, batch, t0;
+    int n_layers, n_heads, D, S;
     const float *cb32;     // [Ly*H][S][256][D]
     void *out;
     int dtype;
     int64_t s_layer, s_batch, s_head, s_pos;
-    int parts, Dp, chunks;
+    int parts, Dp;
 };
 
 __device__ __forceinline__ void store2(void *out, int dtype, int64_t elem, float a, float b)
@@ -38,53 +46,167 @@ __device__ __forceinline__ void store2(void *out, int dtype, int64_t elem, float
     }
 }
 
-__global__ void __launch_bounds__(kThreads) k_gather(const GatherArgs a)
+__device__ __forceinline__ uint32_t pack2(int dtype, float a, float b)
 {
-    extern __shared__ __align__(16) float scb[];   // [S][256][Dp] floats, then offsets and indices
-    const int chunk = blockIdx.x % a.chunks;
-    const int part = (blockIdx.x / a.chunks) % a.parts;
-    const int g = blockIdx.x / (a.chunks * a.parts);
-    const int l = g / a.n_heads, h = g % a.n_heads;
-    const int Dp = a.Dp, S = a.S, D = a.D;
-    const int d0 = part * Dp;
-    // codebook slice -> shared memory (float4 granules; Dp is a multiple of 4)
-    const float *src = a.cb32 + static_cast<int64_t>(g) * S * 256 * D;
-    const int q4 = Dp / 4;
-    for (int i = threadIdx.x; i < S * 256 * q4; i += kThreads) {
-        const int row = i / q4, q = i - row * q4;
-        reinterpret_cast<float4 *>(scb)[i] = __ldg(reinterpret_cast<const float4 *>(src + static_cast<int64_t>(row) * D + d0) + q);
+    if (dtype == FKV_F16) {
+        const __half2 v = __floats2half2_rn(a, b);
+        return *reinterpret_cast<const uint32_t *>(&v);
     }
-    // this block's indices and output offsets -> shared memory (independent
-    // loads, many in flight; 32-bit index arithmetic, checked on the host)
-    int64_t *soff = reinterpret_cast<int64_t *>(scb + S * 256 * Dp);
-    uint8_t *sids = reinterpret_cast<uint8_t *>(soff + kChunk);
-    const int nvec = static_cast<int>(a.batch * a.n_rec);
-    const int v_beg = chunk * static_cast<int>(kChunk);
-    const int nv = min(nvec - v_beg, static_cast<int>(kChunk));
-    const unsigned n_rec = static_cast<unsigned>(a.n_rec);
-    for (int vi = threadIdx.x; vi < nv; vi += kThreads) {
-        const unsigned v = static_cast<unsigned>(v_beg + vi);
-        const unsigned b = v / n_rec;
-        const unsigned rec = v - b * n_rec;
-        const uint8_t *ids = a.sym + (static_cast<int64_t>(b) * a.n_layers + l) * a.stream_stride +
-                             static_cast<int64_t>(rec) * a.R + a.kv_off + h * S;
-        for (int s = 0; s < S; ++s)
-            sids[vi * S + s] = __ldg(ids + s);
-        soff[vi] = l * a.s_layer + b * a.s_batch + h * a.s_head + (a.t0 + rec) * a.s_pos + d0;
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// Four consecutive elements at `elem` (aligned to their size).
+__device__ __forceinline__ void store4(void *out, int dtype, int64_t elem, float4 x)
+{
+    if (dtype == FKV_F32) {
+        *reinterpret_cast<float4 *>(static_cast<float *>(out) + elem) = x;
+        return;
     }
-    __syncthreads();
-    const int tpv = Dp / 2;                  // threads per vector (two dims each)
+    *reinterpret_cast<uint2 *>(static_cast<uint16_t *>(out) + elem) = make_uint2(pack2(dtype, x.x, x.y),
+                                                                                  pack2(dtype, x.z, x.w));
+}
+
+// x0 += c0, x1 += c1 as one packed fp32 add (each lane rounds like a scalar add).
+__device__ __forceinline__ void add2(float &x0, float &x1, float c0, float c1)
+{
+    asm("{\n\t.reg .b64 u, w;\n\t"
+        "mov.b64 u, {%0, %1};\n\t"
+        "mov.b64 w, {%2, %3};\n\t"
+        "add.rn.f32x2 u, u, w;\n\t"
+        "mov.b64 {%0, %1}, u;\n\t}"
+        : "+f"(x0), "+f"(x1)
+        : "f"(c0), "f"(c1));
+}
+
+// The S stage indices of one vector, low byte first: one load of the whole
+// run when it is aligned (WIDE, S = 2, 4 or 8), else bytes.
+template <int S, bool WIDE>
+__device__ __forceinline__ uint64_t load_ids(const uint8_t *p)
+{
+    if (WIDE && S == 4)
+        return __ldg(reinterpret_cast<const unsigned *>(p));
+    if (WIDE && S == 2)
+        return __ldg(reinterpret_cast<const unsigned short *>(p));
+    if (WIDE && S == 8)
+        return __ldg(reinterpret_cast<const unsigned long long *>(p));
+    uint64_t w = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+        w |= static_cast<uint64_t>(__ldg(p + s)) << (8 * s);
+    return w;
+}
+
+template <int S, bool WIDE>
+__global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
+{
+    extern __shared__ __align__(128) float scb[];   // [S][256][Dp] floats
+    const int Dp = a.Dp, D = a.D, parts = a.parts;
+    const int q4 = Dp / 4;                   // 16-byte granules per slice row
+    const bool xor_rows = Dp < 32;           // 16-float rows: XOR-permuted granules
+    const int tpv = Dp / kDT;                // threads per vector
     const int vpi = kThreads / tpv;          // vectors per pass
-    const int dd = (threadIdx.x % tpv) * 2;
-#pragma unroll 2
-    for (int vi = threadIdx.x / tpv; vi < nv; vi += vpi) {
-        float x = 0.0f, y = 0.0f;
-        for (int s = 0; s < S; ++s) {
-            const float2 c = *reinterpret_cast<const float2 *>(scb + (s * 256 + sids[vi * S + s]) * Dp + dd);
-            x += c.x;
-            y += c.y;
+    const int dq = threadIdx.x % tpv;        // this thread's granule of the slice row
+    const int64_t n_rec = a.n_rec;
+    // advancing by vpi vectors: step_r records and step_b sequences, plus one
+    // more sequence when the record wraps
+    const int step_b = static_cast<int>(vpi / n_rec), step_r = static_cast<int>(vpi - step_b * n_rec);
+    const int64_t di_step = step_b * a.ib + step_r * a.ir, di_wrap = a.ib - n_rec * a.ir;
+    const int64_t do_step = step_b * a.s_batch + step_r * a.s_pos, do_wrap = a.s_batch - n_rec * a.s_pos;
+    // this block's share of the work: slots (group * parts + part) * nvec + vector
+    const int64_t nvec = a.batch * n_rec;
+    const int64_t total = static_cast<int64_t>(a.n_layers) * a.n_heads * parts * nvec;
+    int64_t lo = total * blockIdx.x / gridDim.x;
+    const int64_t hi = total * (blockIdx.x + 1) / gridDim.x;
+    int64_t cur = -1;                        // (group, part) whose slice is in shared memory
+    while (lo < hi) {
+        const int64_t gp = lo / nvec;
+        const int64_t v0 = lo - gp * nvec;
+        const int64_t v1 = min(nvec, v0 + (hi - lo));
+        lo += v1 - v0;
+        const int g = static_cast<int>(gp / parts), part = static_cast<int>(gp % parts);
+        const int l = g / a.n_heads, h = g % a.n_heads;
+        const int d0 = part * Dp;
+        if (gp != cur) {
+            // codebook slice -> shared memory: every 16-byte copy in flight, one wait
+            __syncthreads();
+            const float *src = a.cb32 + static_cast<int64_t>(g) * S * 256 * D + d0;
+            for (int i = threadIdx.x; i < S * 256 * q4; i += kThreads) {
+                const int row = i / q4, q = i - row * q4;
+                const int pq = xor_rows ? q ^ ((row >> 1) & 3) : q;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(fkvd::smem_u32(scb + 4 * (row * q4 + pq))),
+                             "l"(src + static_cast<int64_t>(row) * D + 4 * q)
+                             : "memory");
+            }
+            asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+            __syncthreads();
+            cur = gp;
         }
-        store2(a.out, a.dtype, soff[vi] + dd, x, y);
+        const int64_t v = v0 + threadIdx.x / tpv;
+        if (v >= v1)
+            continue;
+        int n_it = static_cast<int>((v1 - v + vpi - 1) / vpi);
+        const int64_t b = v / n_rec;
+        int rec = static_cast<int>(v - b * n_rec);
+        const uint8_t *ip = a.sym + l * a.il + h * a.ih + a.ioff + b * a.ib + rec * a.ir;
+        int64_t oe = l * a.s_layer + h * a.s_head + (a.t0 + rec) * a.s_pos + b * a.s_batch + d0 + dq * kDT;
+        const float4 *row0 = reinterpret_cast<const float4 *>(scb);
+        // kU vectors per round: their index loads are all issued before any is used
+        constexpr int kU = 4;
+        for (; n_it > 0; n_it -= kU) {
+            uint64_t ids[kU];
+            int64_t off[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                ids[u] = u < n_it ? load_ids<S, WIDE>(ip) : 0;
+                off[u] = oe;
+                rec += step_r;
+                ip += di_step;
+                oe += do_step;
+                if (rec >= n_rec) {
+                    rec -= static_cast<int>(n_rec);
+                    ip += di_wrap;
+                    oe += do_wrap;
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                if (u >= n_it)
+                    break;
+                float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+                for (int s = 0; s < S; ++s) {
+                    const int row = s * 256 + static_cast<int>((ids[u] >> (8 * s)) & 0xFF);
+                    const int xq = xor_rows ? (row >> 1) & 3 : 0;
+                    const float4 c = row0[row * q4 + (dq ^ xq)];
+                    add2(x.x, x.y, c.x, c.y);
+                    add2(x.z, x.w, c.z, c.w);
+                }
+                store4(a.out, a.dtype, off[u], x);
+            }
+        }
+    }
+}
+
+template <int S>
+void *gather_kernel(bool wide)
+{
+    if ((S == 2 || S == 4 || S == 8) && wide)
+        return reinterpret_cast<void *>(k_gather<S, true>);
+    return reinterpret_cast<void *>(k_gather<S, false>);
+}
+
+void *gather_kernel_for(int S, bool wide)
+{
+    switch (S) {
+    case 1: return gather_kernel<1>(wide);
+    case 2: return gather_kernel<2>(wide);
+    case 3: return gather_kernel<3>(wide);
+    case 4: return gather_kernel<4>(wide);
+    case 5: return gather_kernel<5>(wide);
+    case 6: return gather_kernel<6>(wide);
+    case 7: return gather_kernel<7>(wide);
+    default: return gather_kernel<8>(wide);
     }
 }
 
@@ -178,22 +300,32 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
 
 }  // namespace
 
-cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int64_t stream_stride,
+cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st)
 {
     const fkv_cbset &cb = c->cb[kv];
     GatherArgs a;
     a.sym = sym;
-    a.stream_stride = stream_stride;
+    const int H = c->H, SK = c->cb[0].stages, S = cb.stages;
+    if (layout == FKV_SYM_PLANAR) {
+        a.il = stream_stride;
+        a.ih = n_rec * S;
+        a.ir = S;
+        a.ioff = kv == 0 ? 0 : static_cast<int64_t>(H) * n_rec * SK;
+    } else {
+        a.il = stream_stride;
+        a.ih = S;
+        a.ir = static_cast<int64_t>(H) * (SK + c->cb[1].stages);
+        a.ioff = kv == 0 ? 0 : static_cast<int64_t>(H) * SK;
+    }
+    a.ib = static_cast<int64_t>(c->Ly) * stream_stride;
     a.n_rec = n_rec;
     a.batch = out->batch;
     a.t0 = t0;
     a.n_layers = c->Ly;
-    a.n_heads = c->H;
+    a.n_heads = H;
     a.D = c->D;
-    a.S = cb.stages;
-    a.R = c->H * (c->cb[0].stages + c->cb[1].stages);
-    a.kv_off = kv == 0 ? 0 : c->H * c->cb[0].stages;
+    a.S = S;
     a.cb32 = cb.cb32;
     a.out = out->data;
     a.dtype = out->dtype;
@@ -201,27 +333,42 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int6
     a.s_batch = out->stride_batch;
     a.s_head = out->stride_head;
     a.s_pos = out->stride_pos;
+    // the widest slice whose codebooks (all stages) fit 128 KB of shared memory,
+    // at least 32 floats wide where possible (one 128-byte bank line per row)
     int parts = 1;
-    while (static_cast<int64_t>(a.S) * 256 * (c->D / parts) * 4 > kSmemBudget && c->D / parts > 4)
+    while (static_cast<int64_t>(a.S) * 256 * (c->D / parts) * 4 > 128 * 1024 && c->D / parts > 16)
         parts *= 2;
     a.parts = parts;
     a.Dp = c->D / parts;
     const int64_t nvec = a.batch * n_rec;
     if (nvec <= 0)
         return cudaSuccess;
-    if (nvec > 0x7FFFFFFF)
-        return cudaErrorInvalidValue;   // vector indices are 32-bit in the kernel
-    const int64_t chunks = (nvec + kChunk - 1) / kChunk;
-    const int64_t blocks = chunks * parts * c->Ly * c->H;
-    if (blocks > 0x7FFFFFFF)
-        return cudaErrorInvalidConfiguration;
-    a.chunks = static_cast<int>(chunks);
-    const size_t smem = static_cast<size_t>(a.S) * 256 * a.Dp * 4 + static_cast<size_t>(kChunk) * (8 + a.S);
-    cudaError_t e = cudaFuncSetAttribute(k_gather, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const size_t smem = static_cast<size_t>(a.S) * 256 * a.Dp * 4;
+    // one load per vector's index run when every run is aligned to its size
+    const int64_t Sv = a.S;
+    const bool wide = reinterpret_cast<uintptr_t>(sym) % Sv == 0 && a.ib % Sv == 0 && a.il % Sv == 0 &&
+                      a.ih % Sv == 0 && a.ir % Sv == 0 && a.ioff % Sv == 0;
+    const void *kern = gather_kernel_for(a.S, wide);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem > 48 * 1024 ? smem : 48 * 1024));
     if (e != cudaSuccess)
         return e;
-    k_gather<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(a);
+    // persistent: as many blocks as fit at once, each taking an equal share
+    int sms = 0, per_sm = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess)
+        return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
+    if (e != cudaSuccess)
+        return e;
+    const int64_t work = static_cast<int64_t>(c->Ly) * c->H * parts * nvec;
+    int64_t blocks = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
+    if (blocks > work)
+        blocks = work;
+    void *args[] = {&a};
+    e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), args, smem, st);
+    if (e != cudaSuccess)
+        return e;
     return cudaGetLastError();
 }
 
