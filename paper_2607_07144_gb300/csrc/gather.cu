@@ -97,15 +97,23 @@ __device__ __forceinline__ uint64_t load_ids(const uint8_t *p)
     return w;
 }
 
+// The slice width: 32 floats (one 128-byte bank line per row) for up to
+// four stages, 16 for more (so that the slice of all stages fits 128 KB).
+__host__ __device__ constexpr int gather_dp(int S)
+{
+    return S <= 4 ? 32 : 16;
+}
+
 template <int S, bool WIDE>
 __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
 {
     extern __shared__ __align__(128) float scb[];   // [S][256][Dp] floats
-    const int Dp = a.Dp, D = a.D, parts = a.parts;
-    const int q4 = Dp / 4;                   // 16-byte granules per slice row
-    const bool xor_rows = Dp < 32;           // 16-float rows: XOR-permuted granules
-    const int tpv = Dp / kDT;                // threads per vector
-    const int vpi = kThreads / tpv;          // vectors per pass
+    constexpr int Dp = gather_dp(S);
+    const int D = a.D, parts = a.parts;
+    constexpr int q4 = Dp / 4;               // 16-byte granules per slice row
+    constexpr bool xor_rows = Dp < 32;       // 16-float rows: XOR-permuted granules
+    constexpr int tpv = Dp / kDT;            // threads per vector
+    constexpr int vpi = kThreads / tpv;      // vectors per pass
     const int dq = threadIdx.x % tpv;        // this thread's granule of the slice row
     const int64_t n_rec = a.n_rec;
     // advancing by vpi vectors: step_r records and step_b sequences, plus one
@@ -152,7 +160,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
         int64_t oe = l * a.s_layer + h * a.s_head + (a.t0 + rec) * a.s_pos + b * a.s_batch + d0 + dq * kDT;
         const float4 *row0 = reinterpret_cast<const float4 *>(scb);
         // kU vectors per round: their index loads are all issued before any is used
-        constexpr int kU = 4;
+        constexpr int kU = 8;
         for (; n_it > 0; n_it -= kU) {
             uint64_t ids[kU];
             int64_t off[kU];
@@ -333,13 +341,9 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int 
     a.s_batch = out->stride_batch;
     a.s_head = out->stride_head;
     a.s_pos = out->stride_pos;
-    // the widest slice whose codebooks (all stages) fit 128 KB of shared memory,
-    // at least 32 floats wide where possible (one 128-byte bank line per row)
-    int parts = 1;
-    while (static_cast<int64_t>(a.S) * 256 * (c->D / parts) * 4 > 128 * 1024 && c->D / parts > 16)
-        parts *= 2;
+    a.Dp = gather_dp(a.S);
+    const int parts = c->D / a.Dp;
     a.parts = parts;
-    a.Dp = c->D / parts;
     const int64_t nvec = a.batch * n_rec;
     if (nvec <= 0)
         return cudaSuccess;
