@@ -107,57 +107,13 @@ __host__ __device__ inline int tables_bytes(int N, int L)
     return (fkvdec::smem_bytes(N, L) + 15) & ~15;
 }
 
-__global__ void __launch_bounds__(kThreads)
-k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
-              uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
-              const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+// Decode 256 spans of one stream (chunk `ck` of the n_streams * bps chunks)
+// into sbuf (one span per thread, symbol i of the chunk at sbuf[i]).
+__device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const double2 *__restrict__ pts, int64_t n,
+                                             int64_t pt_stride, int64_t spans, int64_t stream, int64_t s0,
+                                             uint8_t *sbuf, const fkv_decconst *__restrict__ dc, int L,
+                                             unsigned *status)
 {
-    extern __shared__ __align__(16) uint8_t dsm[];
-    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    uint8_t *sbuf = dsm + tables_bytes(N, L);
-    const int64_t stream = blockIdx.x / bps;
-    const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
-    const int64_t b = s0 * L;
-    const int64_t e = min(n, (s0 + kThreads) * L);
-    uint8_t *dst = sym + stream * sym_stride + b;
-    const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
-    __syncthreads();
-    const int64_t s = s0 + threadIdx.x;
-    if (s < spans) {
-        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
-        const double2 p = pts[stream * pt_stride + s];
-        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
-        uint8_t *my = sbuf + off + threadIdx.x * L;
-        fkvdec::walk(t, X, Y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<uint8_t>(c); });
-        const long long lim = __ldg(&dc->alim[m]);
-        if (X > lim || X < -lim || Y > lim || Y < -lim)
-            atomicOr(status, FKV_ST_CORRUPT);
-    }
-    __syncthreads();
-    stage_out(dst, sbuf, static_cast<int>(e - b), off);
-}
-
-// The same decode for a whole archive of token records, written out in the
-// planar layout the archive gather reads: per stream, the H key planes
-// (n_rec x S_K indices each, one plane per head) and then the H value planes
-// (n_rec x S_V).  A block decodes 256 spans into shared memory and writes
-// every plane's run of its records with consecutive threads on consecutive
-// bytes; a record cut by the block boundary is completed by the neighbour.
-__global__ void __launch_bounds__(kThreads)
-k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
-                     uint8_t *__restrict__ out, int H, int SK, int SV, const fkv_decconst *__restrict__ dc,
-                     const longlong2 *__restrict__ T, int N, int L, unsigned *status)
-{
-    extern __shared__ __align__(16) uint8_t dsm[];
-    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    uint8_t *sbuf = dsm + tables_bytes(N, L);
-    const int R = H * (SK + SV);
-    const int64_t n = n_rec * R;
-    const int64_t stream = blockIdx.x / bps;
-    const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
-    const int64_t q0 = s0 * L;
-    const int64_t q1 = min(n, (s0 + kThreads) * L);
-    __syncthreads();
     const int64_t s = s0 + threadIdx.x;
     if (s < spans) {
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
@@ -169,35 +125,78 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
         if (X > lim || X < -lim || Y > lim || Y < -lim)
             atomicOr(status, FKV_ST_CORRUPT);
     }
+}
+
+// Persistent: a block loads the decoder tables once and walks chunks of 256
+// spans (chunk = stream * bps + span block), blockIdx.x, + gridDim.x, ...
+__global__ void __launch_bounds__(kThreads)
+k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
+              int64_t n_chunks, uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
+              const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    uint8_t *sbuf = dsm + tables_bytes(N, L);
     __syncthreads();
-    // records [rec_lo, rec_lo + nrb) overlap this block's symbols [q0, q1)
-    const int64_t rec_lo = q0 / R;
-    const int nrb = static_cast<int>((q1 - 1) / R - rec_lo + 1);
-    const int nk = H * SK;                       // key indices per record
-    const int runk = nrb * SK, runv = nrb * SV;  // one plane's run of this block's records
-    uint8_t *base = out + stream * n;
-    for (int i = threadIdx.x; i < nrb * R; i += kThreads) {
-        int h, j, st, o;
-        int64_t plane;
-        if (i < H * runk) {
-            h = i / runk;
-            const int w = i - h * runk;
-            j = w / SK;
-            st = w - j * SK;
-            o = h * SK + st;
-            plane = static_cast<int64_t>(h) * n_rec * SK + (rec_lo + j) * SK + st;
-        } else {
-            const int i2 = i - H * runk;
-            h = i2 / runv;
-            const int w = i2 - h * runv;
-            j = w / SV;
-            st = w - j * SV;
-            o = nk + h * SV + st;
-            plane = static_cast<int64_t>(nk) * n_rec + static_cast<int64_t>(h) * n_rec * SV + (rec_lo + j) * SV + st;
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
+        const int64_t stream = ck / bps;
+        const int64_t s0 = (ck - stream * bps) * kThreads;
+        const int64_t b = s0 * L;
+        const int64_t e = min(n, (s0 + kThreads) * L);
+        uint8_t *dst = sym + stream * sym_stride + b;
+        const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
+        decode_chunk(t, pts, n, pt_stride, spans, stream, s0, sbuf + off, dc, L, status);
+        __syncthreads();
+        stage_out(dst, sbuf, static_cast<int>(e - b), off);
+        __syncthreads();
+    }
+}
+
+// The same decode for a whole archive of token records, written out in the
+// planar layout the archive gather reads: per stream, the H key planes
+// (n_rec x S_K indices each, one plane per head) and then the H value planes
+// (n_rec x S_V).  A chunk's records are written plane by plane, a thread per
+// (record, stage) slot of the run, consecutive threads on consecutive bytes; a
+// record cut by the chunk boundary is completed by the neighbouring chunk.
+__global__ void __launch_bounds__(kThreads)
+k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
+                     int64_t n_chunks, uint8_t *__restrict__ out, int H, int SK, int SV,
+                     const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
+                     unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    uint8_t *sbuf = dsm + tables_bytes(N, L);
+    __syncthreads();
+    const int R = H * (SK + SV);
+    const int nk = H * SK;
+    const int64_t n = n_rec * R;
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
+        const int64_t stream = ck / bps;
+        const int64_t s0 = (ck - stream * bps) * kThreads;
+        const int64_t q0 = s0 * L;
+        const int64_t q1 = min(n, (s0 + kThreads) * L);
+        decode_chunk(t, pts, n, pt_stride, spans, stream, s0, sbuf, dc, L, status);
+        __syncthreads();
+        // records [rec_lo, rec_lo + nrb) overlap this chunk's symbols [q0, q1)
+        const int64_t rec_lo = q0 / R;
+        const int nrb = static_cast<int>((q1 - 1) / R - rec_lo + 1);
+        uint8_t *base = out + stream * n;
+        for (int kv = 0; kv < 2; ++kv) {
+            const int S = kv == 0 ? SK : SV;
+            const int o0 = kv == 0 ? 0 : nk;                       // first offset of this half in a record
+            uint8_t *pl = base + (kv == 0 ? 0 : static_cast<int64_t>(nk) * n_rec) + rec_lo * S;
+            for (int i = threadIdx.x; i < nrb * S; i += kThreads) {
+                const int j = i / S, st = i - j * S;               // record j of the chunk, stage st
+                const int64_t qj = (rec_lo + j) * R + o0 + st - q0; // symbol of head 0, relative to q0
+                for (int h = 0; h < H; ++h) {
+                    const int64_t q = qj + h * S;
+                    if (q >= 0 && q < q1 - q0)
+                        pl[static_cast<int64_t>(h) * n_rec * S + i] = sbuf[q];
+                }
+            }
         }
-        const int64_t q = (rec_lo + j) * R + o;
-        if (q >= q0 && q < q1)
-            base[plane] = sbuf[q - q0];
+        __syncthreads();
     }
 }
 
@@ -283,23 +282,45 @@ cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_s
     return cudaGetLastError();
 }
 
+// Persistent decode grid: as many blocks as fit on the GPU at once, at most
+// one per chunk.
+cudaError_t decode_grid(const fkv_ctx *c, const void *kern, int smem, int64_t n_chunks, unsigned *grid)
+{
+    int sms = 0, per_sm = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess)
+        return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
+    if (e != cudaSuccess)
+        return e;
+    int64_t g = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
+    if (g > n_chunks)
+        g = n_chunks;
+    *grid = static_cast<unsigned>(g);
+    return cudaSuccess;
+}
+
 cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
                                int64_t pt_stride, uint8_t *sym, int64_t sym_stride, cudaStream_t st)
 {
     const int64_t spans = cdiv(n, c->L);
     const int64_t bps = cdiv(spans, kThreads);
-    const int64_t blocks = n_streams * bps;
-    if (blocks == 0)
+    const int64_t n_chunks = n_streams * bps;
+    if (n_chunks == 0)
         return cudaSuccess;
-    if (blocks > 0x7FFFFFFF)
+    if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
     const int smem = tables_bytes(c->N, c->L) + kStageBytes;
     cudaError_t e = cudaFuncSetAttribute(k_span_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
-    k_span_decode<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
-        reinterpret_cast<const double2 *>(pts), n, pt_stride, spans, static_cast<int>(bps), sym,
-        sym_stride, c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode), smem, n_chunks, &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_span_decode<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
+                                                static_cast<int>(bps), n_chunks, sym, sym_stride, c->d_dec,
+                                                c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 
@@ -310,18 +331,22 @@ cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64
     const int64_t n = n_rec * c->H * (SK + SV);
     const int64_t spans = cdiv(n, c->L);
     const int64_t bps = cdiv(spans, kThreads);
-    const int64_t blocks = n_streams * bps;
-    if (blocks == 0)
+    const int64_t n_chunks = n_streams * bps;
+    if (n_chunks == 0)
         return cudaSuccess;
-    if (blocks > 0x7FFFFFFF)
+    if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
     const int smem = tables_bytes(c->N, c->L) + kStageBytes;
     cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
-    k_span_decode_planar<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
-        reinterpret_cast<const double2 *>(pts), n_rec, pt_stride, spans, static_cast<int>(bps), out, c->H, SK, SV,
-        c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar), smem, n_chunks, &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_span_decode_planar<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec, pt_stride,
+                                                       spans, static_cast<int>(bps), n_chunks, out, c->H, SK, SV,
+                                                       c->d_dec, c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 
