@@ -53,6 +53,12 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
+# DRAM bytes (read + write) per k_rvq64 launch of this workload, the mean of
+# the key launch (197,753,856) and the value launch (171,147,008) from one ncu
+# capture of the current kernel (profiles/k_rvq64_gpt2_full_cache.md); set it
+# to None whenever that kernel changes until it is captured again.
+RVQ_DRAM_BYTES_PER_LAUNCH = 184450432
+
 # FP64 add/mul issue rate measured on this machine's GB300 (1.6 per clock per SM,
 # 504 Gop/s at the clock of that run); the span encoder is bound by it.
 FP64_OPS_PER_CLK_SM = 1.6
@@ -387,12 +393,7 @@ def main():
         torch.distributed.destroy_process_group()
         return
     peaks = load_peaks()
-    traffic = None
-    tp = os.path.join(ROOT, "profiles", "rvq_traffic.json")
-    if os.path.exists(tp):
-        with open(tp) as f:
-            traffic = json.load(f).get("bytes_per_launch_pair")
-    dominant, kernels, dec_bytes, out_bytes = roofline(res, peaks, traffic)
+    dominant, kernels, dec_bytes, out_bytes = roofline(res, peaks, RVQ_DRAM_BYTES_PER_LAUNCH)
     units = res["units"] * world
     value = units / (ms * 1e-3)
     cpu = None
