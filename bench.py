@@ -146,7 +146,7 @@ def run_gpu(args, rank, world, local_rank):
     names = ["rvq_k", "rvq_v", "span_encode", "append_rvq", "append", "decode_kv", "read_kv"]
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
 
-    def step(record=False):
+    def step(record=False, K=K, V=V, st=st, out=out):
         e = iter(ev) if record else None
         rec_ = (lambda: next(e).record(stream)) if record else (lambda: None)
         rec_()
@@ -200,36 +200,66 @@ def run_gpu(args, rank, world, local_rank):
     clk = clocks.stop()
     ok = ctx.sync_status() == 0
 
-    # end-to-end through the public API with host buffers
+    # end-to-end through the public API with host buffers: every step copies
+    # its K/V caches in from pinned host memory and reads its result (the
+    # archive points and the random-read records) back; steps are pipelined
+    # over three streams (copy in, compute, copy out) with double-buffered
+    # device inputs and archives, as a serving loop would run them
     e2e = None
     if not args.no_e2e:
         Kh = K.cpu().pin_memory()
         Vh = V.cpu().pin_memory()
-        Krh = torch.empty_like(Kh).pin_memory()
-        Vrh = torch.empty_like(Vh).pin_memory()
-        ptsh = torch.empty((ns, ctx.n_spans(n_rec * R), 2), dtype=torch.float64).pin_memory()
+        n_sp = ctx.n_spans(n_rec * R)
+        Kd, Vd = [K, torch.empty_like(K)], [V, torch.empty_like(V)]
+        sts = [st, fkv.Streams(ctx, ns, capacity=n_rec * R)]
+        outs = [out, torch.empty_like(out)]
+        ptsh = [torch.empty((ns, n_sp, 2), dtype=torch.float64).pin_memory() for _ in range(2)]
+        outh = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+        s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+        free = [None, None]      # compute is done with buffer b's inputs
+        read = [None, None]      # buffer b's results are back on the host
 
-        def step_e2e():
-            K.copy_(Kh, non_blocking=True)
-            V.copy_(Vh, non_blocking=True)
-            step()
-            ptsh.copy_(st.points()[:, :ptsh.shape[1]], non_blocking=True)
-            Krh.copy_(Kr, non_blocking=True)
-            Vrh.copy_(Vr, non_blocking=True)
-        for _ in range(2):
-            step_e2e()
+        def step_e2e(i, after=None):
+            b = i % 2
+            with torch.cuda.stream(s_in):
+                if after is not None:
+                    s_in.wait_event(after)
+                if free[b] is not None:
+                    s_in.wait_event(free[b])
+                Kd[b].copy_(Kh, non_blocking=True)
+                Vd[b].copy_(Vh, non_blocking=True)
+                ev_in = torch.cuda.Event()
+                ev_in.record(s_in)
+            stream.wait_event(ev_in)
+            if read[b] is not None:
+                stream.wait_event(read[b])
+            step(K=Kd[b], V=Vd[b], st=sts[b], out=outs[b])
+            done = torch.cuda.Event()
+            done.record(stream)
+            free[b] = done
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(done)
+                ptsh[b].copy_(sts[b].points()[:, :n_sp], non_blocking=True)
+                outh[b].copy_(outs[b], non_blocking=True)
+                back = torch.cuda.Event()
+                back.record(s_out)
+                read[b] = back
+        for i in range(2):
+            step_e2e(i)
         torch.cuda.synchronize()
         if world > 1:
             torch.distributed.barrier()
         s2, t2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s2.record(stream)
-        for _ in range(args.steps):
-            step_e2e()
+        for i in range(args.steps):
+            step_e2e(i, after=s2 if i < 2 else None)
+        for b in range(2):
+            stream.wait_event(read[b])
         t2.record(stream)
         torch.cuda.synchronize()
         e2e_ms = s2.elapsed_time(t2) / args.steps
         h2d = Kh.numel() * Kh.element_size() * 2
-        d2h = ptsh.numel() * 8 + Krh.numel() * Krh.element_size() * 2
+        d2h = ptsh[0].numel() * 8 + outh[0].numel() * outh[0].element_size()
         e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
 
     units = ns * n_rec
