@@ -254,3 +254,44 @@ def indices_from_records(stream, n_heads: int, stages_k: int, stages_v: int):
     k = s[:, :n_heads * stages_k].reshape(P, n_heads, stages_k).transpose(1, 0, 2)
     v = s[:, n_heads * stages_k:].reshape(P, n_heads, stages_v).transpose(1, 0, 2)
     return np.ascontiguousarray(k), np.ascontiguousarray(v)
+
+
+# ------------------------------------------------------- suffix retrieval ---
+def suffix_radius2(r: float, qlen: int) -> float:
+    """Sec. 5: positions sharing an l-symbol suffix have points within 2 r^l of
+    each other.  The squared radius (2 r^l)^2 of the retrieval ball, with r^l
+    formed by l successive binary64 multiplications."""
+    rl = 1.0
+    for _ in range(int(qlen)):
+        rl = rl * r
+    t = 2.0 * rl
+    return t * t
+
+
+def suffix_search(pts, n: int, query, N: int, r: float, L: int):
+    """Sec. 5 retrieval on one span-anchored stream, done in place.
+
+    The query (l symbols, 1 <= l <= L) is encoded from the origin by the Sec. 1
+    map.  A stored point within the 2 r^l ball is a candidate; a candidate is a
+    match when its span's last l symbols equal the query, which the decode
+    verifies.  A span-end point carries only its own span's symbols, so a span
+    shorter than l is never a candidate.  Returns (matches, candidates): sorted
+    int64 arrays of span indices."""
+    qs = np.asarray(query, dtype=np.int32).ravel()
+    l = qs.size
+    if l < 1 or l > L:
+        raise ValueError("query length outside [1, L]")
+    p = np.ascontiguousarray(pts, dtype=np.float64).reshape(-1, 2)
+    spans = p.shape[0]
+    if spans != n_spans(n, L):
+        raise ValueError("point count does not match n and L")
+    q = span_encode(qs, N, r, l)[0]                  # the query's point, one span from the origin
+    m = np.minimum(L, int(n) - np.arange(spans, dtype=np.int64) * L)
+    dx = p[:, 0] - q[0]
+    dy = p[:, 1] - q[1]
+    d2 = dx * dx + dy * dy
+    cand = np.nonzero((m >= l) & (d2 <= suffix_radius2(r, l)))[0].astype(np.int64)
+    sym, _, _ = span_decode(p, n, N, r, L)
+    match = [u for u in cand
+             if np.array_equal(sym[u * L + m[u] - l:u * L + m[u]], qs)]
+    return np.asarray(match, dtype=np.int64), cand
