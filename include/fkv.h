@@ -143,6 +143,26 @@ int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int6
 int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
              const int64_t *req_dev, int64_t n_req, uint8_t *out_dev, void *stream);
 
+/* Sec. 5: in-place suffix retrieval over the stored points, with no
+ * decompression of the archive.  query (host memory) holds qlen symbols,
+ * 1 <= qlen <= span_len, each < N; it is encoded from the origin by the Sec. 1
+ * map.  Two positions sharing an l-symbol suffix have points within 2 r^l, so
+ * every stored point of a span of at least qlen symbols with
+ * |p - q|^2 <= (2 r^qlen)^2 (binary64, r^qlen by successive multiplication)
+ * is a candidate; a candidate is verified by walking its span back qlen steps
+ * with the exact decoder and matches when those symbols are the query.  A
+ * span-end point carries only its own span's symbols, so a match means: the
+ * last qlen symbols of span (stream, span) equal the query.
+ *   match_dev: int64 [cap][2], device, caller-owned: (stream, span) of each
+ *              match, in no particular order; only the first cap are written;
+ *   counts_dev: int64 [2], device, caller-owned: [0] the number of matches
+ *              (all of them, even past cap), [1] the number of candidates.
+ * Points laid out as in fkv_span_encode.  Returns FKV_EINVAL for a bad qlen,
+ * a symbol >= N, a null or misaligned pointer or a negative size. */
+int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
+                      const uint8_t *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
+                      void *stream);
+
 /* -------------------------------------------------- K/V archive path ---- */
 
 /* A K or V cache tensor on the device: head vectors of `dim` contiguous

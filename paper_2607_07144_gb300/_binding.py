@@ -56,6 +56,7 @@ SIGNATURES = {
     "fkv_span_encode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
     "fkv_span_decode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
     "fkv_read": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _P]),
+    "fkv_suffix_search": (_I, [_P, _P, _I64, _I64, _I64, _P, _I, _P, _I64, _P, _P]),
     "fkv_record_len": (_I, [_P]),
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
@@ -214,6 +215,23 @@ class Context:
         self._check(lib().fkv_read(self._h, _ptr(pts), pts.shape[0], n, _rows(pts, 2), _ptr(req), req.shape[0],
                                    _ptr(out), _stream(stream)))
         return out
+
+    def suffix_search(self, pts: torch.Tensor, n: int, query, cap: int = 1 << 16, match: torch.Tensor = None,
+                      counts: torch.Tensor = None, stream=None):
+        """Sec. 5 in-place retrieval: spans whose last len(query) symbols equal
+        the query.  Returns (match int64 [min(count, cap), 2] = (stream, span)
+        in no particular order, number of matches, number of candidates); reads
+        the two counts back (a device synchronisation on `stream`)."""
+        q = np.ascontiguousarray(np.asarray(query, dtype=np.uint8).ravel())
+        if match is None:
+            match = torch.empty((max(cap, 1), 2), dtype=torch.int64, device=pts.device)
+        if counts is None:
+            counts = torch.empty(2, dtype=torch.int64, device=pts.device)
+        self._check(lib().fkv_suffix_search(self._h, _ptr(pts), pts.shape[0], n, _rows(pts, 2),
+                                            q.ctypes.data_as(ctypes.c_void_p), q.size, _ptr(match), cap,
+                                            _ptr(counts), _stream(stream)))
+        c = counts.cpu().tolist()
+        return match[:min(c[0], cap)], c[0], c[1]
 
     def rvq_encode(self, kv: int, x: torch.Tensor, t0: int, t1: int, sym: torch.Tensor, rec0: int = 0, stream=None):
         """x: cache [layers, batch, heads, seq, dim]; sym: uint8 [batch*layers, >= (rec0+t1-t0)*R]."""

@@ -200,6 +200,70 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
     }
 }
 
+// Sec. 5 retrieval in place.  Persistent blocks scan their share of the
+// stored points against the query's point (the query encoded from the
+// origin by the Sec. 1 map, bit for bit as the encoder would): a point of a
+// span of at least l symbols inside the 2 r^l ball is a candidate, and a
+// candidate is walked back l steps by the exact decoder; it matches when
+// those symbols are the query.  Matches are appended (stream, span) in any
+// order; counts[0] counts matches (all of them, even past cap), counts[1]
+// candidates.
+struct SuffixQuery {
+    uint8_t sym[kMaxSpan];
+    int len;
+};
+
+__global__ void __launch_bounds__(kThreads)
+k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride, int64_t spans,
+                const SuffixQuery qy, double thr2, const double2 *__restrict__ V, double r,
+                const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
+                long long *__restrict__ out, long long cap, unsigned long long *__restrict__ counts)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    __shared__ double2 q_s;
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    if (threadIdx.x == 0)
+        q_s = encode_span(qy.sym, qy.len, V, r, 0.0, 0.0);
+    __syncthreads();
+    const double2 q = q_s;
+    const int l = qy.len;
+    // this block's contiguous share of the n_streams * spans points, walked
+    // kThreads apart per thread without division
+    const int64_t total = n_streams * spans;
+    const int64_t hi = total * (blockIdx.x + 1) / gridDim.x;
+    int64_t g = total * blockIdx.x / gridDim.x + threadIdx.x;
+    int64_t stream = g / spans, u = g - stream * spans;
+    const int64_t step_s = kThreads / spans, step_u = kThreads - step_s * spans;
+    for (; g < hi; g += kThreads) {
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+        if (m >= l) {
+            const double2 p = pts[stream * pt_stride + u];
+            const double dx = __dsub_rn(p.x, q.x), dy = __dsub_rn(p.y, q.y);
+            const double d2 = __dadd_rn(__dmul_rn(dx, dx), __dmul_rn(dy, dy));
+            if (d2 <= thr2) {
+                atomicAdd(&counts[1], 1ull);
+                long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+                bool eq = true;
+                // step j recovers the span's symbol m - 1 - j, the query's l - 1 - j
+                fkvdec::walk(t, X, Y, l, [&](int j, int c) { eq = eq && c == qy.sym[l - 1 - j]; });
+                if (eq) {
+                    const unsigned long long slot = atomicAdd(&counts[0], 1ull);
+                    if (static_cast<long long>(slot) < cap) {
+                        out[2 * slot] = stream;
+                        out[2 * slot + 1] = u;
+                    }
+                }
+            }
+        }
+        u += step_u;
+        stream += step_s;
+        if (u >= spans) {
+            u -= spans;
+            ++stream;
+        }
+    }
+}
+
 // Sec. 2 random access: one request per thread, decoding only its span down
 // to the requested offset.
 __global__ void __launch_bounds__(kThreads)
@@ -347,6 +411,42 @@ cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64
     k_span_decode_planar<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec, pt_stride,
                                                        spans, static_cast<int>(bps), n_chunks, out, c->H, SK, SV,
                                                        c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                                 int64_t pt_stride, const uint8_t *query, int qlen, int64_t *out, int64_t cap,
+                                 int64_t *counts, cudaStream_t st)
+{
+    cudaError_t e = cudaMemsetAsync(counts, 0, 2 * sizeof(int64_t), st);
+    if (e != cudaSuccess)
+        return e;
+    const int64_t spans = cdiv(n, c->L);
+    if (n_streams * spans == 0)
+        return cudaSuccess;
+    SuffixQuery qy;
+    for (int i = 0; i < kMaxSpan; ++i)
+        qy.sym[i] = i < qlen ? query[i] : 0;
+    qy.len = qlen;
+    // (2 r^l)^2 with r^l by l successive multiplications (the Sec. 5 ball)
+    double rl = 1.0;
+    for (int i = 0; i < qlen; ++i)
+        rl = rl * c->r;
+    const double t = 2.0 * rl;
+    const double thr2 = t * t;
+    const int smem = tables_bytes(c->N, c->L);
+    e = cudaFuncSetAttribute(k_suffix_search, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_suffix_search), smem, cdiv(n_streams * spans, kThreads),
+                    &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_suffix_search<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride,
+                                                  spans, qy, thr2, c->d_V, c->r, c->d_dec, c->d_T, c->N, c->L,
+                                                  reinterpret_cast<long long *>(out), cap,
+                                                  reinterpret_cast<unsigned long long *>(counts));
     return cudaGetLastError();
 }
 

@@ -458,6 +458,31 @@ int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, 
     return FKV_OK;
 }
 
+int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
+                      const uint8_t *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
+                      void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_streams < 0 || n < 0 || cap < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (qlen < 1 || qlen > ctx->L || !query)
+        return fail(ctx, FKV_EINVAL, "query length outside [1, span_len]");
+    for (int i = 0; i < qlen; ++i)
+        if (query[i] >= ctx->N)
+            return fail(ctx, FKV_EINVAL, "query symbol outside the alphabet");
+    if (!counts_dev || (cap > 0 && !match_dev) || (n_streams > 0 && n > 0 && !pts_dev) ||
+        pt_stride < (n + ctx->L - 1) / ctx->L)
+        return fail(ctx, FKV_EINVAL, "bad pointer or stride");
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16 || reinterpret_cast<uintptr_t>(match_dev) % 8 ||
+        reinterpret_cast<uintptr_t>(counts_dev) % 8)
+        return fail(ctx, FKV_EINVAL, "misaligned buffer");
+    CK(launch_suffix_search(ctx, pts_dev, n_streams, n, pt_stride, query, qlen, match_dev, cap, counts_dev,
+                            as_stream(stream)),
+       "suffix search launch");
+    return FKV_OK;
+}
+
 int fkv_record_len(const fkv_ctx *ctx)
 {
     if (!ctx || !ctx->has_cb)

@@ -70,6 +70,9 @@ cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_st
 cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
                         int64_t pt_stride, const int64_t *req, int64_t n_req, uint8_t *out,
                         cudaStream_t st);
+cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                                 int64_t pt_stride, const uint8_t *query, int qlen, int64_t *out, int64_t cap,
+                                 int64_t *counts, cudaStream_t st);
 cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
                           int64_t n_old, const uint8_t *sym, int64_t m, int64_t sym_stride,
                           cudaStream_t st);
