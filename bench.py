@@ -262,9 +262,38 @@ def run_gpu(args, rank, world, local_rank):
         d2h = ptsh[0].numel() * 8 + outh[0].numel() * outh[0].element_size()
         e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
 
+    # Sec. 5 in-place suffix retrieval, measured on its own workload: four
+    # streams of 2^28 seeded uniform symbols (N = 256, span 6; 2.86 GB of
+    # stored points, far above L2), one 6-symbol query planted from a span
+    suffix = None
+    if not args.no_suffix:
+        sctx = fkv.Context(256)
+        s_sym = synth.gpu_symbols(256, "uniform", 4, 1 << 28, device=dev)
+        s_pts = sctx.span_encode(s_sym)
+        q = s_sym[2, 6 * 1000:6 * 1001].cpu().numpy()
+        del s_sym
+        match = torch.empty((1 << 16, 2), dtype=torch.int64, device=dev)
+        counts = torch.empty(2, dtype=torch.int64, device=dev)
+        for _ in range(3):
+            sctx.suffix_search(s_pts, 1 << 28, q, match=match, counts=counts)
+        reps = 10
+        ss, se = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ss.record(stream)
+        for _ in range(reps):
+            fkv._binding.lib().fkv_suffix_search(
+                sctx.handle, fkv._binding._ptr(s_pts), 4, 1 << 28, s_pts.shape[1], q.ctypes.data_as(
+                    fkv._binding.ctypes.c_void_p), q.size, fkv._binding._ptr(match), match.shape[0],
+                fkv._binding._ptr(counts), fkv._binding._stream(stream))
+        se.record(stream)
+        torch.cuda.synchronize()
+        c = counts.cpu().tolist()
+        suffix = {"ms": ss.elapsed_time(se) / reps, "bytes": s_pts.numel() * 8, "matches": c[0], "candidates": c[1],
+                  "workload": "4 streams x 2^28 uniform symbols, N=256, span 6, one 6-symbol query"}
+        del s_pts, sctx
+
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
-                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L)
+                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix)
 
 
 def roofline(res, peaks, launches_traffic=None):
@@ -368,6 +397,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="fkv", choices=["fkv", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-suffix", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -424,6 +454,12 @@ def main():
         return
     peaks = load_peaks()
     dominant, kernels, dec_bytes, out_bytes = roofline(res, peaks, RVQ_DRAM_BYTES_PER_LAUNCH)
+    if res["suffix"]:
+        sx = res["suffix"]
+        gbs = sx["bytes"] / (sx["ms"] * 1e-3) / 1e9
+        kernels["suffix_search (Sec. 5)"] = {"bound": "hbm", "ms": sx["ms"], "achieved_gbs": gbs,
+                                             "frac": gbs / peaks["hbm_gbs"], "matches": sx["matches"],
+                                             "candidates": sx["candidates"], "workload": sx["workload"]}
     units = res["units"] * world
     value = units / (ms * 1e-3)
     cpu = None

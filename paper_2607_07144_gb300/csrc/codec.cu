@@ -207,7 +207,11 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
 // candidate is walked back l steps by the exact decoder; it matches when
 // those symbols are the query.  Matches are appended (stream, span) in any
 // order; counts[0] counts matches (all of them, even past cap), counts[1]
-// candidates.
+// candidates.  GB300's FP64 pipe would bound a binary64 distance test of every
+// point, so each point first passes an integer box test: the ball's bounding
+// box, rounded outward, in an order-preserving integer image of binary64; only
+// points inside the box take the binary64 test.  Four points per thread are
+// in flight at once.
 struct SuffixQuery {
     uint8_t sym[kMaxSpan];
     int len;
@@ -215,17 +219,29 @@ struct SuffixQuery {
 
 __global__ void __launch_bounds__(kThreads)
 k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride, int64_t spans,
-                const SuffixQuery qy, double thr2, const double2 *__restrict__ V, double r,
+                const SuffixQuery qy, double thr, double thr2, const double2 *__restrict__ V, double r,
                 const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
                 long long *__restrict__ out, long long cap, unsigned long long *__restrict__ counts)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     __shared__ double2 q_s;
+    __shared__ long long box_s[4];
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    if (threadIdx.x == 0)
-        q_s = encode_span(qy.sym, qy.len, V, r, 0.0, 0.0);
+    // order-preserving integer image of a binary64 value (signed compare)
+    auto okey = [](long long b) { return b ^ ((b >> 63) & 0x7FFFFFFFFFFFFFFFll); };
+    if (threadIdx.x == 0) {
+        const double2 qq = encode_span(qy.sym, qy.len, V, r, 0.0, 0.0);
+        q_s = qq;
+        const double tb = __dmul_ru(thr, 1.0 + 0x1p-40);           // the box contains the ball
+        box_s[0] = okey(__double_as_longlong(__dsub_rd(qq.x, tb)));
+        box_s[1] = okey(__double_as_longlong(__dadd_ru(qq.x, tb)));
+        box_s[2] = okey(__double_as_longlong(__dsub_rd(qq.y, tb)));
+        box_s[3] = okey(__double_as_longlong(__dadd_ru(qq.y, tb)));
+    }
     __syncthreads();
     const double2 q = q_s;
+    const long long bx0 = box_s[0], bx1 = box_s[1], by0 = box_s[2], by1 = box_s[3];
+    const longlong2 *pk = reinterpret_cast<const longlong2 *>(pts);
     const int l = qy.len;
     // this block's contiguous share of the n_streams * spans points, walked
     // kThreads apart per thread without division
@@ -234,32 +250,51 @@ k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, i
     int64_t g = total * blockIdx.x / gridDim.x + threadIdx.x;
     int64_t stream = g / spans, u = g - stream * spans;
     const int64_t step_s = kThreads / spans, step_u = kThreads - step_s * spans;
-    for (; g < hi; g += kThreads) {
-        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
-        if (m >= l) {
-            const double2 p = pts[stream * pt_stride + u];
-            const double dx = __dsub_rn(p.x, q.x), dy = __dsub_rn(p.y, q.y);
-            const double d2 = __dadd_rn(__dmul_rn(dx, dx), __dmul_rn(dy, dy));
-            if (d2 <= thr2) {
-                atomicAdd(&counts[1], 1ull);
-                long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
-                bool eq = true;
-                // step j recovers the span's symbol m - 1 - j, the query's l - 1 - j
-                fkvdec::walk(t, X, Y, l, [&](int j, int c) { eq = eq && c == qy.sym[l - 1 - j]; });
-                if (eq) {
-                    const unsigned long long slot = atomicAdd(&counts[0], 1ull);
-                    if (static_cast<long long>(slot) < cap) {
-                        out[2 * slot] = stream;
-                        out[2 * slot + 1] = u;
+    constexpr int kU = 4;
+    while (g < hi) {
+        longlong2 pb[kU];
+        int64_t su[kU], uu[kU];
+        bool live[kU];
+#pragma unroll
+        for (int i = 0; i < kU; ++i) {
+            live[i] = g < hi;
+            su[i] = stream;
+            uu[i] = u;
+            if (live[i])
+                pb[i] = pk[stream * pt_stride + u];
+            g += kThreads;
+            u += step_u;
+            stream += step_s;
+            if (u >= spans) {
+                u -= spans;
+                ++stream;
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kU; ++i) {
+            if (!live[i])
+                break;
+            const int m = static_cast<int>(min(static_cast<int64_t>(L), n - uu[i] * L));
+            const long long kx = okey(pb[i].x), ky = okey(pb[i].y);
+            if (m >= l && kx >= bx0 && kx <= bx1 && ky >= by0 && ky <= by1) {
+                const double2 p = make_double2(__longlong_as_double(pb[i].x), __longlong_as_double(pb[i].y));
+                const double dx = __dsub_rn(p.x, q.x), dy = __dsub_rn(p.y, q.y);
+                const double d2 = __dadd_rn(__dmul_rn(dx, dx), __dmul_rn(dy, dy));
+                if (d2 <= thr2) {
+                    atomicAdd(&counts[1], 1ull);
+                    long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+                    bool eq = true;
+                    // step j recovers the span's symbol m - 1 - j, the query's l - 1 - j
+                    fkvdec::walk(t, X, Y, l, [&](int j, int c) { eq = eq && c == qy.sym[l - 1 - j]; });
+                    if (eq) {
+                        const unsigned long long slot = atomicAdd(&counts[0], 1ull);
+                        if (static_cast<long long>(slot) < cap) {
+                            out[2 * slot] = su[i];
+                            out[2 * slot + 1] = uu[i];
+                        }
                     }
                 }
             }
-        }
-        u += step_u;
-        stream += step_s;
-        if (u >= spans) {
-            u -= spans;
-            ++stream;
         }
     }
 }
@@ -444,7 +479,7 @@ cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_
     if (e != cudaSuccess)
         return e;
     k_suffix_search<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride,
-                                                  spans, qy, thr2, c->d_V, c->r, c->d_dec, c->d_T, c->N, c->L,
+                                                  spans, qy, t, thr2, c->d_V, c->r, c->d_dec, c->d_T, c->N, c->L,
                                                   reinterpret_cast<long long *>(out), cap,
                                                   reinterpret_cast<unsigned long long *>(counts));
     return cudaGetLastError();
