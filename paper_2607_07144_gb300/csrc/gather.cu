@@ -19,7 +19,7 @@
 
 namespace {
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 1024;
 constexpr int kDT = 4;                   // dimensions a thread rebuilds
 
 struct GatherArgs {
@@ -97,11 +97,12 @@ __device__ __forceinline__ uint64_t load_ids(const uint8_t *p)
     return w;
 }
 
-// The slice width: 32 floats (one 128-byte bank line per row) for up to
-// four stages, 16 for more (so that the slice of all stages fits 128 KB).
+// The slice width: the widest of 64, 32 or 16 floats whose codebook slice
+// (all stages) fits 128 KB; rows of 64 or 32 floats span whole 128-byte bank
+// lines.
 __host__ __device__ constexpr int gather_dp(int S)
 {
-    return S <= 4 ? 32 : 16;
+    return S <= 2 ? 64 : (S <= 4 ? 32 : 16);
 }
 
 template <int S, bool WIDE>
@@ -160,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
         int64_t oe = l * a.s_layer + h * a.s_head + (a.t0 + rec) * a.s_pos + b * a.s_batch + d0 + dq * kDT;
         const float4 *row0 = reinterpret_cast<const float4 *>(scb);
         // kU vectors per round: their index loads are all issued before any is used
-        constexpr int kU = 8;
+        constexpr int kU = 4;
         for (; n_it > 0; n_it -= kU) {
             uint64_t ids[kU];
             int64_t off[kU];
