@@ -19,7 +19,10 @@
  *     recorded in a per-context status word; fkv_sync_status() waits for the
  *     stream and returns (and clears) it.  Kernels never trap.
  *   - A context is not thread-safe: calls on one context must be serialised.
- *   - Symbols are uint8: alphabets N <= 256 (the paper's k = 256 codebooks).
+ *   - Symbols are uint8 for alphabets N <= 256 (the paper's k = 256
+ *     codebooks) and uint16 (native byte order, 2-byte aligned) for
+ *     256 < N <= 1024 (the k = 1024 rows of Table 2); fkv_symbol_bytes()
+ *     gives the width.  Symbol strides and counts are in symbols.
  *   - A point is two float64 (x, y), 16 bytes; one point per span.
  */
 #ifndef FKV_H
@@ -56,7 +59,7 @@ typedef struct fkv_streams fkv_streams;
  * touching ratio of adjacent cells,
  *     r_N = 1 / (2 (1 + sum_{k=1}^{floor(N/4)} cos(2 pi k / N))),
  * which is exactly 1/2 for N = 3 and N = 4 as the paper states.
- * Returns 0.0 for N < 3 or N > 256. */
+ * Returns 0.0 for N < 3 or N > 1024. */
 double fkv_packing_ratio(int N);
 
 /* Sec. 1: inversion amplifies rounding by 1/r per step, so one IEEE-754
@@ -82,9 +85,10 @@ typedef struct {
     const float *v;
 } fkv_codebooks;
 
-/* Create a context for alphabet size N in [3, 256], contraction ratio r in
+/* Create a context for alphabet size N in [3, 1024], contraction ratio r in
  * (0, r_N] (r_N per fkv_packing_ratio, with a relative slack of 1e-12) and
- * span length span_len in [1, fkv_max_span_len(r)] (Sec. 1).  cb may be NULL
+ * span length span_len in [1, fkv_max_span_len(r)] (Sec. 1; at most 5
+ * symbols for N = 1024).  cb may be NULL
  * for a symbol-only codec; when given, its codebooks are copied to the
  * current CUDA device (the caller keeps ownership of cb's arrays) and N must
  * be 256.  The context owns the vertex table V(c) (Sec. 1: unit circumradius,
@@ -102,6 +106,10 @@ int fkv_vertices(const fkv_ctx *ctx, double *out);
 /* Alphabet size, ratio and span length of a context (any pointer may be NULL). */
 int fkv_params(const fkv_ctx *ctx, int *N, double *r, int *span_len);
 
+/* Bytes per symbol in every symbol array of the context: 1 (uint8) for
+ * N <= 256, 2 (uint16) above; 0 for a NULL context. */
+int fkv_symbol_bytes(const fkv_ctx *ctx);
+
 /* Last error message of the context (static storage, never NULL). */
 const char *fkv_last_error(const fkv_ctx *ctx);
 
@@ -113,7 +121,7 @@ int fkv_sync_status(fkv_ctx *ctx, void *stream);
 
 /* Sec. 1 / Sec. 2: span-parallel encoding.  Encodes n_streams streams of n
  * symbols each.  Stream i's symbols are sym_dev[i * sym_stride + k],
- * k < n (sym_stride in bytes, >= n).  Every span of span_len symbols starts
+ * k < n (sym_dev typed per fkv_symbol_bytes; sym_stride in symbols, >= n).  Every span of span_len symbols starts
  * at the anchor (0, 0) and applies, per symbol c, p <- V(c) + r (p - V(c))
  * as the binary64 sequence d = p - V(c), t = r * d, p = V(c) + t (no FMA);
  * the point after the span's last symbol is stored.  The last span of a
@@ -121,7 +129,7 @@ int fkv_sync_status(fkv_ctx *ctx, void *stream);
  * span j is the point at pts_dev[2 * (i * pt_stride + j)] (x then y),
  * pt_stride (in points) >= ceil(n / span_len).  Symbols >= N are reported as
  * FKV_ECORRUPT in the status word (their span's point is written as NaN). */
-int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int64_t n,
+int fkv_span_encode(fkv_ctx *ctx, const void *sym_dev, int64_t n_streams, int64_t n,
                     int64_t sym_stride, double *pts_dev, int64_t pt_stride, void *stream);
 
 /* Sec. 1: span-parallel decoding, the inverse of fkv_span_encode (same
@@ -132,24 +140,25 @@ int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int
  * back at the anchor: a residual above 2^-4 in either coordinate sets
  * FKV_ECORRUPT in the status word (the symbols are still written). */
 int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n,
-                    int64_t pt_stride, uint8_t *sym_dev, int64_t sym_stride, void *stream);
+                    int64_t pt_stride, void *sym_dev, int64_t sym_stride, void *stream);
 
 /* Sec. 2, Table 1: O(1) random access.  For each request q < n_req,
  * req_dev[2q] = stream index, req_dev[2q + 1] = symbol position, writes the
  * symbol at that position to out_dev[q] by decoding only the span holding it
  * (at most span_len backward steps).  Points laid out as in fkv_span_encode.
- * A request outside [0, n_streams) x [0, n) writes 0xFF to out_dev[q] and
+ * out_dev holds symbols of the context's width.  A request outside
+ * [0, n_streams) x [0, n) writes all ones (0xFF or 0xFFFF) to out_dev[q] and
  * sets FKV_ECORRUPT. */
 int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
-             const int64_t *req_dev, int64_t n_req, uint8_t *out_dev, void *stream);
+             const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
 
 /* Sec. 5: in-place suffix retrieval over the stored points, with no
- * decompression of the archive.  query (host memory) holds qlen symbols,
- * 1 <= qlen <= span_len, each < N; it is encoded from the origin by the Sec. 1
- * map.  Two positions sharing an l-symbol suffix have points within 2 r^l, so
- * every stored point of a span of at least qlen symbols with
- * |p - q|^2 <= (2 r^qlen)^2 (binary64, r^qlen by successive multiplication)
- * is a candidate; a candidate is verified by walking its span back qlen steps
+ * decompression of the archive.  query (host memory, the context's symbol
+ * width) holds qlen symbols, 1 <= qlen <= span_len, each < N; it is encoded
+ * from the origin by the Sec. 1 map.  Two positions sharing an l-symbol
+ * suffix have points within 2 r^l, so every stored point of a span of at
+ * least qlen symbols with |p - q|^2 <= (2 r^qlen)^2 (binary64, r^qlen by
+ * successive multiplication) is a candidate; a candidate is verified by walking its span back qlen steps
  * with the exact decoder and matches when those symbols are the query.  A
  * span-end point carries only its own span's symbols, so a match means: the
  * last qlen symbols of span (stream, span) equal the query.
@@ -160,7 +169,7 @@ int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, 
  * Points laid out as in fkv_span_encode.  Returns FKV_EINVAL for a bad qlen,
  * a symbol >= N, a null or misaligned pointer or a negative size. */
 int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
-                      const uint8_t *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
+                      const void *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
                       void *stream);
 
 /* -------------------------------------------------- K/V archive path ---- */
@@ -269,7 +278,7 @@ int fkv_streams_info(const fkv_streams *s, int64_t *n_streams, int64_t *length,
  * later spans start at the anchor; sealed spans are never touched.  The
  * result is bit-identical to encoding the extended streams from scratch.
  * The point buffer grows geometrically (x2) when full, with a device copy. */
-int fkv_append(fkv_ctx *ctx, fkv_streams *s, const uint8_t *sym_dev, int64_t m,
+int fkv_append(fkv_ctx *ctx, fkv_streams *s, const void *sym_dev, int64_t m,
                int64_t sym_stride, void *stream);
 
 /* Checkpoint: copy a stream set's length and points to host memory

@@ -51,6 +51,7 @@ SIGNATURES = {
     "fkv_destroy": (_I, [_P]),
     "fkv_vertices": (_I, [_P, _P]),
     "fkv_params": (_I, [_P, _P, _P, _P]),
+    "fkv_symbol_bytes": (_I, [_P]),
     "fkv_last_error": (ctypes.c_char_p, [_P]),
     "fkv_sync_status": (_I, [_P, _P]),
     "fkv_span_encode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
@@ -155,11 +156,20 @@ class Context:
         self._cb_arrays = None
         if rc != OK:
             raise FkvError(rc, "fkv_create(N=%d, r=%r, span_len=%d) rejected" % (self.N, self.r, self.L))
+        # symbols are uint8 up to N = 256, uint16 above; torch.int16 holds the
+        # uint16 symbols bit for bit (every symbol is below 1024)
+        self.sym_bytes = L.fkv_symbol_bytes(self._h)
+        self.sym_dtype = torch.uint8 if self.sym_bytes == 1 else torch.int16
 
     # -- plumbing
     def _check(self, rc):
         if rc != OK:
             raise FkvError(rc, lib().fkv_last_error(self._h).decode())
+
+    def _sym(self, t: torch.Tensor) -> torch.Tensor:
+        if t.element_size() != self.sym_bytes:
+            raise ValueError("symbols of this context are %d-byte integers, got %s" % (self.sym_bytes, t.dtype))
+        return t
 
     def close(self):
         if self._h:
@@ -192,8 +202,8 @@ class Context:
         return (int(n) + self.L - 1) // self.L
 
     def span_encode(self, sym: torch.Tensor, pts: torch.Tensor = None, stream=None) -> torch.Tensor:
-        """sym uint8 [n_streams, n] -> pts float64 [n_streams, spans, 2]."""
-        ns, n = sym.shape
+        """sym [n_streams, n] (sym_dtype) -> pts float64 [n_streams, spans, 2]."""
+        ns, n = self._sym(sym).shape
         if pts is None:
             pts = torch.empty((ns, self.n_spans(n), 2), dtype=torch.float64, device=sym.device)
         self._check(lib().fkv_span_encode(self._h, _ptr(sym), ns, n, _rows(sym), _ptr(pts), _rows(pts, 2),
@@ -203,15 +213,17 @@ class Context:
     def span_decode(self, pts: torch.Tensor, n: int, sym: torch.Tensor = None, stream=None) -> torch.Tensor:
         ns = pts.shape[0]
         if sym is None:
-            sym = torch.empty((ns, n), dtype=torch.uint8, device=pts.device)
+            sym = torch.empty((ns, n), dtype=self.sym_dtype, device=pts.device)
+        self._sym(sym)
         self._check(lib().fkv_span_decode(self._h, _ptr(pts), ns, n, _rows(pts, 2), _ptr(sym), _rows(sym),
                                           _stream(stream)))
         return sym
 
     def read(self, pts: torch.Tensor, n: int, req: torch.Tensor, out: torch.Tensor = None, stream=None):
-        """req int64 [n_req, 2] = (stream, position) -> uint8 [n_req]."""
+        """req int64 [n_req, 2] = (stream, position) -> symbols [n_req] (sym_dtype)."""
         if out is None:
-            out = torch.empty(req.shape[0], dtype=torch.uint8, device=pts.device)
+            out = torch.empty(req.shape[0], dtype=self.sym_dtype, device=pts.device)
+        self._sym(out)
         self._check(lib().fkv_read(self._h, _ptr(pts), pts.shape[0], n, _rows(pts, 2), _ptr(req), req.shape[0],
                                    _ptr(out), _stream(stream)))
         return out
@@ -222,7 +234,10 @@ class Context:
         the query.  Returns (match int64 [min(count, cap), 2] = (stream, span)
         in no particular order, number of matches, number of candidates); reads
         the two counts back (a device synchronisation on `stream`)."""
-        q = np.ascontiguousarray(np.asarray(query, dtype=np.uint8).ravel())
+        q = np.asarray(query).ravel()
+        if q.size and (q.min() < 0 or q.max() >= 1 << (8 * self.sym_bytes)):
+            raise ValueError("query symbol does not fit the symbol width")
+        q = np.ascontiguousarray(q.astype(np.uint8 if self.sym_bytes == 1 else np.uint16))
         if match is None:
             match = torch.empty((max(cap, 1), 2), dtype=torch.int64, device=pts.device)
         if counts is None:
@@ -312,7 +327,8 @@ class Streams:
         lib().fkv_streams_reset(self._h)
 
     def append(self, sym: torch.Tensor, stream=None):
-        """sym uint8 [n_streams, m]."""
+        """sym [n_streams, m] of the context's sym_dtype."""
+        self.ctx._sym(sym)
         self.ctx._check(lib().fkv_append(self.ctx.handle, self._h, _ptr(sym), sym.shape[1], _rows(sym),
                                          _stream(stream)))
 

@@ -15,7 +15,13 @@ namespace {
 
 constexpr int kThreads = 256;   // spans per block
 constexpr int kMaxSpan = 44;    // floor(44 / log2(1/r)) with r <= 1/2
-constexpr int kStageBytes = kThreads * kMaxSpan + 32;
+
+// Symbols are uint8 for alphabets N <= 256 and uint16 up to FKV_MAX_N; every
+// kernel that touches symbols is instantiated for both.
+template <typename Sym>
+__host__ __device__ constexpr int stage_bytes() { return kThreads * kMaxSpan * static_cast<int>(sizeof(Sym)) + 32; }
+template <typename Sym>
+__host__ __device__ constexpr int vtab_len() { return sizeof(Sym) == 1 ? 256 : FKV_MAX_N; }
 
 // Copy len bytes from global src into shared buf so that buf[off + i] =
 // src[i], off = src mod 16: aligned 16-byte vectors inside the range, single
@@ -60,11 +66,15 @@ __device__ __forceinline__ void stage_out(uint8_t *dst, const uint8_t *buf, int 
 }
 
 // Sec. 1 forward map for one span from the anchor (0, 0), binary64, no FMA.
-__device__ __forceinline__ double2 encode_span(const uint8_t *s, int m, const double2 *sV, double r,
+// A symbol >= N takes a NaN vertex, so its span's point comes out NaN.
+template <typename Sym>
+__device__ __forceinline__ double2 encode_span(const Sym *s, int m, const double2 *sV, int N, double r,
                                                double x, double y)
 {
     for (int k = 0; k < m; ++k) {
-        const double2 v = sV[s[k]];
+        const unsigned c = s[k];
+        const double2 v = c < static_cast<unsigned>(N) ? sV[c] : make_double2(__longlong_as_double(-1ll),
+                                                                              __longlong_as_double(-1ll));
         const double dx = __dsub_rn(x, v.x);
         const double dy = __dsub_rn(y, v.y);
         const double tx = __dmul_rn(r, dx);
@@ -75,24 +85,28 @@ __device__ __forceinline__ double2 encode_span(const uint8_t *s, int m, const do
     return make_double2(x, y);
 }
 
+template <typename Sym>
 __global__ void __launch_bounds__(kThreads)
-k_span_encode(const uint8_t *__restrict__ sym, int64_t n, int64_t sym_stride, int64_t spans, int bps,
-              double2 *__restrict__ pts, int64_t pt_stride, const double2 *__restrict__ V, double r, int L,
+k_span_encode(const Sym *__restrict__ sym, int64_t n, int64_t sym_stride, int64_t spans, int bps,
+              double2 *__restrict__ pts, int64_t pt_stride, const double2 *__restrict__ V, int N, double r, int L,
               unsigned *status)
 {
-    __shared__ __align__(16) uint8_t sbuf[kStageBytes];
-    __shared__ double2 sV[256];
+    __shared__ __align__(16) uint8_t sbuf[stage_bytes<Sym>()];
+    __shared__ double2 sV[vtab_len<Sym>()];
     const int64_t stream = blockIdx.x / bps;
     const int64_t s0 = static_cast<int64_t>(blockIdx.x % bps) * kThreads;
-    sV[threadIdx.x] = V[threadIdx.x];
+    for (int i = threadIdx.x; i < N; i += kThreads)
+        sV[i] = V[i];
     const int64_t b = s0 * L;
     const int64_t e = min(n, (s0 + kThreads) * L);
-    const int off = stage_in(sbuf, sym + stream * sym_stride + b, static_cast<int>(e - b));
+    const int off = stage_in(sbuf, reinterpret_cast<const uint8_t *>(sym + stream * sym_stride + b),
+                             static_cast<int>(e - b) * static_cast<int>(sizeof(Sym)));
     __syncthreads();
     const int64_t s = s0 + threadIdx.x;
     if (s < spans) {
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
-        const double2 p = encode_span(sbuf + off + threadIdx.x * L, m, sV, r, 0.0, 0.0);
+        const Sym *my = reinterpret_cast<const Sym *>(sbuf + off) + threadIdx.x * L;
+        const double2 p = encode_span(my, m, sV, N, r, 0.0, 0.0);
         if (isnan(p.x))   // a symbol >= N reads a NaN vertex
             atomicOr(status, FKV_ST_CORRUPT);
         pts[stream * pt_stride + s] = p;
@@ -109,9 +123,10 @@ __host__ __device__ inline int tables_bytes(int N, int L)
 
 // Decode 256 spans of one stream (chunk `ck` of the n_streams * bps chunks)
 // into sbuf (one span per thread, symbol i of the chunk at sbuf[i]).
+template <typename Sym>
 __device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const double2 *__restrict__ pts, int64_t n,
                                              int64_t pt_stride, int64_t spans, int64_t stream, int64_t s0,
-                                             uint8_t *sbuf, const fkv_decconst *__restrict__ dc, int L,
+                                             Sym *sbuf, const fkv_decconst *__restrict__ dc, int L,
                                              unsigned *status)
 {
     const int64_t s = s0 + threadIdx.x;
@@ -119,8 +134,8 @@ __device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const doub
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
         const double2 p = pts[stream * pt_stride + s];
         long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
-        uint8_t *my = sbuf + threadIdx.x * L;
-        fkvdec::walk(t, X, Y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<uint8_t>(c); });
+        Sym *my = sbuf + threadIdx.x * L;
+        fkvdec::walk(t, X, Y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<Sym>(c); });
         const long long lim = __ldg(&dc->alim[m]);
         if (X > lim || X < -lim || Y > lim || Y < -lim)
             atomicOr(status, FKV_ST_CORRUPT);
@@ -129,9 +144,10 @@ __device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const doub
 
 // Persistent: a block loads the decoder tables once and walks chunks of 256
 // spans (chunk = stream * bps + span block), blockIdx.x, + gridDim.x, ...
+template <typename Sym>
 __global__ void __launch_bounds__(kThreads)
 k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
-              int64_t n_chunks, uint8_t *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
+              int64_t n_chunks, Sym *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
               const longlong2 *__restrict__ T, int N, int L, unsigned *status)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
@@ -143,11 +159,11 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
         const int64_t s0 = (ck - stream * bps) * kThreads;
         const int64_t b = s0 * L;
         const int64_t e = min(n, (s0 + kThreads) * L);
-        uint8_t *dst = sym + stream * sym_stride + b;
+        uint8_t *dst = reinterpret_cast<uint8_t *>(sym + stream * sym_stride + b);
         const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
-        decode_chunk(t, pts, n, pt_stride, spans, stream, s0, sbuf + off, dc, L, status);
+        decode_chunk(t, pts, n, pt_stride, spans, stream, s0, reinterpret_cast<Sym *>(sbuf + off), dc, L, status);
         __syncthreads();
-        stage_out(dst, sbuf, static_cast<int>(e - b), off);
+        stage_out(dst, sbuf, static_cast<int>(e - b) * static_cast<int>(sizeof(Sym)), off);
         __syncthreads();
     }
 }
@@ -158,15 +174,16 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
 // (n_rec x S_V).  A chunk's records are written plane by plane, a thread per
 // (record, stage) slot of the run, consecutive threads on consecutive bytes; a
 // record cut by the chunk boundary is completed by the neighbouring chunk.
+template <typename Sym>
 __global__ void __launch_bounds__(kThreads)
 k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
-                     int64_t n_chunks, uint8_t *__restrict__ out, int H, int SK, int SV,
+                     int64_t n_chunks, Sym *__restrict__ out, int H, int SK, int SV,
                      const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
                      unsigned *status)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    uint8_t *sbuf = dsm + tables_bytes(N, L);
+    Sym *sbuf = reinterpret_cast<Sym *>(dsm + tables_bytes(N, L));
     __syncthreads();
     const int R = H * (SK + SV);
     const int nk = H * SK;
@@ -181,11 +198,11 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
         // records [rec_lo, rec_lo + nrb) overlap this chunk's symbols [q0, q1)
         const int64_t rec_lo = q0 / R;
         const int nrb = static_cast<int>((q1 - 1) / R - rec_lo + 1);
-        uint8_t *base = out + stream * n;
+        Sym *base = out + stream * n;
         for (int kv = 0; kv < 2; ++kv) {
             const int S = kv == 0 ? SK : SV;
             const int o0 = kv == 0 ? 0 : nk;                       // first offset of this half in a record
-            uint8_t *pl = base + (kv == 0 ? 0 : static_cast<int64_t>(nk) * n_rec) + rec_lo * S;
+            Sym *pl = base + (kv == 0 ? 0 : static_cast<int64_t>(nk) * n_rec) + rec_lo * S;
             for (int i = threadIdx.x; i < nrb * S; i += kThreads) {
                 const int j = i / S, st = i - j * S;               // record j of the chunk, stage st
                 const int64_t qj = (rec_lo + j) * R + o0 + st - q0; // symbol of head 0, relative to q0
@@ -213,7 +230,7 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
 // points inside the box take the binary64 test.  Four points per thread are
 // in flight at once.
 struct SuffixQuery {
-    uint8_t sym[kMaxSpan];
+    uint16_t sym[kMaxSpan];
     int len;
 };
 
@@ -230,7 +247,7 @@ k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, i
     // order-preserving integer image of a binary64 value (signed compare)
     auto okey = [](long long b) { return b ^ ((b >> 63) & 0x7FFFFFFFFFFFFFFFll); };
     if (threadIdx.x == 0) {
-        const double2 qq = encode_span(qy.sym, qy.len, V, r, 0.0, 0.0);
+        const double2 qq = encode_span(qy.sym, qy.len, V, N, r, 0.0, 0.0);
         q_s = qq;
         const double tb = __dmul_ru(thr, 1.0 + 0x1p-40);           // the box contains the ball
         box_s[0] = okey(__double_as_longlong(__dsub_rd(qq.x, tb)));
@@ -301,9 +318,10 @@ k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, i
 
 // Sec. 2 random access: one request per thread, decoding only its span down
 // to the requested offset.
+template <typename Sym>
 __global__ void __launch_bounds__(kThreads)
 k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride,
-       const int64_t *__restrict__ req, int64_t n_req, uint8_t *__restrict__ out,
+       const int64_t *__restrict__ req, int64_t n_req, Sym *__restrict__ out,
        const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L, unsigned *status)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
@@ -314,7 +332,7 @@ k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt
         return;
     const int64_t st = req[2 * q], pos = req[2 * q + 1];
     if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
-        out[q] = 0xFF;
+        out[q] = static_cast<Sym>(~0u);
         atomicOr(status, FKV_ST_CORRUPT);
         return;
     }
@@ -325,19 +343,21 @@ k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt
     long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
     int sym = 0;
     fkvdec::walk(t, X, Y, m - o, [&](int j, int c) { sym = c; });
-    out[q] = static_cast<uint8_t>(sym);
+    out[q] = static_cast<Sym>(sym);
 }
 
 // Sec. 2 append: one thread per (stream, span touched by the new symbols).
 // The first touched span continues from the stored tail point when the old
 // length is not a multiple of L; every later span starts at the anchor.
+template <typename Sym>
 __global__ void __launch_bounds__(kThreads)
 k_append(double2 *__restrict__ pts, int64_t n_streams, int64_t pt_stride, int64_t n_old,
-         const uint8_t *__restrict__ sym, int64_t m, int64_t sym_stride, int64_t u_first, int64_t cnt,
-         const double2 *__restrict__ V, double r, int L, unsigned *status)
+         const Sym *__restrict__ sym, int64_t m, int64_t sym_stride, int64_t u_first, int64_t cnt,
+         const double2 *__restrict__ V, int N, double r, int L, unsigned *status)
 {
-    __shared__ double2 sV[256];
-    sV[threadIdx.x] = V[threadIdx.x];
+    __shared__ double2 sV[vtab_len<Sym>()];
+    for (int i = threadIdx.x; i < N; i += kThreads)
+        sV[i] = V[i];
     __syncthreads();
     const int64_t t = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
     if (t >= n_streams * cnt)
@@ -350,12 +370,12 @@ k_append(double2 *__restrict__ pts, int64_t n_streams, int64_t pt_stride, int64_
     double2 p = make_double2(0.0, 0.0);
     if (u * L < n_old)
         p = pts[stream * pt_stride + u];
-    uint8_t s[kMaxSpan];
-    const uint8_t *src = sym + stream * sym_stride + (b - n_old);
+    Sym s[kMaxSpan];
+    const Sym *src = sym + stream * sym_stride + (b - n_old);
     const int len = static_cast<int>(e - b);
     for (int k = 0; k < len; ++k)
         s[k] = src[k];
-    p = encode_span(s, len, sV, r, p.x, p.y);
+    p = encode_span(s, len, sV, N, r, p.x, p.y);
     if (isnan(p.x))
         atomicOr(status, FKV_ST_CORRUPT);
     pts[stream * pt_stride + u] = p;
@@ -365,8 +385,17 @@ inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
 }  // namespace
 
-cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_streams, int64_t n,
-                               int64_t sym_stride, double *pts, int64_t pt_stride, cudaStream_t st)
+// Symbol width of a context: 1 byte for N <= 256, else 2.
+inline bool wide(const fkv_ctx *c) { return c->N > 256; }
+
+int codec_smem_bytes(int N, int L)
+{
+    return tables_bytes(N, L) + (N > 256 ? stage_bytes<uint16_t>() : stage_bytes<uint8_t>());
+}
+
+template <typename Sym>
+cudaError_t span_encode_t(const fkv_ctx *c, const Sym *sym, int64_t n_streams, int64_t n, int64_t sym_stride,
+                          double *pts, int64_t pt_stride, cudaStream_t st)
 {
     const int64_t spans = cdiv(n, c->L);
     const int64_t bps = cdiv(spans, kThreads);
@@ -375,10 +404,18 @@ cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_s
         return cudaSuccess;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    k_span_encode<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+    k_span_encode<Sym><<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
         sym, n, sym_stride, spans, static_cast<int>(bps), reinterpret_cast<double2 *>(pts), pt_stride,
-        c->d_V, c->r, c->L, c->d_status);
+        c->d_V, c->N, c->r, c->L, c->d_status);
     return cudaGetLastError();
+}
+
+cudaError_t launch_span_encode(const fkv_ctx *c, const void *sym, int64_t n_streams, int64_t n,
+                               int64_t sym_stride, double *pts, int64_t pt_stride, cudaStream_t st)
+{
+    if (wide(c))
+        return span_encode_t(c, static_cast<const uint16_t *>(sym), n_streams, n, sym_stride, pts, pt_stride, st);
+    return span_encode_t(c, static_cast<const uint8_t *>(sym), n_streams, n, sym_stride, pts, pt_stride, st);
 }
 
 // Persistent decode grid: as many blocks as fit on the GPU at once, at most
@@ -399,8 +436,9 @@ cudaError_t decode_grid(const fkv_ctx *c, const void *kern, int smem, int64_t n_
     return cudaSuccess;
 }
 
-cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                               int64_t pt_stride, uint8_t *sym, int64_t sym_stride, cudaStream_t st)
+template <typename Sym>
+cudaError_t span_decode_t(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
+                          Sym *sym, int64_t sym_stride, cudaStream_t st)
 {
     const int64_t spans = cdiv(n, c->L);
     const int64_t bps = cdiv(spans, kThreads);
@@ -409,22 +447,31 @@ cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_st
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + kStageBytes;
-    cudaError_t e = cudaFuncSetAttribute(k_span_decode, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    const int smem = tables_bytes(c->N, c->L) + stage_bytes<Sym>();
+    cudaError_t e = cudaFuncSetAttribute(k_span_decode<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
     unsigned grid = 0;
-    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode), smem, n_chunks, &grid);
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode<Sym>), smem, n_chunks, &grid);
     if (e != cudaSuccess)
         return e;
-    k_span_decode<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
-                                                static_cast<int>(bps), n_chunks, sym, sym_stride, c->d_dec,
-                                                c->d_T, c->N, c->L, c->d_status);
+    k_span_decode<Sym><<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
+                                                     static_cast<int>(bps), n_chunks, sym, sym_stride, c->d_dec,
+                                                     c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 
-cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
-                                      int64_t pt_stride, uint8_t *out, cudaStream_t st)
+cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                               int64_t pt_stride, void *sym, int64_t sym_stride, cudaStream_t st)
+{
+    if (wide(c))
+        return span_decode_t(c, pts, n_streams, n, pt_stride, static_cast<uint16_t *>(sym), sym_stride, st);
+    return span_decode_t(c, pts, n_streams, n, pt_stride, static_cast<uint8_t *>(sym), sym_stride, st);
+}
+
+template <typename Sym>
+cudaError_t span_decode_planar_t(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
+                                 int64_t pt_stride, Sym *out, cudaStream_t st)
 {
     const int SK = c->cb[0].stages, SV = c->cb[1].stages;
     const int64_t n = n_rec * c->H * (SK + SV);
@@ -435,22 +482,32 @@ cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + kStageBytes;
-    cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    const int smem = tables_bytes(c->N, c->L) + stage_bytes<Sym>();
+    cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         smem);
     if (e != cudaSuccess)
         return e;
     unsigned grid = 0;
-    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar), smem, n_chunks, &grid);
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar<Sym>), smem, n_chunks, &grid);
     if (e != cudaSuccess)
         return e;
-    k_span_decode_planar<<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec, pt_stride,
-                                                       spans, static_cast<int>(bps), n_chunks, out, c->H, SK, SV,
-                                                       c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    k_span_decode_planar<Sym><<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec,
+                                                            pt_stride, spans, static_cast<int>(bps), n_chunks,
+                                                            out, c->H, SK, SV, c->d_dec, c->d_T, c->N, c->L,
+                                                            c->d_status);
     return cudaGetLastError();
 }
 
+cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
+                                      int64_t pt_stride, void *out, cudaStream_t st)
+{
+    if (wide(c))
+        return span_decode_planar_t(c, pts, n_streams, n_rec, pt_stride, static_cast<uint16_t *>(out), st);
+    return span_decode_planar_t(c, pts, n_streams, n_rec, pt_stride, static_cast<uint8_t *>(out), st);
+}
+
 cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                                 int64_t pt_stride, const uint8_t *query, int qlen, int64_t *out, int64_t cap,
+                                 int64_t pt_stride, const uint16_t *query, int qlen, int64_t *out, int64_t cap,
                                  int64_t *counts, cudaStream_t st)
 {
     cudaError_t e = cudaMemsetAsync(counts, 0, 2 * sizeof(int64_t), st);
@@ -485,9 +542,9 @@ cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_
     return cudaGetLastError();
 }
 
-cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                        int64_t pt_stride, const int64_t *req, int64_t n_req, uint8_t *out,
-                        cudaStream_t st)
+template <typename Sym>
+cudaError_t read_t(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
+                   const int64_t *req, int64_t n_req, Sym *out, cudaStream_t st)
 {
     const int64_t blocks = cdiv(n_req, kThreads);
     if (blocks == 0)
@@ -495,18 +552,27 @@ cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, 
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
     const int smem = tables_bytes(c->N, c->L);
-    cudaError_t e = cudaFuncSetAttribute(k_read, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(k_read<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
-    k_read<<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
+    k_read<Sym><<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
         reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride, req, n_req, out, c->d_dec, c->d_T,
         c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 
-cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
-                          int64_t n_old, const uint8_t *sym, int64_t m, int64_t sym_stride,
-                          cudaStream_t st)
+cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
+                        int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
+                        cudaStream_t st)
+{
+    if (wide(c))
+        return read_t(c, pts, n_streams, n, pt_stride, req, n_req, static_cast<uint16_t *>(out), st);
+    return read_t(c, pts, n_streams, n, pt_stride, req, n_req, static_cast<uint8_t *>(out), st);
+}
+
+template <typename Sym>
+cudaError_t append_t(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride, int64_t n_old,
+                     const Sym *sym, int64_t m, int64_t sym_stride, cudaStream_t st)
 {
     if (m <= 0 || n_streams <= 0)
         return cudaSuccess;
@@ -517,9 +583,9 @@ cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int6
         const int64_t blocks = cdiv(n_streams, kThreads);
         if (blocks > 0x7FFFFFFF)
             return cudaErrorInvalidConfiguration;
-        k_append<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
+        k_append<Sym><<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(
             reinterpret_cast<double2 *>(pts), n_streams, pt_stride, n_old, sym, head, sym_stride, n_old / L, 1,
-            c->d_V, c->r, L, c->d_status);
+            c->d_V, c->N, c->r, L, c->d_status);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess)
             return e;
@@ -528,6 +594,16 @@ cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int6
         return cudaSuccess;
     // every later span starts at the anchor: the bulk span encoder on the
     // remaining symbols, writing from span (n_old + head) / L on
-    return launch_span_encode(c, sym + head, n_streams, m - head, sym_stride,
-                              pts + 2 * ((n_old + head) / L), pt_stride, st);
+    return span_encode_t(c, sym + head, n_streams, m - head, sym_stride, pts + 2 * ((n_old + head) / L),
+                         pt_stride, st);
+}
+
+cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
+                          int64_t n_old, const void *sym, int64_t m, int64_t sym_stride,
+                          cudaStream_t st)
+{
+    if (wide(c))
+        return append_t(c, pts, n_streams, pt_stride, n_old, static_cast<const uint16_t *>(sym), m, sym_stride,
+                        st);
+    return append_t(c, pts, n_streams, pt_stride, n_old, static_cast<const uint8_t *>(sym), m, sym_stride, st);
 }

@@ -57,6 +57,12 @@ long long q_round(long double v, int frac_bits)
     return llroundl(ldexpl(v, frac_bits));
 }
 
+// Bytes per symbol: uint8 up to N = 256, uint16 above.
+int sym_size(const fkv_ctx *c)
+{
+    return c->N > 256 ? 2 : 1;
+}
+
 void destroy_cbset(fkv_cbset &s)
 {
     cudaFree(s.cb32);
@@ -246,7 +252,7 @@ extern "C" {
 
 double fkv_packing_ratio(int N)
 {
-    if (N < 3 || N > 256)
+    if (N < 3 || N > FKV_MAX_N)
         return 0.0;
     double s = 0.0;
     for (int k = 1; k <= N / 4; ++k) {
@@ -274,7 +280,7 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
         fkv_destroy(ctx);
         return code;
     };
-    if (N < 3 || N > 256)
+    if (N < 3 || N > FKV_MAX_N)
         return bail(FKV_EINVAL);
     const double rN = fkv_packing_ratio(N);
     if (!(r > 0.0) || r > rN * (1.0 + 1e-12))
@@ -282,14 +288,18 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
     const int Lmax = fkv_max_span_len(r);
     if (span_len < 1 || span_len > Lmax || span_len > 44)
         return bail(FKV_EINVAL);
+    // the decoder tables must fit one block (always true: r <= r_N bounds
+    // span_len by 44 / log2(1 / r_N), 6 symbols for every N > 256)
+    if (codec_smem_bytes(N, span_len) > kMaxDynSmem)
+        return bail(FKV_EINVAL);
     ctx->N = N;
     ctx->r = r;
     ctx->L = span_len;
     if (cudaGetDevice(&ctx->device) != cudaSuccess)
         return bail(FKV_ECUDA);
 
-    // vertex table, padded to 256 entries with NaN (a symbol >= N poisons its span)
-    std::vector<double2> V(256, make_double2(nan(""), nan("")));
+    // vertex table (the encoders give a symbol >= N a NaN vertex)
+    std::vector<double2> V(N);
     for (int c = 0; c < N; ++c)
         vertex(N, c, &V[c].x, &V[c].y);
     // decoder constants: vertices in Q1.62 and float, the step table
@@ -317,8 +327,8 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
         dec.alim[m] = q_round(0.0625L * rj, 62);
         rj *= static_cast<long double>(r);
     }
-    CK(cudaMalloc(&ctx->d_V, 256 * sizeof(double2)), "vertex alloc");
-    CK(cudaMemcpy(ctx->d_V, V.data(), 256 * sizeof(double2), cudaMemcpyHostToDevice), "vertex copy");
+    CK(cudaMalloc(&ctx->d_V, N * sizeof(double2)), "vertex alloc");
+    CK(cudaMemcpy(ctx->d_V, V.data(), N * sizeof(double2), cudaMemcpyHostToDevice), "vertex copy");
     CK(cudaMalloc(&ctx->d_dec, sizeof(fkv_decconst)), "decoder alloc");
     CK(cudaMemcpy(ctx->d_dec, &dec, sizeof(dec), cudaMemcpyHostToDevice), "decoder copy");
     CK(cudaMalloc(&ctx->d_T, T.size() * sizeof(longlong2)), "decoder alloc");
@@ -384,6 +394,11 @@ int fkv_params(const fkv_ctx *ctx, int *N, double *r, int *span_len)
     return FKV_OK;
 }
 
+int fkv_symbol_bytes(const fkv_ctx *ctx)
+{
+    return ctx ? sym_size(ctx) : 0;
+}
+
 const char *fkv_last_error(const fkv_ctx *ctx)
 {
     return ctx ? ctx->err.c_str() : kNoCtx;
@@ -404,7 +419,7 @@ int fkv_sync_status(fkv_ctx *ctx, void *stream)
     return FKV_OK;
 }
 
-int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int64_t n,
+int fkv_span_encode(fkv_ctx *ctx, const void *sym_dev, int64_t n_streams, int64_t n,
                     int64_t sym_stride, double *pts_dev, int64_t pt_stride, void *stream)
 {
     if (!ctx)
@@ -417,13 +432,15 @@ int fkv_span_encode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t n_streams, int
         return fail(ctx, FKV_EINVAL, "bad pointer or stride");
     if (reinterpret_cast<uintptr_t>(pts_dev) % 16)
         return fail(ctx, FKV_EINVAL, "points must be 16-byte aligned");
+    if (reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))
+        return fail(ctx, FKV_EINVAL, "uint16 symbols must be 2-byte aligned");
     CK(launch_span_encode(ctx, sym_dev, n_streams, n, sym_stride, pts_dev, pt_stride, as_stream(stream)),
        "span encode launch");
     return FKV_OK;
 }
 
 int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n,
-                    int64_t pt_stride, uint8_t *sym_dev, int64_t sym_stride, void *stream)
+                    int64_t pt_stride, void *sym_dev, int64_t sym_stride, void *stream)
 {
     if (!ctx)
         return FKV_EINVAL;
@@ -435,13 +452,15 @@ int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int6
         return fail(ctx, FKV_EINVAL, "bad pointer or stride");
     if (reinterpret_cast<uintptr_t>(pts_dev) % 16)
         return fail(ctx, FKV_EINVAL, "points must be 16-byte aligned");
+    if (reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))
+        return fail(ctx, FKV_EINVAL, "uint16 symbols must be 2-byte aligned");
     CK(launch_span_decode(ctx, pts_dev, n_streams, n, pt_stride, sym_dev, sym_stride, as_stream(stream)),
        "span decode launch");
     return FKV_OK;
 }
 
 int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
-             const int64_t *req_dev, int64_t n_req, uint8_t *out_dev, void *stream)
+             const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream)
 {
     if (!ctx)
         return FKV_EINVAL;
@@ -451,7 +470,8 @@ int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, 
         return FKV_OK;
     if (!pts_dev || !req_dev || !out_dev || pt_stride < (n + ctx->L - 1) / ctx->L)
         return fail(ctx, FKV_EINVAL, "bad pointer or stride");
-    if (reinterpret_cast<uintptr_t>(pts_dev) % 16 || reinterpret_cast<uintptr_t>(req_dev) % 8)
+    if (reinterpret_cast<uintptr_t>(pts_dev) % 16 || reinterpret_cast<uintptr_t>(req_dev) % 8 ||
+        reinterpret_cast<uintptr_t>(out_dev) % sym_size(ctx))
         return fail(ctx, FKV_EINVAL, "misaligned buffer");
     CK(launch_read(ctx, pts_dev, n_streams, n, pt_stride, req_dev, n_req, out_dev, as_stream(stream)),
        "read launch");
@@ -459,7 +479,7 @@ int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, 
 }
 
 int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
-                      const uint8_t *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
+                      const void *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
                       void *stream)
 {
     if (!ctx)
@@ -468,16 +488,19 @@ int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, in
         return fail(ctx, FKV_EINVAL, "negative size");
     if (qlen < 1 || qlen > ctx->L || !query)
         return fail(ctx, FKV_EINVAL, "query length outside [1, span_len]");
-    for (int i = 0; i < qlen; ++i)
-        if (query[i] >= ctx->N)
+    uint16_t q16[64];
+    for (int i = 0; i < qlen; ++i) {
+        q16[i] = ctx->N > 256 ? static_cast<const uint16_t *>(query)[i] : static_cast<const uint8_t *>(query)[i];
+        if (q16[i] >= ctx->N)
             return fail(ctx, FKV_EINVAL, "query symbol outside the alphabet");
+    }
     if (!counts_dev || (cap > 0 && !match_dev) || (n_streams > 0 && n > 0 && !pts_dev) ||
         pt_stride < (n + ctx->L - 1) / ctx->L)
         return fail(ctx, FKV_EINVAL, "bad pointer or stride");
     if (reinterpret_cast<uintptr_t>(pts_dev) % 16 || reinterpret_cast<uintptr_t>(match_dev) % 8 ||
         reinterpret_cast<uintptr_t>(counts_dev) % 8)
         return fail(ctx, FKV_EINVAL, "misaligned buffer");
-    CK(launch_suffix_search(ctx, pts_dev, n_streams, n, pt_stride, query, qlen, match_dev, cap, counts_dev,
+    CK(launch_suffix_search(ctx, pts_dev, n_streams, n, pt_stride, q16, qlen, match_dev, cap, counts_dev,
                             as_stream(stream)),
        "suffix search launch");
     return FKV_OK;
@@ -651,12 +674,12 @@ int fkv_streams_info(const fkv_streams *s, int64_t *n_streams, int64_t *length, 
     return FKV_OK;
 }
 
-int fkv_append(fkv_ctx *ctx, fkv_streams *s, const uint8_t *sym_dev, int64_t m, int64_t sym_stride,
+int fkv_append(fkv_ctx *ctx, fkv_streams *s, const void *sym_dev, int64_t m, int64_t sym_stride,
                void *stream)
 {
     if (!ctx || !s || s->ctx != ctx)
         return fail(ctx, FKV_EINVAL, "bad stream set");
-    if (m < 0 || (m > 0 && (!sym_dev || sym_stride < m)))
+    if (m < 0 || (m > 0 && (!sym_dev || sym_stride < m || reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))))
         return fail(ctx, FKV_EINVAL, "bad symbols");
     if (m == 0)
         return FKV_OK;

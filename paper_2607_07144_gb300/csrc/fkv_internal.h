@@ -28,10 +28,13 @@ struct fkv_cbset {
     __half *cbaug = nullptr;  // [Ly*H][S] blocks of 256 x 16 fp16 in core-matrix layout (8 KB)
 };
 
+// Largest alphabet: symbols are uint8 up to N = 256 and uint16 above.
+#define FKV_MAX_N 1024
+
 // Decoder constants (see decode_core.cuh).  Fixed point is Q1.62 (value * 2^62).
 struct fkv_decconst {
-    long long vx[256], vy[256];    // V(c)
-    float vfx[256], vfy[256];      // V(c) rounded to float
+    long long vx[FKV_MAX_N], vy[FKV_MAX_N];    // V(c)
+    float vfx[FKV_MAX_N], vfy[FKV_MAX_N];      // V(c) rounded to float
     long long alim[48];            // anchor limit 2^-4 r^m in Q1.62, per span length m
 };
 
@@ -40,7 +43,7 @@ struct fkv_ctx {
     double r = 0.0;
     int L = 0;
     int device = 0;
-    double2 *d_V = nullptr;        // [256] vertices, entries >= N are NaN
+    double2 *d_V = nullptr;        // [N] vertices
     fkv_decconst *d_dec = nullptr; // decoder constants (device copy)
     longlong2 *d_T = nullptr;      // [L][N] (1-r) r^j V(c) in Q1.62
     unsigned *d_status = nullptr;
@@ -63,18 +66,24 @@ struct fkv_streams {
 
 // ---------------------------------------------------------------- launches
 // codec.cu
-cudaError_t launch_span_encode(const fkv_ctx *c, const uint8_t *sym, int64_t n_streams, int64_t n,
+// Dynamic shared memory the codec's decoding kernels take for (N, L): the
+// decoder tables plus one chunk of staged symbols.
+int codec_smem_bytes(int N, int L);
+constexpr int kMaxDynSmem = 232448;   // 227 KB per block on sm_103a
+
+// Symbols are uint8 when c->N <= 256, else uint16; strides count symbols.
+cudaError_t launch_span_encode(const fkv_ctx *c, const void *sym, int64_t n_streams, int64_t n,
                                int64_t sym_stride, double *pts, int64_t pt_stride, cudaStream_t st);
 cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                               int64_t pt_stride, uint8_t *sym, int64_t sym_stride, cudaStream_t st);
+                               int64_t pt_stride, void *sym, int64_t sym_stride, cudaStream_t st);
 cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                        int64_t pt_stride, const int64_t *req, int64_t n_req, uint8_t *out,
+                        int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
                         cudaStream_t st);
 cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
-                                 int64_t pt_stride, const uint8_t *query, int qlen, int64_t *out, int64_t cap,
+                                 int64_t pt_stride, const uint16_t *query, int qlen, int64_t *out, int64_t cap,
                                  int64_t *counts, cudaStream_t st);
 cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
-                          int64_t n_old, const uint8_t *sym, int64_t m, int64_t sym_stride,
+                          int64_t n_old, const void *sym, int64_t m, int64_t sym_stride,
                           cudaStream_t st);
 // rvq.cu
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
@@ -85,7 +94,7 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
 // n_rec x S_V), which launch_span_decode_planar writes for the gather.
 enum { FKV_SYM_RECORDS = 0, FKV_SYM_PLANAR = 1 };
 cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
-                                      int64_t pt_stride, uint8_t *out, cudaStream_t st);
+                                      int64_t pt_stride, void *out, cudaStream_t st);
 // fkv_api.cu: both output views (either may be null) hold [t0, t0 + n_rec);
 // the planar decode of a whole archive into `scratch` (n_streams * n_rec * R
 // bytes) and the K/V gathers from it, once every argument has been checked.

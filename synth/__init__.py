@@ -337,9 +337,10 @@ def gpu_kv_cache(cfg: KVConfig, kv: int, device="cuda", out=None):
 
 
 def gpu_symbols(N: int, dist: str, n_streams: int, n: int, device="cuda", cfg_id: int = 2, first_stream: int = 0):
-    """uint8 [n_streams, n] symbol streams on the device, equal to symbols()."""
+    """[n_streams, n] symbol streams on the device, equal to symbols(): uint8
+    for N <= 256, else int16 holding the uint16 symbols."""
     import torch
-    out = torch.empty((n_streams, n), dtype=torch.uint8, device=device)
+    out = torch.empty((n_streams, n), dtype=torch.uint8 if N <= 256 else torch.int16, device=device)
     thr = torch.from_numpy(zipf_thresholds(N).astype(np.uint32)).to(device)
     k0, k1 = seed_key(cfg_id)
     tid = TID_SYM + (0 if dist == "uniform" else 16) + 32 * N

@@ -62,7 +62,8 @@ __global__ void k_gen_kv(void *out, int dtype, int64_t B, int64_t H, int64_t T, 
 }
 
 // symbols of one stream: uniform floor(w N / 2^32) or Zipf inverse CDF.
-__global__ void k_gen_sym(uint8_t *out, int64_t n, uint64_t stream, uint32_t tid, uint32_t N, int zipf,
+// One byte per symbol for N <= 256, else two (uint16).
+__global__ void k_gen_sym(void *out, int64_t n, uint64_t stream, uint32_t tid, uint32_t N, int zipf,
                           const uint32_t *thr, uint32_t k0, uint32_t k1)
 {
     for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
@@ -83,7 +84,10 @@ __global__ void k_gen_sym(uint8_t *out, int64_t n, uint64_t stream, uint32_t tid
             }
             s = lo;
         }
-        out[i] = static_cast<uint8_t>(s);
+        if (N <= 256)
+            static_cast<uint8_t *>(out)[i] = static_cast<uint8_t>(s);
+        else
+            static_cast<uint16_t *>(out)[i] = static_cast<uint16_t>(s);
     }
 }
 
@@ -117,7 +121,7 @@ int synth_gen_kv(void *out, int dtype, int64_t Ly, int64_t B, int64_t H, int64_t
     return static_cast<int>(cudaGetLastError());
 }
 
-int synth_gen_symbols(uint8_t *out, int64_t n, uint64_t stream_id, uint32_t tid, uint32_t N, int zipf,
+int synth_gen_symbols(void *out, int64_t n, uint64_t stream_id, uint32_t tid, uint32_t N, int zipf,
                       const uint32_t *thr, uint32_t k0, uint32_t k1, void *stream)
 {
     k_gen_sym<<<grid_for(n), 256, 0, static_cast<cudaStream_t>(stream)>>>(out, n, stream_id, tid, N, zipf, thr,

@@ -39,11 +39,11 @@ def test_binding_covers_the_header():
 def test_host_geometry_matches_oracle(libfkv, oracle_mod):
     from paper_2607_07144_gb300 import _binding
     L = _binding.lib()
-    for N in [3, 4, 5, 6, 8, 16, 64, 100, 256]:
+    for N in [3, 4, 5, 6, 8, 16, 64, 100, 256, 257, 512, 1000, 1024]:
         assert L.fkv_packing_ratio(N) == oracle_mod.packing_ratio(N)
         r = oracle_mod.packing_ratio(N)
         assert L.fkv_max_span_len(r) == oracle_mod.max_span_len(r)
-    assert L.fkv_packing_ratio(2) == 0.0 and L.fkv_packing_ratio(257) == 0.0
+    assert L.fkv_packing_ratio(2) == 0.0 and L.fkv_packing_ratio(1025) == 0.0
     assert L.fkv_max_span_len(0.0) == 0 and L.fkv_max_span_len(0.6) == 0
 
 
@@ -56,4 +56,6 @@ def test_create_rejects_bad_parameters_without_touching_the_gpu(libfkv):
     assert L.fkv_create(4, r4 * 1.001, 4, None, ctypes.byref(h)) == _binding.EINVAL   # r > r_N
     assert L.fkv_create(4, r4, 45, None, ctypes.byref(h)) == _binding.EINVAL          # span too long
     assert L.fkv_create(4, r4, 0, None, ctypes.byref(h)) == _binding.EINVAL
+    assert L.fkv_create(1025, 0.003, 4, None, ctypes.byref(h)) == _binding.EINVAL     # N above 1024
+    assert L.fkv_symbol_bytes(None) == 0
     assert not h.value
