@@ -69,12 +69,15 @@ int fkv_max_span_len(double r);
 
 /* ----------------------------------------------------------- context --- */
 
-/* Per-head residual-VQ codebooks (Sec. 3 "Setup"; 256 codewords per stage,
- * one codebook per layer, KV head, K or V and stage).  All host memory,
- * float32, row-major:
- *   k: [n_layers][n_heads][stages_k][256][dim]
- *   v: [n_layers][n_heads][stages_v][256][dim]
- * dim must be 64 or 128; stages_k, stages_v in [1, 8]. */
+/* Residual-VQ codebooks (Sec. 3 "Setup", Table 2): K codewords per stage
+ * (K = codewords), one codebook per layer, K or V, stage and either KV head
+ * (per-head, pooled = 0) or the whole layer (pooled = 1: all heads of a layer
+ * share it).  With Hc = pooled ? 1 : n_heads, all host memory, float32,
+ * row-major:
+ *   k: [n_layers][Hc][stages_k][K][dim]
+ *   v: [n_layers][Hc][stages_v][K][dim]
+ * K = 256 (0 is read as 256): dim 64 or 128, stages_k, stages_v in [1, 8].
+ * K = 1024 (uint16 symbols): dim 64, stages_k, stages_v in [1, 2]. */
 typedef struct {
     int n_layers;
     int n_heads;
@@ -83,6 +86,8 @@ typedef struct {
     int stages_v;
     const float *k;
     const float *v;
+    int codewords;
+    int pooled;
 } fkv_codebooks;
 
 /* Create a context for alphabet size N in [3, 1024], contraction ratio r in
@@ -91,7 +96,7 @@ typedef struct {
  * symbols for N = 1024).  cb may be NULL
  * for a symbol-only codec; when given, its codebooks are copied to the
  * current CUDA device (the caller keeps ownership of cb's arrays) and N must
- * be 256.  The context owns the vertex table V(c) (Sec. 1: unit circumradius,
+ * equal its codewords per stage.  The context owns the vertex table V(c) (Sec. 1: unit circumradius,
  * V(0) = (1, 0), counter-clockwise), the codebook copies and a status word.
  * *out receives the context, or NULL on failure.  Synchronous. */
 int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx **out);
@@ -192,14 +197,16 @@ typedef struct {
 /* Symbols per token record: n_heads * (stages_k + stages_v). */
 int fkv_record_len(const fkv_ctx *ctx);
 
-/* Sec. 3 "Setup": per-head residual-VQ assignment of every archived vector.
+/* Sec. 3 "Setup": residual-VQ assignment of every archived vector.
  * kv = 0 quantises keys (stages_k stages), kv = 1 values (stages_v).  For
  * each layer l, sequence b, head h and position t in [t0, t1) of `x`, stage
- * by stage the index is the codeword of codebook (l, h, kv, stage) nearest in
+ * by stage the index is the codeword of codebook (l, h or, pooled, l alone,
+ * kv, stage) nearest in
  * squared L2 to the running residual (lowest index on a tie), and the
- * residual then drops that codeword.  Indices are written in token-record
- * order (the paper does not fix one): stream (b * n_layers + l) starts at
- * sym_dev + (b * n_layers + l) * stream_stride; the record of position t is
+ * residual then drops that codeword.  Indices (symbols of the context's
+ * width) are written in token-record order (the paper does not fix one):
+ * stream (b * n_layers + l) starts at sym_dev + (b * n_layers + l) *
+ * stream_stride (in symbols); the record of position t is
  * record rec0 + (t - t0) of R = fkv_record_len symbols, holding the key
  * indices of heads 0..H-1 (stages inner) then the value indices likewise.
  * Only the kv half of each record is written.  Runs on the tensor cores
@@ -207,14 +214,14 @@ int fkv_record_len(const fkv_ctx *ctx);
  * residual's squared norm; ties closer than that may differ from a float64
  * search. */
 int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
-                   uint8_t *sym_dev, int64_t stream_stride, int64_t rec0, void *stream);
+                   void *sym_dev, int64_t stream_stride, int64_t rec0, void *stream);
 
 /* Sec. 3 "Setup": the reconstruction is the sum of the selected centroids.
  * Rebuilds positions [t0, t0 + n_rec) of every (layer, sequence, head) of
  * k_out and v_out (either may be NULL) from records 0..n_rec-1 of the symbol
  * streams laid out as in fkv_rvq_encode: sum of the stage codewords in
  * float32, stage order, rounded to nearest-even into the cache dtype. */
-int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, int64_t n_rec,
+int fkv_rvq_decode(fkv_ctx *ctx, const void *sym_dev, int64_t stream_stride, int64_t n_rec,
                    fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
 
 /* Sec. 1-3: full archive read.  Decodes records 0..n_rec-1 of the
@@ -222,7 +229,7 @@ int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, 
  * its points at pts_dev + 2 * (b * n_layers + l) * pt_stride) and writes the
  * reconstructed K and V at positions [t0, t0 + n_rec), as fkv_span_decode
  * followed by fkv_rvq_decode.  Uses a context-owned scratch buffer of
- * batch * n_layers * n_rec * R bytes, grown on demand (a synchronous
+ * batch * n_layers * n_rec * R symbols, grown on demand (a synchronous
  * allocation the first time a larger archive is decoded). */
 int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
                   fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
@@ -234,7 +241,8 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
  * Same arguments, layouts and results as fkv_decode_kv, but the decoded
  * symbols go through a 16 MiB scratch array compiled into the library
  * instead of a context-owned buffer: it calls no cudaMalloc or cudaFree.
- * Limit: batch * n_layers * n_rec * fkv_record_len(ctx) <= 16 MiB, else
+ * Limit: batch * n_layers * n_rec * fkv_record_len(ctx) *
+ * fkv_symbol_bytes(ctx) <= 16 MiB, else
  * FKV_EINVAL with nothing launched (decode fewer sequences per call).  The
  * first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any stream

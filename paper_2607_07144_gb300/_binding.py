@@ -32,7 +32,8 @@ class FkvError(RuntimeError):
 class _Codebooks(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int), ("n_heads", ctypes.c_int), ("dim", ctypes.c_int),
                 ("stages_k", ctypes.c_int), ("stages_v", ctypes.c_int),
-                ("k", ctypes.c_void_p), ("v", ctypes.c_void_p)]
+                ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("codewords", ctypes.c_int), ("pooled", ctypes.c_int)]
 
 
 class _Cache(ctypes.Structure):
@@ -132,10 +133,13 @@ def cache_view(t: torch.Tensor) -> _Cache:
 
 class Context:
     """An fkv_ctx: alphabet N, ratio r (default r_N), span length (default
-    floor(44/log2(1/r))) and optional per-head codebooks (k, v) as float32
-    arrays [n_layers, n_heads, stages, 256, dim]."""
+    floor(44/log2(1/r))) and optional codebooks (k, v) as float32 arrays
+    [n_layers, n_heads, stages, N, dim] (N = 256 or 1024 codewords per stage),
+    or, pooled (one codebook per layer shared by its heads), arrays
+    [n_layers, 1, stages, N, dim] with the head count given as n_heads."""
 
-    def __init__(self, N: int, r: float = None, span_len: int = None, codebooks=None):
+    def __init__(self, N: int, r: float = None, span_len: int = None, codebooks=None, pooled: bool = False,
+                 n_heads: int = None):
         L = lib()
         self.N = int(N)
         self.r = float(r) if r is not None else L.fkv_packing_ratio(self.N)
@@ -144,13 +148,18 @@ class Context:
         cbp = None
         if codebooks is not None:
             k, v = (np.ascontiguousarray(a, np.float32) for a in codebooks)
-            if k.ndim != 5 or v.ndim != 5 or k.shape[:2] != v.shape[:2] or k.shape[4] != v.shape[4]:
-                raise ValueError("codebooks must be [layers, heads, stages, 256, dim]")
+            if (k.ndim != 5 or v.ndim != 5 or k.shape[:2] != v.shape[:2] or k.shape[3:] != v.shape[3:]
+                    or (pooled and k.shape[1] != 1)):
+                raise ValueError("codebooks must be [layers, heads (1 if pooled), stages, codewords, dim]")
+            H = int(n_heads) if pooled else k.shape[1]
+            if pooled and n_heads is None:
+                raise ValueError("pooled codebooks need n_heads")
             self._cb_arrays = (k, v)          # keep alive during create
-            cb = _Codebooks(k.shape[0], k.shape[1], k.shape[4], k.shape[2], v.shape[2],
-                            k.ctypes.data, v.ctypes.data)
+            cb = _Codebooks(k.shape[0], H, k.shape[4], k.shape[2], v.shape[2],
+                            k.ctypes.data, v.ctypes.data, k.shape[3], int(bool(pooled)))
             cbp = ctypes.byref(cb)
-            self.n_layers, self.n_heads, self.dim = k.shape[0], k.shape[1], k.shape[4]
+            self.n_layers, self.n_heads, self.dim = k.shape[0], H, k.shape[4]
+            self.pooled = bool(pooled)
             self.stages_k, self.stages_v = k.shape[2], v.shape[2]
         rc = L.fkv_create(self.N, self.r, self.L, cbp, ctypes.byref(self._h))
         self._cb_arrays = None
@@ -249,7 +258,8 @@ class Context:
         return match[:min(c[0], cap)], c[0], c[1]
 
     def rvq_encode(self, kv: int, x: torch.Tensor, t0: int, t1: int, sym: torch.Tensor, rec0: int = 0, stream=None):
-        """x: cache [layers, batch, heads, seq, dim]; sym: uint8 [batch*layers, >= (rec0+t1-t0)*R]."""
+        """x: cache [layers, batch, heads, seq, dim]; sym: [batch*layers, >= (rec0+t1-t0)*R] of sym_dtype."""
+        self._sym(sym)
         c = cache_view(x)
         self._check(lib().fkv_rvq_encode(self._h, int(kv), ctypes.byref(c), t0, t1, _ptr(sym), _rows(sym), rec0,
                                          _stream(stream)))
@@ -257,6 +267,7 @@ class Context:
 
     def rvq_decode(self, sym: torch.Tensor, n_rec: int, k_out: torch.Tensor = None, v_out: torch.Tensor = None,
                    t0: int = 0, stream=None):
+        self._sym(sym)
         ck = cache_view(k_out) if k_out is not None else None
         cv = cache_view(v_out) if v_out is not None else None
         self._check(lib().fkv_rvq_decode(self._h, _ptr(sym), _rows(sym), n_rec,

@@ -86,8 +86,8 @@ extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t
     const int64_t R = fkv_record_len(ctx);
     const int64_t n_streams = ref->batch * ctx->Ly;
     const int64_t n = n_rec * R;
-    if (n_streams <= 0 || n > static_cast<int64_t>(kStaticScratchBytes) / n_streams) {
-        ctx->err = "fkv_decode_kv_static: batch * n_layers * n_rec * record_len exceeds the 16 MiB static "
+    if (n_streams <= 0 || n > static_cast<int64_t>(kStaticScratchBytes) / fkv_symbol_bytes(ctx) / n_streams) {
+        ctx->err = "fkv_decode_kv_static: batch * n_layers * n_rec * record_len symbols exceed the 16 MiB static "
                    "scratch; decode fewer sequences per call";
         return FKV_EINVAL;
     }

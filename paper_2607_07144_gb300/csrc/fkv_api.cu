@@ -69,6 +69,7 @@ void destroy_cbset(fkv_cbset &s)
     cudaFree(s.cnorm);
     cudaFree(s.cb16);
     cudaFree(s.escale);
+    cudaFree(s.escale_h);
     cudaFree(s.cbaug);
     s = fkv_cbset();
 }
@@ -116,23 +117,24 @@ void split3(double v, __half *out)
 //   D = 128 (k_rvq<128>): hi/lo split of c 2^-e, max |c 2^-e| in [2^14, 2^15).
 //   D = 64 (k_rvq64): hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^3, 2^9)
 //   (in [2^8, 2^9) at a group's first stage; later stages keep the previous
-//   e while they can), and a 256 x 16 norm operand per (group, stage):
+//   e while they can), and a K x 16 norm operand per (group, stage):
 //   columns 0-2 hold three fp16 parts of ||c 2^-e||^2 2^-10, the rest zero.
+// G = Ly * H codebook groups per-head, Ly pooled; K = ctx->KC codewords.
 int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
 {
     fkv_cbset &s = ctx->cb[kv];
     s.stages = stages;
-    const int G = ctx->Ly * ctx->H, D = ctx->D;
+    const int G = ctx->Ly * (ctx->pooled ? 1 : ctx->H), D = ctx->D, K = ctx->KC;
     const bool d64 = D == 64;
-    const size_t ncode = static_cast<size_t>(G) * stages * 256;
+    const size_t ncode = static_cast<size_t>(G) * stages * K;
     std::vector<float> cn(ncode);
     std::vector<int> es(static_cast<size_t>(G) * stages);
     std::vector<__half> c16(ncode * 2 * D);
     std::vector<__half> caug(d64 ? ncode * 16 : 0, __float2half(0.0f));
     for (int gs = 0; gs < G * stages; ++gs) {
-        const float *cb = host + static_cast<size_t>(gs) * 256 * D;
+        const float *cb = host + static_cast<size_t>(gs) * K * D;
         float m = 0.0f;
-        for (int i = 0; i < 256 * D; ++i) {
+        for (int i = 0; i < K * D; ++i) {
             if (!isfinite(cb[i]))
                 return fail(ctx, FKV_EINVAL, "codebook holds a non-finite value");
             m = fmaxf(m, fabsf(cb[i]));
@@ -152,7 +154,7 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         }
         es[gs] = e;
         const float mul = d64 ? -2.0f : 1.0f;
-        for (int j = 0; j < 256; ++j) {
+        for (int j = 0; j < K; ++j) {
             double nn = 0.0, ns = 0.0;
             for (int d = 0; d < D; ++d) {
                 const double v = cb[j * D + d];
@@ -162,12 +164,13 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
                 const float sv = mul * ldexpf(cb[j * D + d], -e);
                 const __half hi = __float2half_rn(sv);
                 const __half lo = __float2half_rn(sv - __half2float(hi));
-                c16[((static_cast<size_t>(gs) * 2 + 0) * 256 + j) * D + d] = hi;
-                c16[((static_cast<size_t>(gs) * 2 + 1) * 256 + j) * D + d] = lo;
+                c16[((static_cast<size_t>(gs) * 2 + 0) * K + j) * D + d] = hi;
+                c16[((static_cast<size_t>(gs) * 2 + 1) * K + j) * D + d] = lo;
             }
-            cn[static_cast<size_t>(gs) * 256 + j] = static_cast<float>(nn);
+            cn[static_cast<size_t>(gs) * K + j] = static_cast<float>(nn);
             if (d64) {
-                __half *blk = caug.data() + static_cast<size_t>(gs) * 256 * 16;
+                // K rows in the core-matrix layout: 256-row blocks of 8 KB, back to back
+                __half *blk = caug.data() + static_cast<size_t>(gs) * K * 16;
                 __half parts[3];
                 split3(ldexp(ns, -10), parts);
                 for (int k = 0; k < 16; ++k) {
@@ -185,6 +188,16 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
     CK(cudaMemcpy(s.cnorm, cn.data(), ncode * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.cb16, c16.data(), c16.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.escale, es.data(), es.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
+    {
+        // each head's copy of its codebook group's scales
+        const int GH = ctx->Ly * ctx->H;
+        std::vector<int> eh(static_cast<size_t>(GH) * stages);
+        for (int g = 0; g < GH; ++g)
+            for (int st = 0; st < stages; ++st)
+                eh[static_cast<size_t>(g) * stages + st] = es[static_cast<size_t>(ctx->pooled ? g / ctx->H : g) * stages + st];
+        CK(cudaMalloc(&s.escale_h, eh.size() * sizeof(int)), "codebook alloc");
+        CK(cudaMemcpy(s.escale_h, eh.data(), eh.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
+    }
     if (d64) {
         CK(cudaMalloc(&s.cbaug, caug.size() * sizeof(__half)), "codebook alloc");
         CK(cudaMemcpy(s.cbaug, caug.data(), caug.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
@@ -237,7 +250,7 @@ bool check_outputs(const fkv_ctx *ctx, const fkv_cache *k_out, const fkv_cache *
 }
 
 int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
-                   uint8_t *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st)
+                   void *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st)
 {
     const int64_t stride = n_rec * fkv_record_len(ctx);
     CK(launch_span_decode_planar(ctx, pts, n_streams, n_rec, pt_stride, scratch, st), "span decode launch");
@@ -337,8 +350,12 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
     CK(cudaMemset(ctx->d_status, 0, sizeof(unsigned)), "status init");
 
     if (cb) {
-        if (N != 256 || cb->n_layers < 1 || cb->n_heads < 1 || (cb->dim != 64 && cb->dim != 128) ||
-            cb->stages_k < 1 || cb->stages_k > 8 || cb->stages_v < 1 || cb->stages_v > 8 || !cb->k || !cb->v)
+        const int K = cb->codewords == 0 ? 256 : cb->codewords;
+        const int smax = K == 256 ? 8 : 2;
+        if (N != K || (K != 256 && K != 1024) || (cb->pooled != 0 && cb->pooled != 1) || cb->n_layers < 1 ||
+            cb->n_heads < 1 || (cb->dim != 64 && cb->dim != 128) || (K == 1024 && cb->dim != 64) ||
+            cb->stages_k < 1 || cb->stages_k > smax || cb->stages_v < 1 || cb->stages_v > smax || !cb->k ||
+            !cb->v)
             return bail(FKV_EINVAL);
         if (cb->n_heads * (cb->stages_k + cb->stages_v) > 1024)
             return bail(FKV_EINVAL);
@@ -346,6 +363,8 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
         ctx->Ly = cb->n_layers;
         ctx->H = cb->n_heads;
         ctx->D = cb->dim;
+        ctx->KC = K;
+        ctx->pooled = cb->pooled != 0;
         int rc = upload_cbset(ctx, 0, cb->k, cb->stages_k);
         if (rc == FKV_OK)
             rc = upload_cbset(ctx, 1, cb->v, cb->stages_v);
@@ -513,7 +532,7 @@ int fkv_record_len(const fkv_ctx *ctx)
     return ctx->H * (ctx->cb[0].stages + ctx->cb[1].stages);
 }
 
-int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t t1, uint8_t *sym_dev,
+int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t t1, void *sym_dev,
                    int64_t stream_stride, int64_t rec0, void *stream)
 {
     if (!ctx)
@@ -526,6 +545,8 @@ int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t
         return fail(ctx, FKV_EINVAL, "bad cache view (dtype, alignment or strides)");
     if (t0 < 0 || t1 < t0 || t1 > x->seq || rec0 < 0 || !sym_dev)
         return fail(ctx, FKV_EINVAL, "bad position range");
+    if (reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))
+        return fail(ctx, FKV_EINVAL, "uint16 symbols must be 2-byte aligned");
     if (t1 == t0)
         return FKV_OK;
     const int64_t R = fkv_record_len(ctx);
@@ -536,14 +557,14 @@ int fkv_rvq_encode(fkv_ctx *ctx, int kv, const fkv_cache *x, int64_t t0, int64_t
     return FKV_OK;
 }
 
-int fkv_rvq_decode(fkv_ctx *ctx, const uint8_t *sym_dev, int64_t stream_stride, int64_t n_rec,
+int fkv_rvq_decode(fkv_ctx *ctx, const void *sym_dev, int64_t stream_stride, int64_t n_rec,
                    fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream)
 {
     if (!ctx)
         return FKV_EINVAL;
     if (!ctx->has_cb)
         return fail(ctx, FKV_EINVAL, "context has no codebooks");
-    if (!sym_dev || n_rec < 0 || t0 < 0)
+    if (!sym_dev || n_rec < 0 || t0 < 0 || reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))
         return fail(ctx, FKV_EINVAL, "bad arguments");
     const int64_t R = fkv_record_len(ctx);
     if (stream_stride < n_rec * R)
@@ -583,7 +604,7 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
     const int64_t n = n_rec * R;
     if (pt_stride < (n + ctx->L - 1) / ctx->L || reinterpret_cast<uintptr_t>(pts_dev) % 16)
         return fail(ctx, FKV_EINVAL, "bad point stride or alignment");
-    const size_t need = static_cast<size_t>(n_streams) * static_cast<size_t>(n);
+    const size_t need = static_cast<size_t>(n_streams) * static_cast<size_t>(n) * sym_size(ctx);
     if (need > ctx->scratch_bytes) {
         CK(cudaStreamSynchronize(as_stream(stream)), "scratch sync");
         cudaFree(ctx->d_scratch);

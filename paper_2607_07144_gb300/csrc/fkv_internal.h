@@ -15,17 +15,19 @@
 #define FKV_ST_CORRUPT 1u
 #define FKV_ST_TIMEOUT 2u
 
-// Codebook-side constants of one K-or-V half of the archive.
+// Codebook-side constants of one K-or-V half of the archive.  G codebook
+// groups (G = Ly * H per-head, Ly pooled), K = ctx->KC codewords per stage.
 struct fkv_cbset {
     int stages = 0;
-    float *cb32 = nullptr;    // [Ly*H][S][256][D] float32 (gather, residual update)
-    float *cnorm = nullptr;   // [Ly*H][S][256] float32 squared norms
-    __half *cb16 = nullptr;   // [Ly*H][S][2][256][D] fp16 hi/lo split, scaled by 2^-e
-    int *escale = nullptr;    // [Ly*H][S] exponent e of the fp16 split
+    float *cb32 = nullptr;    // [G][S][K][D] float32 (gather, residual update)
+    float *cnorm = nullptr;   // [G][S][K] float32 squared norms
+    __half *cb16 = nullptr;   // [G][S][2][K][D] fp16 hi/lo split, scaled by 2^-e
+    int *escale = nullptr;    // [G][S] exponent e of the fp16 split
+    int *escale_h = nullptr;  // [Ly*H][S] the same per head (its group's), for k_rvq64
     CUtensorMap tmap;         // TMA map over cb16 as [rows][D], box {64, 256}, 128B swizzle
     // 64-dimensional heads only (rvq.cu k_rvq64): cb16 holds the hi/lo split of
     // -2 c 2^-e with max |c 2^-e| in [2^3, 2^9), and cbaug the norm operand.
-    __half *cbaug = nullptr;  // [Ly*H][S] blocks of 256 x 16 fp16 in core-matrix layout (8 KB)
+    __half *cbaug = nullptr;  // [G][S] blocks of K x 16 fp16 in core-matrix layout (32 B per codeword)
 };
 
 // Largest alphabet: symbols are uint8 up to N = 256 and uint16 above.
@@ -50,6 +52,8 @@ struct fkv_ctx {
     // archive geometry and codebooks
     bool has_cb = false;
     int Ly = 0, H = 0, D = 0;
+    int KC = 256;                  // codewords per stage (= N): 256 or 1024
+    bool pooled = false;           // one codebook per layer shared by its heads
     fkv_cbset cb[2];
     uint8_t *d_scratch = nullptr;
     size_t scratch_bytes = 0;
@@ -87,22 +91,22 @@ cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int6
                           cudaStream_t st);
 // rvq.cu
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
-                              uint8_t *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
+                              void *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
 // Decoded archive symbols in one of two layouts: the token records of the
-// stream itself (stream_stride bytes per stream), or planar (per stream of
-// n_rec * R bytes: H key planes of n_rec x S_K, then H value planes of
+// stream itself (stream_stride symbols per stream), or planar (per stream of
+// n_rec * R symbols: H key planes of n_rec x S_K, then H value planes of
 // n_rec x S_V), which launch_span_decode_planar writes for the gather.
 enum { FKV_SYM_RECORDS = 0, FKV_SYM_PLANAR = 1 };
 cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
                                       int64_t pt_stride, void *out, cudaStream_t st);
 // fkv_api.cu: both output views (either may be null) hold [t0, t0 + n_rec);
 // the planar decode of a whole archive into `scratch` (n_streams * n_rec * R
-// bytes) and the K/V gathers from it, once every argument has been checked.
+// symbols) and the K/V gathers from it, once every argument has been checked.
 bool check_outputs(const fkv_ctx *ctx, const fkv_cache *k_out, const fkv_cache *v_out, int64_t n_rec, int64_t t0);
 int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
-                   uint8_t *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st);
+                   void *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st);
 // gather.cu
-cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int layout, int64_t stream_stride,
+cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st);
 cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
                            int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,

@@ -3,10 +3,11 @@
 // and for random record reads (Sec. 2).
 //
 // Whole archive: persistent blocks, each taking an equal share of the
-// (codebook group, dimension slice, vector) work.  A block holds the float32
-// codebooks of one group and one slice of the head dimension (all stages) in
-// shared memory while it works on that slice, so HBM sees only the index
-// bytes in and the rebuilt K/V out.  A thread rebuilds four dimensions (one
+// (codebook group, dimension slice, head sharing the group, vector) work.  A
+// block holds the float32 codebooks of one group and one slice of the head
+// dimension (all stages) in shared memory while it works on that slice, so
+// HBM sees only the indices in and the rebuilt K/V out.  Codebooks of 256
+// codewords take uint8 indices, of 1024 codewords uint16.  A thread rebuilds four dimensions (one
 // 16-byte granule of a slice row) of a vector.  Sums run in float32, stage
 // order, then round to nearest-even into the cache dtype.
 //
@@ -15,6 +16,8 @@
 // eight threads of a quarter warp read the eight consecutive granules of one
 // row.  A 16-float slice (two rows per bank line, for more than four stages)
 // permutes its granules by an XOR of the row instead.
+#include <type_traits>
+
 #include "decode_core.cuh"
 
 namespace {
@@ -23,11 +26,12 @@ constexpr int kThreads = 1024;
 constexpr int kDT = 4;                   // dimensions a thread rebuilds
 
 struct GatherArgs {
-    const uint8_t *sym;    // the S indices of (b, l, h, rec) at sym + b ib + l il + h ih + rec ir + ioff
+    const void *sym;       // the S indices of (b, l, h, rec) at sym + b ib + l il + h ih + rec ir + ioff (symbols)
     int64_t ib, il, ih, ir, ioff;
     int64_t n_rec, batch, t0;
     int n_layers, n_heads, D, S;
-    const float *cb32;     // [Ly*H][S][256][D]
+    int pooled;            // one codebook per layer (1) or per (layer, head) (0)
+    const float *cb32;     // [G][S][KC][D]
     void *out;
     int dtype;
     int64_t s_layer, s_batch, s_head, s_pos;
@@ -79,37 +83,42 @@ __device__ __forceinline__ void add2(float &x0, float &x1, float c0, float c1)
         : "f"(c0), "f"(c1));
 }
 
-// The S stage indices of one vector, low byte first: one load of the whole
-// run when it is aligned (WIDE, S = 2, 4 or 8), else bytes.
-template <int S, bool WIDE>
-__device__ __forceinline__ uint64_t load_ids(const uint8_t *p)
+// The S stage indices of one vector, first stage in the low bits (8 or 16
+// bits each, by symbol type): one load of the whole run when it is aligned
+// (WIDE, a run of 2, 4 or 8 bytes), else one load per index.
+template <int S, bool WIDE, typename Sym>
+__device__ __forceinline__ uint64_t load_ids(const Sym *p)
 {
-    if (WIDE && S == 4)
+    constexpr int bytes = S * static_cast<int>(sizeof(Sym));
+    if (WIDE && bytes == 4)
         return __ldg(reinterpret_cast<const unsigned *>(p));
-    if (WIDE && S == 2)
+    if (WIDE && bytes == 2)
         return __ldg(reinterpret_cast<const unsigned short *>(p));
-    if (WIDE && S == 8)
+    if (WIDE && bytes == 8)
         return __ldg(reinterpret_cast<const unsigned long long *>(p));
     uint64_t w = 0;
 #pragma unroll
     for (int s = 0; s < S; ++s)
-        w |= static_cast<uint64_t>(__ldg(p + s)) << (8 * s);
+        w |= static_cast<uint64_t>(__ldg(p + s)) << (8 * sizeof(Sym) * s);
     return w;
 }
 
 // The slice width: the widest of 64, 32 or 16 floats whose codebook slice
-// (all stages) fits 128 KB; rows of 64 or 32 floats span whole 128-byte bank
-// lines.
-__host__ __device__ constexpr int gather_dp(int S)
+// (all stages, KC codewords each) fits 128 KB; rows of 64 or 32 floats span
+// whole 128-byte bank lines.
+__host__ __device__ constexpr int gather_dp(int S, int KC)
 {
-    return S <= 2 ? 64 : (S <= 4 ? 32 : 16);
+    return KC == 256 ? (S <= 2 ? 64 : (S <= 4 ? 32 : 16)) : (S <= 1 ? 32 : 16);
 }
 
-template <int S, bool WIDE>
+template <int S, bool WIDE, int KC>
 __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
 {
-    extern __shared__ __align__(128) float scb[];   // [S][256][Dp] floats
-    constexpr int Dp = gather_dp(S);
+    using Sym = typename std::conditional<KC == 256, uint8_t, uint16_t>::type;
+    constexpr int kBits = 8 * sizeof(Sym);
+    constexpr uint64_t kMask = (1ull << kBits) - 1;
+    extern __shared__ __align__(128) float scb[];   // [S][KC][Dp] floats
+    constexpr int Dp = gather_dp(S, KC);
     const int D = a.D, parts = a.parts;
     constexpr int q4 = Dp / 4;               // 16-byte granules per slice row
     constexpr bool xor_rows = Dp < 32;       // 16-float rows: XOR-permuted granules
@@ -122,25 +131,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
     const int step_b = static_cast<int>(vpi / n_rec), step_r = static_cast<int>(vpi - step_b * n_rec);
     const int64_t di_step = step_b * a.ib + step_r * a.ir, di_wrap = a.ib - n_rec * a.ir;
     const int64_t do_step = step_b * a.s_batch + step_r * a.s_pos, do_wrap = a.s_batch - n_rec * a.s_pos;
-    // this block's share of the work: slots (group * parts + part) * nvec + vector
+    // this block's share of the work: slots ((cgroup * parts + part) * HH +
+    // head of the group) * nvec + vector, HH heads sharing a codebook group
+    const int HH = a.pooled ? a.n_heads : 1;
     const int64_t nvec = a.batch * n_rec;
     const int64_t total = static_cast<int64_t>(a.n_layers) * a.n_heads * parts * nvec;
     int64_t lo = total * blockIdx.x / gridDim.x;
     const int64_t hi = total * (blockIdx.x + 1) / gridDim.x;
     int64_t cur = -1;                        // (group, part) whose slice is in shared memory
     while (lo < hi) {
-        const int64_t gp = lo / nvec;
-        const int64_t v0 = lo - gp * nvec;
+        const int64_t gph = lo / nvec;
+        const int64_t v0 = lo - gph * nvec;
         const int64_t v1 = min(nvec, v0 + (hi - lo));
         lo += v1 - v0;
-        const int g = static_cast<int>(gp / parts), part = static_cast<int>(gp % parts);
+        const int64_t gp = gph / HH;
+        const int hh = static_cast<int>(gph - gp * HH);
+        const int cgi = static_cast<int>(gp / parts), part = static_cast<int>(gp % parts);
+        const int g = a.pooled ? cgi * a.n_heads + hh : cgi;
         const int l = g / a.n_heads, h = g % a.n_heads;
         const int d0 = part * Dp;
         if (gp != cur) {
             // codebook slice -> shared memory: every 16-byte copy in flight, one wait
             __syncthreads();
-            const float *src = a.cb32 + static_cast<int64_t>(g) * S * 256 * D + d0;
-            for (int i = threadIdx.x; i < S * 256 * q4; i += kThreads) {
+            const float *src = a.cb32 + static_cast<int64_t>(cgi) * S * KC * D + d0;
+            for (int i = threadIdx.x; i < S * KC * q4; i += kThreads) {
                 const int row = i / q4, q = i - row * q4;
                 const int pq = xor_rows ? q ^ ((row >> 1) & 3) : q;
                 asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(fkvd::smem_u32(scb + 4 * (row * q4 + pq))),
@@ -157,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
         int n_it = static_cast<int>((v1 - v + vpi - 1) / vpi);
         const int64_t b = v / n_rec;
         int rec = static_cast<int>(v - b * n_rec);
-        const uint8_t *ip = a.sym + l * a.il + h * a.ih + a.ioff + b * a.ib + rec * a.ir;
+        const Sym *ip = static_cast<const Sym *>(a.sym) + l * a.il + h * a.ih + a.ioff + b * a.ib + rec * a.ir;
         int64_t oe = l * a.s_layer + h * a.s_head + (a.t0 + rec) * a.s_pos + b * a.s_batch + d0 + dq * kDT;
         const float4 *row0 = reinterpret_cast<const float4 *>(scb);
         // kU vectors per round: their index loads are all issued before any is used
@@ -185,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
                 float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
                 for (int s = 0; s < S; ++s) {
-                    const int row = s * 256 + static_cast<int>((ids[u] >> (8 * s)) & 0xFF);
+                    const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
                     const int xq = xor_rows ? (row >> 1) & 3 : 0;
                     const float4 c = row0[row * q4 + (dq ^ xq)];
                     add2(x.x, x.y, c.x, c.y);
@@ -197,25 +211,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
     }
 }
 
-template <int S>
+template <int S, int KC>
 void *gather_kernel(bool wide)
 {
-    if ((S == 2 || S == 4 || S == 8) && wide)
-        return reinterpret_cast<void *>(k_gather<S, true>);
-    return reinterpret_cast<void *>(k_gather<S, false>);
+    constexpr int bytes = S * (KC == 256 ? 1 : 2);
+    if ((bytes == 2 || bytes == 4 || bytes == 8) && wide)
+        return reinterpret_cast<void *>(k_gather<S, true, KC>);
+    return reinterpret_cast<void *>(k_gather<S, false, KC>);
 }
 
-void *gather_kernel_for(int S, bool wide)
+// 256-codeword codebooks take 1..8 stages, 1024-codeword ones 1 or 2.
+void *gather_kernel_for(int S, bool wide, int KC)
 {
+    if (KC == 1024)
+        return S == 1 ? gather_kernel<1, 1024>(wide) : gather_kernel<2, 1024>(wide);
     switch (S) {
-    case 1: return gather_kernel<1>(wide);
-    case 2: return gather_kernel<2>(wide);
-    case 3: return gather_kernel<3>(wide);
-    case 4: return gather_kernel<4>(wide);
-    case 5: return gather_kernel<5>(wide);
-    case 6: return gather_kernel<6>(wide);
-    case 7: return gather_kernel<7>(wide);
-    default: return gather_kernel<8>(wide);
+    case 1: return gather_kernel<1, 256>(wide);
+    case 2: return gather_kernel<2, 256>(wide);
+    case 3: return gather_kernel<3, 256>(wide);
+    case 4: return gather_kernel<4, 256>(wide);
+    case 5: return gather_kernel<5, 256>(wide);
+    case 6: return gather_kernel<6, 256>(wide);
+    case 7: return gather_kernel<7, 256>(wide);
+    default: return gather_kernel<8, 256>(wide);
     }
 }
 
@@ -231,6 +249,7 @@ struct ReadArgs {
     void *out;
     int dtype;
     int n_layers, n_heads, D, SK, SV, R, N, L;
+    int KC, pooled;                // codewords per stage; one codebook per layer (1) or per head (0)
     const float *cbk, *cbv;
     const fkv_decconst *dec;
     const longlong2 *T;
@@ -244,11 +263,12 @@ __host__ __device__ inline int read_tables_bytes(int N, int L)
 
 // One warp per request: its lanes decode the spans covering the record into
 // shared memory, then gather the record's 2 * H head vectors.
+template <typename Sym>
 __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(a.dec, a.T, a.N, a.L, dsm);
-    uint8_t *srec = dsm + read_tables_bytes(a.N, a.L);
+    Sym *srec = reinterpret_cast<Sym *>(dsm + read_tables_bytes(a.N, a.L));
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t q = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp;
@@ -267,7 +287,7 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
     const int64_t n = a.n_rec * R;
     const int64_t sym0 = rec * R;
     const int64_t u0 = sym0 / L, u1 = (sym0 + R - 1) / L;
-    uint8_t *my = srec + warp * kMaxRecord;
+    Sym *my = srec + warp * kMaxRecord;
     bool bad = false;
     for (int64_t u = u0 + lane; u <= u1; u += 32) {
         const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
@@ -277,7 +297,7 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
         fkvdec::walk(t, X, Y, m, [&](int j, int c) {
             const int64_t pos = base + m - 1 - j;
             if (pos >= 0 && pos < R)
-                my[pos] = static_cast<uint8_t>(c);
+                my[pos] = static_cast<Sym>(c);
         });
         const long long lim = __ldg(&a.dec->alim[m]);
         bad |= X > lim || X < -lim || Y > lim || Y < -lim;
@@ -291,13 +311,14 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
         const float *cb = kv == 0 ? a.cbk : a.cbv;
         const int off = kv == 0 ? 0 : H * a.SK;
         for (int hh = 0; hh < H; ++hh) {
-            const float *gcb = cb + (static_cast<int64_t>(l) * H + hh) * S * 256 * D;
+            const int64_t cg = a.pooled ? l : static_cast<int64_t>(l) * H + hh;
+            const float *gcb = cb + cg * S * a.KC * D;
             const int64_t obase = q * out_vec + (static_cast<int64_t>(kv) * H + hh) * D;
             for (int d = lane * 2; d < D; d += 64) {
                 float x = 0.0f, y = 0.0f;
                 for (int s = 0; s < S; ++s) {
                     const float2 c = __ldg(reinterpret_cast<const float2 *>(
-                        gcb + (static_cast<int64_t>(s) * 256 + my[off + hh * S + s]) * D + d));
+                        gcb + (static_cast<int64_t>(s) * a.KC + my[off + hh * S + s]) * D + d));
                     x += c.x;
                     y += c.y;
                 }
@@ -309,7 +330,7 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
 
 }  // namespace
 
-cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int layout, int64_t stream_stride,
+cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st)
 {
     const fkv_cbset &cb = c->cb[kv];
@@ -335,6 +356,7 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int 
     a.n_heads = H;
     a.D = c->D;
     a.S = S;
+    a.pooled = c->pooled ? 1 : 0;
     a.cb32 = cb.cb32;
     a.out = out->data;
     a.dtype = out->dtype;
@@ -342,18 +364,18 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const uint8_t *sym, int 
     a.s_batch = out->stride_batch;
     a.s_head = out->stride_head;
     a.s_pos = out->stride_pos;
-    a.Dp = gather_dp(a.S);
+    a.Dp = gather_dp(a.S, c->KC);
     const int parts = c->D / a.Dp;
     a.parts = parts;
     const int64_t nvec = a.batch * n_rec;
     if (nvec <= 0)
         return cudaSuccess;
-    const size_t smem = static_cast<size_t>(a.S) * 256 * a.Dp * 4;
+    const size_t smem = static_cast<size_t>(a.S) * c->KC * a.Dp * 4;
     // one load per vector's index run when every run is aligned to its size
-    const int64_t Sv = a.S;
-    const bool wide = reinterpret_cast<uintptr_t>(sym) % Sv == 0 && a.ib % Sv == 0 && a.il % Sv == 0 &&
+    const int64_t Sv = a.S, esz = c->KC == 256 ? 1 : 2;
+    const bool wide = reinterpret_cast<uintptr_t>(sym) % (Sv * esz) == 0 && a.ib % Sv == 0 && a.il % Sv == 0 &&
                       a.ih % Sv == 0 && a.ir % Sv == 0 && a.ioff % Sv == 0;
-    const void *kern = gather_kernel_for(a.S, wide);
+    const void *kern = gather_kernel_for(a.S, wide, c->KC);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem > 48 * 1024 ? smem : 48 * 1024));
     if (e != cudaSuccess)
@@ -398,6 +420,8 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     a.R = c->H * (a.SK + a.SV);
     a.N = c->N;
     a.L = c->L;
+    a.KC = c->KC;
+    a.pooled = c->pooled ? 1 : 0;
     a.cbk = c->cb[0].cb32;
     a.cbv = c->cb[1].cb32;
     a.dec = c->d_dec;
@@ -408,10 +432,16 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     const int64_t blocks = (n_req + kReadWarps - 1) / kReadWarps;
     if (blocks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = read_tables_bytes(a.N, a.L) + kReadWarps * kMaxRecord;
-    cudaError_t e = cudaFuncSetAttribute(k_read_kv, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    const int esz = c->KC == 256 ? 1 : 2;
+    const int smem = read_tables_bytes(a.N, a.L) + kReadWarps * kMaxRecord * esz;
+    const void *kern = esz == 1 ? reinterpret_cast<const void *>(k_read_kv<uint8_t>)
+                                : reinterpret_cast<const void *>(k_read_kv<uint16_t>);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
-    k_read_kv<<<static_cast<unsigned>(blocks), kReadWarps * 32, smem, st>>>(a);
+    void *args[] = {&a};
+    e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kReadWarps * 32), args, smem, st);
+    if (e != cudaSuccess)
+        return e;
     return cudaGetLastError();
 }

@@ -19,6 +19,8 @@
 //     (tcgen05.ld), form the scores, take the running argmin (lowest index on
 //     ties), subtract the chosen float32 codeword and re-split the residual
 //     into the operand tiles for the next stage.
+#include <type_traits>
+
 #include "fkv_internal.h"
 
 using namespace fkvd;
@@ -39,8 +41,12 @@ struct RvqArgs {
     const float *cb32;
     const float *cnorm;
     const int *escale;
+    const int *escale_h;   // [Ly*H][S] escale of each head's codebook group
     const __half *cbaug;
-    uint8_t *sym;
+    const __half *cb16;    // [G][S][2][KC][64] hi/lo of -2 c 2^-e (64-dim heads)
+    int KC;                // codewords per stage: 256 or 1024
+    int pooled;            // codebook group = layer (1) or (layer, head) (0)
+    void *sym;             // uint8 indices for KC = 256, uint16 for KC = 1024
     int64_t stream_stride, rec0;
     int R, kv_off;
     int tiles_per_group;
@@ -204,6 +210,7 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
     const int g = blockIdx.x / a.tiles_per_group;
     const int tile = blockIdx.x % a.tiles_per_group;
     const int l = g / a.n_heads, h = g % a.n_heads;
+    const int cg = a.pooled ? l : g;          // codebook group
     const int S = a.S;
     const int64_t nvec = a.batch * a.n_pos;
     const int64_t v = static_cast<int64_t>(tile) * kRows + tid;
@@ -226,7 +233,7 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(base + Lay::SLOT);
 
     auto issue_codebook = [&](int s) {
-        const int row0 = (g * S + s) * 2 * kCodes;
+        const int row0 = (cg * S + s) * 2 * kCodes;
         mbar_arrive_expect_tx(bar_b, 2u * Lay::KB * kCodes * 128u);
 #pragma unroll
         for (int kb = 0; kb < Lay::KB; ++kb) {
@@ -265,14 +272,14 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
         }
         lo_nz |= store_split8(ahi, alo, tid, c, f);
     }
-    const float *cn_g = a.cnorm + static_cast<int64_t>(g) * S * kCodes;
+    const float *cn_g = a.cnorm + static_cast<int64_t>(cg) * S * kCodes;
     cn[tid] = cn_g[tid];
     cn[tid + kThreads] = cn_g[tid + kThreads];
     fence_proxy_async_smem();
     int lo_any = __syncthreads_or(lo_nz);
 
     uint8_t idx[8];
-    const float *cb_g = a.cb32 + static_cast<int64_t>(g) * S * kCodes * D;
+    const float *cb_g = a.cb32 + static_cast<int64_t>(cg) * S * kCodes * D;
     const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
 
     for (int s = 0; s < S; ++s) {
@@ -307,7 +314,7 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
         tc_fence_after();
 
         // --- epilogue: scores ||c||^2 - 2 r.c, argmin over this row's 256 columns
-        const int eb = a.escale[g * S + s];
+        const int eb = a.escale[cg * S + s];
         const float sc = -ldexpf(1.0f, ea + eb + 1);
         float best = INFINITY;
         int bi = 0;
@@ -371,7 +378,7 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
     }
 
     if (valid && !*abort_flag) {
-        uint8_t *dst = a.sym + (b * a.n_layers + l) * a.stream_stride +
+        uint8_t *dst = static_cast<uint8_t *>(a.sym) + (b * a.n_layers + l) * a.stream_stride +
                        (a.rec0 + (t - a.t0)) * a.R + a.kv_off + h * S;
         for (int s = 0; s < S; ++s)
             dst[s] = idx[s];
@@ -602,8 +609,9 @@ __device__ __forceinline__ void unpack_row64(const uint4 *xr, int dtype, float *
 }
 
 // Exact fp32 scoring of one scaled row against the 256 codewords of a buffer
-// (c' = -(hi + lo) / 2), for rows outside the fast path.  Lowest index on ties.
-__device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb)
+// (c' = -(hi + lo) / 2), for rows outside the fast path.  Lowest index on ties;
+// *dmin receives the best squared distance.
+__device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb, float *dmin)
 {
     float best = INFINITY;
     int bidx = 0;
@@ -631,6 +639,7 @@ __device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb)
             bidx = j;
         }
     }
+    *dmin = best;
     return bidx;
 }
 
@@ -640,8 +649,8 @@ __device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb)
 // which the elementwise minimum across chunks equals it.  When the row minimum
 // is held by exactly one chunk and one position, that column is the unique
 // argmin; otherwise (an exact tie, or no finite value) *amb is set and the
-// caller rescans.
-__device__ __forceinline__ int argmin_row(uint32_t trow, bool *amb)
+// caller rescans.  *vmin receives the row minimum.
+__device__ __forceinline__ int argmin_row(uint32_t trow, bool *amb, float *vmin)
 {
     float m[16];
     float best = INFINITY;
@@ -674,6 +683,7 @@ __device__ __forceinline__ int argmin_row(uint32_t trow, bool *amb)
     for (int p = 0; p < 16; ++p)
         pm |= (m[p] == best ? 1u : 0u) << p;
     *amb = tie || pm == 0 || (pm & (pm - 1)) != 0;
+    *vmin = best;
     return bc * 16 + (__ffs(pm) - 1);
 }
 
@@ -698,11 +708,19 @@ __device__ __forceinline__ int exact_argmin_tmem(uint32_t trow)
     return bidx;
 }
 
-template <int ESZ>
+// NB = codewords per stage / 256: each stage runs as NB blocks of 256
+// codewords through the same buffers, the running argmin carried across the
+// blocks (a later block wins only with a strictly smaller score, so ties keep
+// the lowest index) and the residual updated once, after the last block, from
+// the chosen codeword's global fp16 hi/lo copy (the stage buffer that held it
+// may already be reused).
+template <int ESZ, int NB>
 __global__ void __launch_bounds__(v2::kThreads, 1)
 k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per_group, int n_pairs)
 {
     using namespace v2;
+    using Sym = typename std::conditional<NB == 1, uint8_t, uint16_t>::type;
+    constexpr int KC = NB * kCodes;              // codewords per stage
     constexpr int XN = 64 * ESZ / 16;            // 16-byte chunks per input row
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -745,6 +763,8 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
     const int S = a.S;
     const int64_t nvec = a.batch * a.n_pos;
     const int tiles = a.tiles_per_group;
+    // codebook group of head group g = (layer, head): the layer when pooled
+    auto cgroup = [&](int g) { return a.pooled ? g / a.n_heads : g; };
 
     if (warp == 0) {
         // ---------------------------------------------------- TMA producer
@@ -752,22 +772,25 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             int it = 0;
             int last[2] = {-1, -1};               // last iteration that loaded each buffer
             for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
-                const int g = p / pairs_per_group;
+                const int cg = cgroup(p / pairs_per_group);
                 bool ok = true;
-                for (int s = 0; s < S; ++s, ++it) {
-                    const int bi = it & 1;
-                    const uint32_t ph = (it >> 1) & 1;
-                    if (!wait_or_abort(bar(2 + bi), ph ^ 1, a.status, abort_flag)) {
-                        ok = false;
-                        break;
+                for (int s = 0; s < S && ok; ++s) {
+                    for (int u = 0; u < NB; ++u, ++it) {
+                        const int bi = it & 1;
+                        const uint32_t ph = (it >> 1) & 1;
+                        if (!wait_or_abort(bar(2 + bi), ph ^ 1, a.status, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t bb = sbase + OFF_B + bi * B_BUF;
+                        const int row0 = (cg * S + s) * 2 * KC + u * kCodes;
+                        mbar_arrive_expect_tx(bar(bi), 2u * B_TILE + B_AUG);
+                        tma_load_2d(bb, &tmap, 0, row0, bar(bi));
+                        tma_load_2d(bb + B_TILE, &tmap, 0, row0 + KC, bar(bi));
+                        bulk_load(bb + 2 * B_TILE, a.cbaug + (static_cast<int64_t>(cg * S + s) * KC + u * kCodes) * 16,
+                                  B_AUG, bar(bi));
+                        last[bi] = it;
                     }
-                    const uint32_t bb = sbase + OFF_B + bi * B_BUF;
-                    const int row0 = (g * S + s) * 2 * kCodes;
-                    mbar_arrive_expect_tx(bar(bi), 2u * B_TILE + B_AUG);
-                    tma_load_2d(bb, &tmap, 0, row0, bar(bi));
-                    tma_load_2d(bb + B_TILE, &tmap, 0, row0 + kCodes, bar(bi));
-                    bulk_load(bb + 2 * B_TILE, a.cbaug + static_cast<int64_t>(g * S + s) * kCodes * 16, B_AUG, bar(bi));
-                    last[bi] = it;
                 }
                 if (!ok)
                     break;
@@ -789,38 +812,40 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
                 ++pc;
-                for (int s = 0; s < S && ok; ++s, ++it) {
-                    const int bi = it & 1;
-                    const uint32_t ph = (it >> 1) & 1;
-                    ok = wait_or_abort(bar(bi), ph, a.status, abort_flag);
-                    if (!ok)
-                        break;
-                    const uint32_t bb = sbase + OFF_B + bi * B_BUF;
-                    for (int k = 0; k < 2; ++k) {
-                        ok = wait_or_abort(bar(4 + k), aph[k], a.status, abort_flag);
+                for (int s = 0; s < S && ok; ++s) {
+                    for (int u = 0; u < NB && ok; ++u, ++it) {
+                        const int bi = it & 1;
+                        const uint32_t ph = (it >> 1) & 1;
+                        ok = wait_or_abort(bar(bi), ph, a.status, abort_flag);
                         if (!ok)
                             break;
-                        aph[k] ^= 1;
-                        tc_fence_after();
-                        // the lo operand is nonzero after the first stage; at the
-                        // first stage only if a row's input needs it
-                        const bool lo = s > 0 || lo_stamp[k] == pc;
-                        const uint32_t ab = sbase + OFF_A + k * A_SLOT;
-                        const uint32_t acc = tmem + k * 256;
-                        // codeword norms first (K = 16, no swizzle), then the split dot products
-                        umma_f16(acc, daug, sdesc_core16(bb + 2 * B_TILE), idesc, 0);
+                        const uint32_t bb = sbase + OFF_B + bi * B_BUF;
+                        for (int k = 0; k < 2; ++k) {
+                            ok = wait_or_abort(bar(4 + k), aph[k], a.status, abort_flag);
+                            if (!ok)
+                                break;
+                            aph[k] ^= 1;
+                            tc_fence_after();
+                            // the lo operand is nonzero after the first stage; at the
+                            // first stage only if a row's input needs it
+                            const bool lo = s > 0 || lo_stamp[k] == pc;
+                            const uint32_t ab = sbase + OFF_A + k * A_SLOT;
+                            const uint32_t acc = tmem + k * 256;
+                            // codeword norms first (K = 16, no swizzle), then the split dot products
+                            umma_f16(acc, daug, sdesc_core16(bb + 2 * B_TILE), idesc, 0);
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk) {
-                            const uint64_t dah = sdesc_sw128(ab + kk * 32);
-                            const uint64_t dal = sdesc_sw128(ab + A_TILE + kk * 32);
-                            const uint64_t dbh = sdesc_sw128(bb + kk * 32);
-                            const uint64_t dbl = sdesc_sw128(bb + B_TILE + kk * 32);
-                            umma_f16(acc, dah, dbh, idesc, 1);
-                            umma_f16(acc, dah, dbl, idesc, 1);
-                            if (lo)
-                                umma_f16(acc, dal, dbh, idesc, 1);
+                            for (int kk = 0; kk < 4; ++kk) {
+                                const uint64_t dah = sdesc_sw128(ab + kk * 32);
+                                const uint64_t dal = sdesc_sw128(ab + A_TILE + kk * 32);
+                                const uint64_t dbh = sdesc_sw128(bb + kk * 32);
+                                const uint64_t dbl = sdesc_sw128(bb + B_TILE + kk * 32);
+                                umma_f16(acc, dah, dbh, idesc, 1);
+                                umma_f16(acc, dah, dbl, idesc, 1);
+                                if (lo)
+                                    umma_f16(acc, dal, dbh, idesc, 1);
+                            }
+                            umma_commit(bar(6 + k));
                         }
-                        umma_commit(bar(6 + k));
                     }
                 }
             }
@@ -888,7 +913,7 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             const bool valid = tile < tiles && v < nvec;
             float r[64];
             unpack_row64<ESZ>(xr, a.dtype, r);
-            int e = __ldg(&a.escale[g * S]);
+            int e = __ldg(&a.escale_h[g * S]);
             scale_row(r, pow2f(-e));
             bool fast;
             ++pc;
@@ -896,42 +921,71 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                 lo_stamp[k] = pc;
             fence_proxy_async_smem();
             mbar_arrive(bar(4 + k));
-            uint8_t idx[8];
+            Sym idx[8];
             bool ok = true;
-            for (int s = 0; s < S; ++s, ++it) {
-                const int bi = it & 1;
-                const int e_next = s + 1 < S ? __ldg(&a.escale[g * S + s + 1]) : e;   // in flight during the waits
-                ok = wait_or_abort(bar(6 + k), fph, a.status, abort_flag) &&
-                     wait_or_abort(bar(bi), (it >> 1) & 1, a.status, abort_flag);
-                // the tensor-memory loads below are warp-collective: the warp
-                // goes on, or leaves, as one
-                ok = __all_sync(0xFFFFFFFFu, ok);
+            for (int s = 0; s < S; ++s) {
+                const int e_next = s + 1 < S ? __ldg(&a.escale_h[g * S + s + 1]) : e;   // in flight during the waits
+                float bv = INFINITY;
+                int bidx = 0, bi = 0;
+                const uint8_t *bb = nullptr;
+                for (int u = 0; u < NB; ++u, ++it) {
+                    bi = it & 1;
+                    ok = wait_or_abort(bar(6 + k), fph, a.status, abort_flag) &&
+                         wait_or_abort(bar(bi), (it >> 1) & 1, a.status, abort_flag);
+                    // the tensor-memory loads below are warp-collective: the warp
+                    // goes on, or leaves, as one
+                    ok = __all_sync(0xFFFFFFFFu, ok);
+                    if (!ok)
+                        break;
+                    fph ^= 1;
+                    tc_fence_after();
+                    bb = base + OFF_B + bi * B_BUF;
+                    __syncwarp();
+                    bool amb;
+                    float vu;
+                    int j = argmin_row(trow, &amb, &vu);
+                    if (__any_sync(0xFFFFFFFFu, fast && amb)) {   // warp-collective loads: every lane takes part
+                        const int jj = exact_argmin_tmem(trow);
+                        if (amb)
+                            j = jj;
+                    }
+                    tc_fence_before();
+                    if (!fast)
+                        j = slow_argmin(r, bb, &vu);
+                    if (NB == 1 || u == 0 || vu < bv) {
+                        bv = vu;
+                        bidx = u * kCodes + j;
+                    }
+                    if (u + 1 < NB) {
+                        // this block's scores are read: the buffer and the
+                        // accumulator slot go back (the operands stay)
+                        mbar_arrive(bar(2 + bi));
+                        mbar_arrive(bar(4 + k));
+                    }
+                }
                 if (!ok)
                     break;
-                fph ^= 1;
-                tc_fence_after();
-                const uint8_t *bb = base + OFF_B + bi * B_BUF;
-                __syncwarp();
-                bool amb;
-                int bidx = argmin_row(trow, &amb);
-                if (__any_sync(0xFFFFFFFFu, fast && amb)) {   // warp-collective loads: every lane takes part
-                    const int b = exact_argmin_tmem(trow);
-                    if (amb)
-                        bidx = b;
-                }
-                tc_fence_before();
-                if (!fast)
-                    bidx = slow_argmin(r, bb);
-                idx[s] = static_cast<uint8_t>(bidx);
+                idx[s] = static_cast<Sym>(bidx);
                 if (s == S - 1 && has_next)
                     load_row(p + gridDim.x);      // r is dead from here: the next input takes its registers
                 if (s + 1 < S) {
-                    // r' <- r' - c'_bidx = r' + (hi + lo) / 2
+                    // r' <- r' - c'_bidx = r' + (hi + lo) / 2, the codeword read from the
+                    // stage buffer (one block) or from its global copy
+                    const uint4 *gh = nullptr;
+                    if (NB > 1)
+                        gh = reinterpret_cast<const uint4 *>(a.cb16 +
+                                                             ((static_cast<int64_t>(cgroup(g) * S + s) * 2) * KC + bidx) * 64);
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
-                        const uint32_t bo = swz(bidx, c);
-                        const uint4 hv = *reinterpret_cast<const uint4 *>(bb + bo);
-                        const uint4 lv = *reinterpret_cast<const uint4 *>(bb + B_TILE + bo);
+                        uint4 hv, lv;
+                        if (NB == 1) {
+                            const uint32_t bo = swz(bidx, c);
+                            hv = *reinterpret_cast<const uint4 *>(bb + bo);
+                            lv = *reinterpret_cast<const uint4 *>(bb + B_TILE + bo);
+                        } else {
+                            hv = __ldg(gh + c);
+                            lv = __ldg(gh + KC * 8 + c);
+                        }
                         const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
                         const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
 #pragma unroll
@@ -962,8 +1016,8 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             if (valid) {
                 const int64_t b = v / a.n_pos;
                 const int64_t t = a.t0 + (v - b * a.n_pos);
-                uint8_t *dst = a.sym + (b * a.n_layers + l) * a.stream_stride + (a.rec0 + (t - a.t0)) * a.R +
-                               a.kv_off + h * S;
+                Sym *dst = static_cast<Sym *>(a.sym) + (b * a.n_layers + l) * a.stream_stride +
+                           (a.rec0 + (t - a.t0)) * a.R + a.kv_off + h * S;
                 for (int s = 0; s < S; ++s)
                     dst[s] = idx[s];
             }
@@ -979,8 +1033,19 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
 
 }  // namespace
 
+template <int ESZ, int NB>
+cudaError_t launch_rvq64(const CUtensorMap &tmap, const RvqArgs &a, int ppg, int n_pairs, unsigned grid,
+                         cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(k_rvq64<ESZ, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, v2::SMEM);
+    if (e != cudaSuccess)
+        return e;
+    k_rvq64<ESZ, NB><<<grid, v2::kThreads, v2::SMEM, st>>>(tmap, a, ppg, n_pairs);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
-                              uint8_t *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st)
+                              void *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st)
 {
     const fkv_cbset &cb = c->cb[kv];
     RvqArgs a;
@@ -999,7 +1064,11 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
     a.cb32 = cb.cb32;
     a.cnorm = cb.cnorm;
     a.escale = cb.escale;
+    a.escale_h = cb.escale_h;
     a.cbaug = cb.cbaug;
+    a.cb16 = cb.cb16;
+    a.KC = c->KC;
+    a.pooled = c->pooled ? 1 : 0;
     a.sym = sym;
     a.stream_stride = stream_stride;
     a.rec0 = rec0;
@@ -1024,19 +1093,12 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
         if (e != cudaSuccess)
             return e;
         const unsigned grid = static_cast<unsigned>(n_pairs < sms ? n_pairs : sms);
-        if (x->dtype == FKV_F32) {
-            e = cudaFuncSetAttribute(k_rvq64<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, v2::SMEM);
-            if (e != cudaSuccess)
-                return e;
-            k_rvq64<4><<<grid, v2::kThreads, v2::SMEM, st>>>(cb.tmap, a, static_cast<int>(ppg),
-                                                               static_cast<int>(n_pairs));
-        } else {
-            e = cudaFuncSetAttribute(k_rvq64<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, v2::SMEM);
-            if (e != cudaSuccess)
-                return e;
-            k_rvq64<2><<<grid, v2::kThreads, v2::SMEM, st>>>(cb.tmap, a, static_cast<int>(ppg),
-                                                               static_cast<int>(n_pairs));
-        }
+        const int pp = static_cast<int>(ppg), np = static_cast<int>(n_pairs);
+        if (c->KC == 1024)
+            return x->dtype == FKV_F32 ? launch_rvq64<4, 4>(cb.tmap, a, pp, np, grid, st)
+                                       : launch_rvq64<2, 4>(cb.tmap, a, pp, np, grid, st);
+        return x->dtype == FKV_F32 ? launch_rvq64<4, 1>(cb.tmap, a, pp, np, grid, st)
+                                   : launch_rvq64<2, 1>(cb.tmap, a, pp, np, grid, st);
     } else {
         static bool attr = false;
         if (!attr) {

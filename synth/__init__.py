@@ -113,6 +113,7 @@ class KVConfig:
     outlier_scale: float
     lognormal_sigma: float  # per-channel log-normal scale sigma (0 = none)
     N: int = 256            # symbol alphabet (= codewords per stage)
+    pooled: bool = False    # one codebook per layer shared by its heads (Sec. 3, Table 2)
 
     @property
     def record_len(self) -> int:
@@ -143,6 +144,11 @@ CFG1 = KVConfig(1, "gpt2-12layer-b8-t1024-f16", 12, 8, 12, 64, 1024, "f16", 4, 2
 CFG3 = KVConfig(3, "llama3-8b-32layer-b4-t32768-bf16", 32, 4, 8, 128, 32768, "bf16", 4, 2, 3, 10.0, 0.5)
 # Decode-time streaming (Llama-3-8B shape, 64 sequences x 131072 prefilled).
 CFG4 = KVConfig(4, "llama3-8b-stream-b64-t131072-bf16", 32, 64, 8, 128, 131072 + 36, "bf16", 4, 2, 3, 10.0, 0.5)
+# Table 2's pooled rows at k = 1024 on the GPT-2 shape: RVQ 1024 x 2 and VQ 1024.
+CFG5 = KVConfig(5, "gpt2-12layer-b8-t1024-f16-pooled-rvq1024x2", 12, 8, 12, 64, 1024, "f16", 2, 2, 4, 8.0, 0.0,
+                N=1024, pooled=True)
+CFG6 = KVConfig(6, "gpt2-12layer-b8-t1024-f16-pooled-vq1024", 12, 8, 12, 64, 1024, "f16", 1, 1, 4, 8.0, 0.0,
+                N=1024, pooled=True)
 
 
 def small_config(base: KVConfig, cfg_id: int, n_layers: int, batch: int, seq: int,
@@ -228,21 +234,24 @@ def kv_cache(cfg: KVConfig, kv: int) -> np.ndarray:
 
 @functools.lru_cache(maxsize=8)
 def codebooks(cfg: KVConfig, kv: int) -> np.ndarray:
-    """Synthetic per-head RVQ codebooks, float32 [Ly, H, S, 256, D] (memoised,
-    returned read-only).
+    """Synthetic RVQ codebooks, float32 [Ly, H, S, K, D] per head, or
+    [Ly, 1, S, K, D] pooled (memoised, returned read-only); K = cfg.N.
 
     The paper trains them by k-means on KV from a disjoint span of the same
-    text; here stage s draws 256 codewords from the data's own per-channel
+    text; here stage s draws K codewords from the data's own per-channel
     distribution (a disjoint Philox stream) shrunk by STAGE_SHRINK**s, standing
-    in for samples of the stage-s residual."""
+    in for samples of the stage-s residual.  A pooled codebook serves every
+    head of its layer, so codeword j draws from head j mod H's distribution."""
     S = cfg.stages_k if kv == 0 else cfg.stages_v
-    Ly, H, D = cfg.n_layers, cfg.n_heads, cfg.dim
+    Ly, D = cfg.n_layers, cfg.dim
+    H = 1 if cfg.pooled else cfg.n_heads
     K = cfg.N
     l, h, s, j, d = np.meshgrid(np.arange(Ly), np.arange(H), np.arange(S), np.arange(K),
                                 np.arange(D), indexing="ij")
     flat = ((((l * H + h) * S + s) * K + j) * D + d).astype(np.int64)
     z = irwin_hall(flat, TID_CB_K if kv == 0 else TID_CB_V, cfg.cfg_id)
-    sig = channel_sigma(cfg, kv)[l, h, d] * (STAGE_SHRINK ** s)
+    hs = j % cfg.n_heads if cfg.pooled else h
+    sig = channel_sigma(cfg, kv)[l, hs, d] * (STAGE_SHRINK ** s)
     sc = (sig / IRWIN_HALL_STD).astype(np.float32)
     out = (z.astype(np.float32) * sc).astype(np.float32)
     out.flags.writeable = False

@@ -30,6 +30,31 @@ def test_matches_bruteforce(oracle_mod):
         assert np.all(gap >= 0)
 
 
+def test_matches_bruteforce_1024_codewords(oracle_mod):
+    # Table 2's k = 1024 rows: the same nearest-codeword search over 1024 entries
+    rng = np.random.default_rng(5)
+    for D, S in [(64, 1), (64, 2)]:
+        x = rng.normal(size=(200, D))
+        cb = (rng.normal(size=(S, 1024, D)) * 0.8 ** np.arange(S)[:, None, None]).astype(np.float32)
+        idx, gap = oracle_mod.rvq_encode(x, cb)
+        assert np.array_equal(idx, _bruteforce_rvq(x, cb))
+        assert idx.max() >= 768                    # the upper codewords are reachable
+    cb = rng.normal(size=(1, 1024, 16)).astype(np.float32)
+    cb[0, 1000] = cb[0, 3]                         # a tie across the 256-codeword blocks
+    idx, gap = oracle_mod.rvq_encode(cb[0, [3, 1000]].astype(np.float64), cb)
+    assert list(idx[:, 0]) == [3, 3] and np.all(gap[:, 0] == 0.0)
+
+
+def test_storage_identities_k1024():
+    # Table 2: one pooled k = 1024 codebook per layer; 12 heads x (K, V) x 2
+    # stages of 10-bit symbols per layer and token, five symbols per double.
+    import synth
+    c = synth.CFG5
+    assert c.record_len == 48 and c.pooled and c.N == 1024
+    cb = synth.codebooks(synth.small_config(c, 905, n_layers=2, batch=1, seq=40), 0)
+    assert cb.shape == (2, 1, 2, 1024, 64)
+
+
 def test_codeword_equal_to_input(oracle_mod):
     rng = np.random.default_rng(1)
     cb = rng.normal(size=(1, 256, 64)).astype(np.float32)
