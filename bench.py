@@ -115,6 +115,24 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ------------------------------------------------------------ multi-rank --
+def rank_workload(rank: int):
+    """One rank's replica of the workload: the GPT-2 full cache with its own
+    seed (rank 0 runs the base configuration); the archive shards by
+    (sequence, layer) stream, so ranks share nothing but the codebooks."""
+    base = synth.CFG1
+    return synth.dataclasses.replace(base, cfg_id=base.cfg_id + 1000 * rank) if rank else base
+
+
+def max_over_ranks(values, device):
+    """Element-wise maximum of per-rank timings over all ranks (one
+    all_reduce; the job's time is its slowest rank's)."""
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
 # ---------------------------------------------------------------- GPU arm --
 def run_gpu(args, rank, world, local_rank):
     import torch
@@ -123,7 +141,7 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     base = synth.CFG1
-    cfg = synth.dataclasses.replace(base, cfg_id=base.cfg_id + 1000 * rank) if rank else base
+    cfg = rank_workload(rank)
     cbk, cbv = synth.codebooks(base, 0), synth.codebooks(base, 1)     # replicated codebooks
     K = synth.gpu_kv_cache(cfg, 0, device=dev)
     V = synth.gpu_kv_cache(cfg, 1, device=dev)
@@ -291,9 +309,55 @@ def run_gpu(args, rank, world, local_rank):
                   "workload": "4 streams x 2^28 uniform symbols, N=256, span 6, one 6-symbol query"}
         del s_pts, sctx
 
+    # Table 2's pooled RVQ 1024 x 2 archive on the same GPT-2 shape: one
+    # 1024-codeword codebook per layer and stage shared by the 12 heads,
+    # uint16 symbols (N = 1024, r_1024, span 5); archive write and full read
+    k1024 = None
+    if not args.no_k1024:
+        c5 = synth.CFG5
+        kctx = fkv.Context(c5.N, codebooks=(synth.codebooks(c5, 0), synth.codebooks(c5, 1)), pooled=True,
+                           n_heads=c5.n_heads)
+        K5 = synth.gpu_kv_cache(c5, 0, device=dev)
+        V5 = synth.gpu_kv_cache(c5, 1, device=dev)
+        R5, P5 = kctx.record_len(), c5.n_archived
+        sym5 = torch.empty((ns, P5 * R5), dtype=kctx.sym_dtype, device=dev)
+        pts5 = torch.empty((ns, kctx.n_spans(P5 * R5), 2), dtype=torch.float64, device=dev)
+        K5r, V5r = torch.zeros_like(K5), torch.zeros_like(V5)
+        ev5 = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+
+        def step5(record=False):
+            if record:
+                ev5[0].record(stream)
+            kctx.rvq_encode(0, K5, c5.t0, c5.t1, sym5)
+            if record:
+                ev5[1].record(stream)
+            kctx.rvq_encode(1, V5, c5.t0, c5.t1, sym5)
+            if record:
+                ev5[2].record(stream)
+            kctx.span_encode(sym5, pts5)
+            if record:
+                ev5[3].record(stream)
+            kctx.decode_kv(pts5, P5, K5r, V5r, t0=c5.t0)
+            if record:
+                ev5[4].record(stream)
+        for _ in range(3):
+            step5()
+        reps = 5
+        acc = np.zeros(4)
+        for _ in range(reps):
+            step5(record=True)
+            torch.cuda.synchronize()
+            acc += np.array([ev5[i].elapsed_time(ev5[i + 1]) for i in range(4)])
+        acc /= reps
+        k1024 = {"rvq_k": acc[0], "rvq_v": acc[1], "span_encode": acc[2], "decode_kv": acc[3],
+                 "nvec": ns * c5.n_heads * P5, "stages": (c5.stages_k, c5.stages_v), "R": R5, "P": P5, "L": kctx.L,
+                 "ok": kctx.sync_status() == 0,
+                 "out_bytes": 2 * K5.numel() // c5.seq * P5 * K5.element_size()}
+        del K5, V5, K5r, V5r, sym5, pts5, kctx
+
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
-                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix)
+                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024)
 
 
 def roofline(res, peaks, launches_traffic=None):
@@ -398,6 +462,7 @@ def main():
     ap.add_argument("--impl", default="fkv", choices=["fkv", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-suffix", action="store_true")
+    ap.add_argument("--no-k1024", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -442,13 +507,9 @@ def main():
     res = run_gpu(args, rank, world, local_rank)
     ms = res["ms"]
     if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-        e = torch.tensor([res["e2e"]["ms"] if res["e2e"] else 0.0], device="cuda")
-        torch.distributed.all_reduce(e, op=torch.distributed.ReduceOp.MAX)
+        ms, e2e_ms = max_over_ranks([ms, res["e2e"]["ms"] if res["e2e"] else 0.0], "cuda")
         if res["e2e"]:
-            res["e2e"]["ms"] = float(e.item())
+            res["e2e"]["ms"] = e2e_ms
     if rank != 0:
         torch.distributed.destroy_process_group()
         return
@@ -460,6 +521,22 @@ def main():
         kernels["suffix_search (Sec. 5)"] = {"bound": "hbm", "ms": sx["ms"], "achieved_gbs": gbs,
                                              "frac": gbs / peaks["hbm_gbs"], "matches": sx["matches"],
                                              "candidates": sx["candidates"], "workload": sx["workload"]}
+    if res["k1024"]:
+        kx = res["k1024"]
+        rvq_ms = kx["rvq_k"] + kx["rvq_v"]
+        flops = kx["nvec"] * sum(kx["stages"]) * 2 * 64 * 1024
+        tf = flops / (rvq_ms * 1e-3) / 1e12
+        dec_b = res["ns"] * kx["P"] * kx["R"] * 2 + res["ns"] * (-(-kx["P"] * kx["R"] // kx["L"])) * 16 + kx["out_bytes"]
+        kernels["pooled RVQ 1024 x 2 archive (Table 2)"] = {
+            "workload": "gpt2-shaped full KV cache (12 layers x batch 8 x 12 heads x 1024 tok x 64, fp16), one "
+                        "1024-codeword codebook per layer and stage shared by all heads, K 2 / V 2 stages; "
+                        "uint16 symbols, N=1024, r=r_1024, L=5",
+            "rvq_ms": rvq_ms, "bound": "tensor", "achieved_tflops": tf, "frac": tf / peaks["bf16_tflops"],
+            "span_encode_ms": kx["span_encode"], "decode_kv_ms": kx["decode_kv"],
+            "decode_kv_gbs": dec_b / (kx["decode_kv"] * 1e-3) / 1e9,
+            "decode_kv_frac": dec_b / (kx["decode_kv"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "archived_positions_per_s": res["ns"] * kx["P"] / ((rvq_ms + kx["span_encode"]) * 1e-3),
+            "status_ok": kx["ok"]}
     units = res["units"] * world
     value = units / (ms * 1e-3)
     cpu = None
