@@ -20,6 +20,18 @@ constexpr int kMaxSpan = 44;    // floor(44 / log2(1/r)) with r <= 1/2
 // kernel that touches symbols is instantiated for both.
 template <typename Sym>
 __host__ __device__ constexpr int stage_bytes() { return kThreads * kMaxSpan * static_cast<int>(sizeof(Sym)) + 32; }
+// Block size of the bulk decoders: 256 spans per chunk for uint8 symbols; for
+// uint16 (N up to 1024, 104 KB of decoder tables per block) one 1024-thread
+// block per SM shares the tables.
+template <typename Sym>
+__host__ __device__ constexpr int dec_threads() { return sizeof(Sym) == 1 ? 256 : 1024; }
+// Shared staging of one decoded chunk: dec_threads spans of L symbols plus
+// the 16-byte realignment slack.
+template <typename Sym>
+__host__ __device__ inline int dec_stage_bytes(int L)
+{
+    return (dec_threads<Sym>() * L * static_cast<int>(sizeof(Sym)) + 32 + 15) & ~15;
+}
 template <typename Sym>
 __host__ __device__ constexpr int vtab_len() { return sizeof(Sym) == 1 ? 256 : FKV_MAX_N; }
 
@@ -145,7 +157,7 @@ __device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const doub
 // Persistent: a block loads the decoder tables once and walks chunks of 256
 // spans (chunk = stream * bps + span block), blockIdx.x, + gridDim.x, ...
 template <typename Sym>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(dec_threads<Sym>())
 k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
               int64_t n_chunks, Sym *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
               const longlong2 *__restrict__ T, int N, int L, unsigned *status)
@@ -154,11 +166,12 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
     uint8_t *sbuf = dsm + tables_bytes(N, L);
     __syncthreads();
+    constexpr int TPB = dec_threads<Sym>();
     for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
         const int64_t stream = ck / bps;
-        const int64_t s0 = (ck - stream * bps) * kThreads;
+        const int64_t s0 = (ck - stream * bps) * TPB;
         const int64_t b = s0 * L;
-        const int64_t e = min(n, (s0 + kThreads) * L);
+        const int64_t e = min(n, (s0 + TPB) * L);
         uint8_t *dst = reinterpret_cast<uint8_t *>(sym + stream * sym_stride + b);
         const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
         decode_chunk(t, pts, n, pt_stride, spans, stream, s0, reinterpret_cast<Sym *>(sbuf + off), dc, L, status);
@@ -175,7 +188,7 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
 // (record, stage) slot of the run, consecutive threads on consecutive bytes; a
 // record cut by the chunk boundary is completed by the neighbouring chunk.
 template <typename Sym>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(dec_threads<Sym>())
 k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
                      int64_t n_chunks, Sym *__restrict__ out, int H, int SK, int SV,
                      const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
@@ -188,11 +201,12 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
     const int R = H * (SK + SV);
     const int nk = H * SK;
     const int64_t n = n_rec * R;
+    constexpr int TPB = dec_threads<Sym>();
     for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
         const int64_t stream = ck / bps;
-        const int64_t s0 = (ck - stream * bps) * kThreads;
+        const int64_t s0 = (ck - stream * bps) * TPB;
         const int64_t q0 = s0 * L;
-        const int64_t q1 = min(n, (s0 + kThreads) * L);
+        const int64_t q1 = min(n, (s0 + TPB) * L);
         decode_chunk(t, pts, n, pt_stride, spans, stream, s0, sbuf, dc, L, status);
         __syncthreads();
         // records [rec_lo, rec_lo + nrb) overlap this chunk's symbols [q0, q1)
@@ -203,7 +217,7 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
             const int S = kv == 0 ? SK : SV;
             const int o0 = kv == 0 ? 0 : nk;                       // first offset of this half in a record
             Sym *pl = base + (kv == 0 ? 0 : static_cast<int64_t>(nk) * n_rec) + rec_lo * S;
-            for (int i = threadIdx.x; i < nrb * S; i += kThreads) {
+            for (int i = threadIdx.x; i < nrb * S; i += TPB) {
                 const int j = i / S, st = i - j * S;               // record j of the chunk, stage st
                 const int64_t qj = (rec_lo + j) * R + o0 + st - q0; // symbol of head 0, relative to q0
                 for (int h = 0; h < H; ++h) {
@@ -317,9 +331,10 @@ k_suffix_search(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, i
 }
 
 // Sec. 2 random access: one request per thread, decoding only its span down
-// to the requested offset.
+// to the requested offset.  Persistent: a block loads the decoder tables once
+// and takes requests blockIdx.x * TPB + threadIdx.x, + gridDim.x * TPB, ...
 template <typename Sym>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(dec_threads<Sym>())
 k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt_stride,
        const int64_t *__restrict__ req, int64_t n_req, Sym *__restrict__ out,
        const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L, unsigned *status)
@@ -327,23 +342,24 @@ k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
     __syncthreads();
-    const int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
-    if (q >= n_req)
-        return;
-    const int64_t st = req[2 * q], pos = req[2 * q + 1];
-    if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
-        out[q] = static_cast<Sym>(~0u);
-        atomicOr(status, FKV_ST_CORRUPT);
-        return;
+    constexpr int TPB = dec_threads<Sym>();
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * TPB + threadIdx.x; q < n_req;
+         q += static_cast<int64_t>(gridDim.x) * TPB) {
+        const int64_t st = req[2 * q], pos = req[2 * q + 1];
+        if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
+            out[q] = static_cast<Sym>(~0u);
+            atomicOr(status, FKV_ST_CORRUPT);
+            continue;
+        }
+        const int64_t u = pos / L;
+        const int o = static_cast<int>(pos - u * L);
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+        const double2 p = pts[st * pt_stride + u];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        int sym = 0;
+        fkvdec::walk(t, X, Y, m - o, [&](int j, int c) { sym = c; });
+        out[q] = static_cast<Sym>(sym);
     }
-    const int64_t u = pos / L;
-    const int o = static_cast<int>(pos - u * L);
-    const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
-    const double2 p = pts[st * pt_stride + u];
-    long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
-    int sym = 0;
-    fkvdec::walk(t, X, Y, m - o, [&](int j, int c) { sym = c; });
-    out[q] = static_cast<Sym>(sym);
 }
 
 // Sec. 2 append: one thread per (stream, span touched by the new symbols).
@@ -390,7 +406,7 @@ inline bool wide(const fkv_ctx *c) { return c->N > 256; }
 
 int codec_smem_bytes(int N, int L)
 {
-    return tables_bytes(N, L) + (N > 256 ? stage_bytes<uint16_t>() : stage_bytes<uint8_t>());
+    return tables_bytes(N, L) + (N > 256 ? dec_stage_bytes<uint16_t>(L) : dec_stage_bytes<uint8_t>(L));
 }
 
 template <typename Sym>
@@ -418,15 +434,16 @@ cudaError_t launch_span_encode(const fkv_ctx *c, const void *sym, int64_t n_stre
     return span_encode_t(c, static_cast<const uint8_t *>(sym), n_streams, n, sym_stride, pts, pt_stride, st);
 }
 
-// Persistent decode grid: as many blocks as fit on the GPU at once, at most
-// one per chunk.
-cudaError_t decode_grid(const fkv_ctx *c, const void *kern, int smem, int64_t n_chunks, unsigned *grid)
+// Persistent decode grid: as many blocks of `threads` as fit on the GPU at
+// once, at most one per chunk.
+cudaError_t decode_grid(const fkv_ctx *c, const void *kern, int smem, int64_t n_chunks, unsigned *grid,
+                        int threads = kThreads)
 {
     int sms = 0, per_sm = 0;
     cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess)
         return e;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
     if (e != cudaSuccess)
         return e;
     int64_t g = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
@@ -440,22 +457,23 @@ template <typename Sym>
 cudaError_t span_decode_t(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
                           Sym *sym, int64_t sym_stride, cudaStream_t st)
 {
+    constexpr int TPB = dec_threads<Sym>();
     const int64_t spans = cdiv(n, c->L);
-    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t bps = cdiv(spans, TPB);
     const int64_t n_chunks = n_streams * bps;
     if (n_chunks == 0)
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + stage_bytes<Sym>();
+    const int smem = tables_bytes(c->N, c->L) + dec_stage_bytes<Sym>(c->L);
     cudaError_t e = cudaFuncSetAttribute(k_span_decode<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
     unsigned grid = 0;
-    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode<Sym>), smem, n_chunks, &grid);
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode<Sym>), smem, n_chunks, &grid, TPB);
     if (e != cudaSuccess)
         return e;
-    k_span_decode<Sym><<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
+    k_span_decode<Sym><<<grid, TPB, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
                                                      static_cast<int>(bps), n_chunks, sym, sym_stride, c->d_dec,
                                                      c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
@@ -475,23 +493,24 @@ cudaError_t span_decode_planar_t(const fkv_ctx *c, const double *pts, int64_t n_
 {
     const int SK = c->cb[0].stages, SV = c->cb[1].stages;
     const int64_t n = n_rec * c->H * (SK + SV);
+    constexpr int TPB = dec_threads<Sym>();
     const int64_t spans = cdiv(n, c->L);
-    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t bps = cdiv(spans, TPB);
     const int64_t n_chunks = n_streams * bps;
     if (n_chunks == 0)
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + stage_bytes<Sym>();
+    const int smem = tables_bytes(c->N, c->L) + dec_stage_bytes<Sym>(c->L);
     cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          smem);
     if (e != cudaSuccess)
         return e;
     unsigned grid = 0;
-    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar<Sym>), smem, n_chunks, &grid);
+    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar<Sym>), smem, n_chunks, &grid, TPB);
     if (e != cudaSuccess)
         return e;
-    k_span_decode_planar<Sym><<<grid, kThreads, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec,
+    k_span_decode_planar<Sym><<<grid, TPB, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec,
                                                             pt_stride, spans, static_cast<int>(bps), n_chunks,
                                                             out, c->H, SK, SV, c->d_dec, c->d_T, c->N, c->L,
                                                             c->d_status);
@@ -546,16 +565,19 @@ template <typename Sym>
 cudaError_t read_t(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
                    const int64_t *req, int64_t n_req, Sym *out, cudaStream_t st)
 {
-    const int64_t blocks = cdiv(n_req, kThreads);
+    constexpr int TPB = dec_threads<Sym>();
+    const int64_t blocks = cdiv(n_req, TPB);
     if (blocks == 0)
         return cudaSuccess;
-    if (blocks > 0x7FFFFFFF)
-        return cudaErrorInvalidConfiguration;
     const int smem = tables_bytes(c->N, c->L);
     cudaError_t e = cudaFuncSetAttribute(k_read<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
-    k_read<Sym><<<static_cast<unsigned>(blocks), kThreads, smem, st>>>(
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_read<Sym>), smem, blocks, &grid, TPB);
+    if (e != cudaSuccess)
+        return e;
+    k_read<Sym><<<grid, TPB, smem, st>>>(
         reinterpret_cast<const double2 *>(pts), n_streams, n, pt_stride, req, n_req, out, c->d_dec, c->d_T,
         c->N, c->L, c->d_status);
     return cudaGetLastError();
