@@ -12,7 +12,10 @@ and adds the bookkeeping the paper states in words:
 * the exact window of Sec. 3 "Setup" (4 sink + 32 recent positions kept),
 * the token-record order of the archived index stream (a reading: the paper
   does not state it), and
-* the round-to-nearest-even cast of a float64 reconstruction to fp16/bf16/fp32.
+* the round-to-nearest-even cast of a float64 reconstruction to fp16/bf16/fp32,
+* the in-place suffix retrieval of Sec. 5, and
+* the lossy truncation of Sec. 4 (B-bit codes of the stored points, their
+  packed layout, recency allocation across spans).
 """
 from __future__ import annotations
 
@@ -295,3 +298,59 @@ def suffix_search(pts, n: int, query, N: int, r: float, L: int):
     match = [u for u in cand
              if np.array_equal(sym[u * L + m[u] - l:u * L + m[u]], qs)]
     return np.asarray(match, dtype=np.int64), cand
+
+
+# ------------------------------------------------------ lossy truncation ---
+def truncate_codes(pts, bits: int) -> np.ndarray:
+    """Sec. 4: truncating a code point to B bits.  Reading: each coordinate
+    x of a stored point (|x| < 1) becomes the B-bit two's complement code
+    k = floor(x * 2^(B-1)) (one sign bit, B-1 fraction bits), so that
+    k * 2^-(B-1) is x with every bit below 2^-(B-1) dropped.  Exact in binary64
+    (power-of-two scaling and floor).  Returns int64 [spans, 2]."""
+    if not 2 <= bits <= 53:
+        raise ValueError("bits outside [2, 53]")
+    p = np.ascontiguousarray(pts, dtype=np.float64).reshape(-1, 2)
+    return np.floor(np.ldexp(p, bits - 1)).astype(np.int64)
+
+
+def truncated_points(codes, bits: int) -> np.ndarray:
+    """The truncated point k * 2^-(B-1) of each code, float64 [spans, 2] (exact)."""
+    return np.ldexp(np.asarray(codes, dtype=np.int64).reshape(-1, 2).astype(np.float64), -(bits - 1))
+
+
+def pack_codes(codes, bits: int) -> np.ndarray:
+    """Packed form of one stream's codes (a reading: the paper keeps B bits per
+    point but fixes no format).  Span u's x code occupies bits
+    [2uB, 2uB + B) and its y code bits [2uB + B, 2uB + 2B) of a stream of
+    uint32 words, bit i of the stream being bit i % 32 of word i // 32, each
+    code as a B-bit two's complement field, least significant bit first.
+    Returns uint32 [ceil(2 * spans * B / 32)]."""
+    c = np.asarray(codes, dtype=np.int64).reshape(-1)            # x0, y0, x1, y1, ...
+    field = c & np.int64((1 << bits) - 1)                        # B-bit two's complement
+    bitmat = ((field[:, None] >> np.arange(bits, dtype=np.int64)[None, :]) & 1).astype(np.uint8)
+    flat = bitmat.reshape(-1)                                    # stream bit i = flat[i]
+    nwords = (flat.size + 31) // 32
+    flat = np.concatenate([flat, np.zeros(nwords * 32 - flat.size, np.uint8)])
+    by = np.packbits(flat, bitorder="little")                    # byte j holds bits 8j .. 8j+7
+    return by.view("<u4").astype(np.uint32)
+
+
+def lossy_points(pts, bits: int, keep_exact: int) -> np.ndarray:
+    """Sec. 4, recency allocation across spans: the stream's last keep_exact
+    spans keep their exact points, every earlier span its B-bit truncated
+    point.  float64 [spans, 2]."""
+    p = np.ascontiguousarray(pts, dtype=np.float64).reshape(-1, 2).copy()
+    t = max(0, p.shape[0] - int(keep_exact))
+    p[:t] = truncated_points(truncate_codes(p[:t], bits), bits)
+    return p
+
+
+def lossy_decode(pts, n: int, N: int, r: float, L: int, bits: int, keep_exact: int) -> np.ndarray:
+    """Sec. 4: the symbols a decoder recovers from the lossy archive -- the
+    Sec. 1 inverse map (span_decode: nearest vertex, binary64 inverse step) run
+    from each span's kept point.  Truncation perturbs the point by less than
+    2^-(B-1) per coordinate and the inverse map amplifies that by 1/r per step,
+    so a span's last symbols stay exact and its first ones degrade.  int32 [n]."""
+    sym, _, _ = span_decode(lossy_points(pts, bits, keep_exact), n, N, r, L)
+    return sym
+
