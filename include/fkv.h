@@ -177,6 +177,50 @@ int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, in
                       const void *query, int qlen, int64_t *match_dev, int64_t cap, int64_t *counts_dev,
                       void *stream);
 
+/* ------------------------------------------------------ lossy archive --- */
+
+/* Sec. 4: lossy operation, with precision allocated across spans by recency.
+ * A stream of n symbols has S = ceil(n / span_len) spans; its last keep_exact
+ * spans stay exact and the T = max(0, S - keep_exact) older ones are truncated:
+ * each coordinate x of the span's point becomes the B-bit two's complement
+ * code k = floor(x * 2^(B-1)) (B = bits in [2, 53]; the kept value k 2^-(B-1)
+ * is x with the bits below 2^-(B-1) dropped).  Truncation perturbs the point
+ * by less than 2^-(B-1) and decoding amplifies that by 1/r per step, so a
+ * truncated span keeps its last symbols exact and loses its first ones: about
+ * (B - 1) / log2(1/r) trailing symbols survive.
+ * Layout: codes_dev is uint32 [n_streams][code_stride], code_stride >=
+ * ceil(2 T B / 32) words; span u's x code occupies bits [2uB, 2uB + B) and its
+ * y code bits [2uB + B, 2uB + 2B) of the stream's words (bit i of the stream is
+ * bit i % 32 of word i / 32), least significant bit first.  tail_dev is
+ * float64 [n_streams][tail_stride][2], tail_stride >= S - T: the exact points
+ * of spans T .. S-1.  Together they replace the 16 S bytes of points per
+ * stream with 4 code_stride + 16 (S - T).
+ *
+ * fkv_truncate writes the codes of spans 0 .. T-1 from a point array laid out
+ * as in fkv_span_encode, and copies spans T .. S-1 to tail_dev when it is not
+ * NULL.  Returns FKV_EINVAL for bits outside [2, 53], a negative size, a short
+ * stride or a misaligned buffer. */
+int fkv_truncate(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride, int bits,
+                 int64_t keep_exact, uint32_t *codes_dev, int64_t code_stride, double *tail_dev,
+                 int64_t tail_stride, void *stream);
+
+/* Sec. 4 decode of a lossy archive: every span is decoded from its kept point
+ * (the truncated value k 2^-(B-1) or the exact tail point) by the Sec. 1
+ * inverse map in the paper's binary64 arithmetic: the nearest vertex (least
+ * binary64 squared distance, lowest index on a tie), then
+ * p <- (p - (1 - r) V(c)) / r with an IEEE division.  Symbols are written as
+ * in fkv_span_decode; no anchor check (a truncated span does not return to
+ * the anchor). */
+int fkv_lossy_decode(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride, const double *tail_dev,
+                     int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                     void *sym_dev, int64_t sym_stride, void *stream);
+
+/* Sec. 2 random access into a lossy archive: requests as in fkv_read, each
+ * decoded from its span's kept point as fkv_lossy_decode does. */
+int fkv_lossy_read(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride, const double *tail_dev,
+                   int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                   const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
+
 /* -------------------------------------------------- K/V archive path ---- */
 
 /* A K or V cache tensor on the device: head vectors of `dim` contiguous

@@ -59,6 +59,9 @@ SIGNATURES = {
     "fkv_span_decode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
     "fkv_read": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _P]),
     "fkv_suffix_search": (_I, [_P, _P, _I64, _I64, _I64, _P, _I, _P, _I64, _P, _P]),
+    "fkv_truncate": (_I, [_P, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P, _I64, _P]),
+    "fkv_lossy_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P]),
+    "fkv_lossy_read": (_I, [_P, _P, _I64, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P, _P]),
     "fkv_record_len": (_I, [_P]),
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
@@ -256,6 +259,47 @@ class Context:
                                             _ptr(counts), _stream(stream)))
         c = counts.cpu().tolist()
         return match[:min(c[0], cap)], c[0], c[1]
+
+    # -- Sec. 4 lossy archive
+    def lossy_geometry(self, n: int, bits: int, keep_exact: int):
+        """(truncated spans T, code words per stream, exact tail spans)."""
+        S = self.n_spans(n)
+        T = max(0, S - int(keep_exact))
+        return T, (2 * T * int(bits) + 31) // 32, S - T
+
+    def truncate(self, pts: torch.Tensor, n: int, bits: int, keep_exact: int, codes: torch.Tensor = None,
+                 tail: torch.Tensor = None, stream=None):
+        """pts float64 [n_streams, spans, 2] -> (codes int32 [n_streams, words]
+        holding the uint32 code words, tail float64 [n_streams, S - T, 2])."""
+        ns = pts.shape[0]
+        T, words, ts = self.lossy_geometry(n, bits, keep_exact)
+        if codes is None:
+            codes = torch.empty((ns, max(words, 1)), dtype=torch.int32, device=pts.device)
+        if tail is None:
+            tail = torch.empty((ns, max(ts, 1), 2), dtype=torch.float64, device=pts.device)
+        self._check(lib().fkv_truncate(self._h, _ptr(pts), ns, n, _rows(pts, 2), int(bits), int(keep_exact),
+                                       _ptr(codes), _rows(codes), _ptr(tail), _rows(tail, 2), _stream(stream)))
+        return codes, tail
+
+    def lossy_decode(self, codes: torch.Tensor, tail: torch.Tensor, n: int, bits: int, keep_exact: int,
+                     sym: torch.Tensor = None, stream=None) -> torch.Tensor:
+        ns = codes.shape[0]
+        if sym is None:
+            sym = torch.empty((ns, n), dtype=self.sym_dtype, device=codes.device)
+        self._sym(sym)
+        self._check(lib().fkv_lossy_decode(self._h, _ptr(codes), _rows(codes), _ptr(tail), _rows(tail, 2), ns, n,
+                                           int(bits), int(keep_exact), _ptr(sym), _rows(sym), _stream(stream)))
+        return sym
+
+    def lossy_read(self, codes: torch.Tensor, tail: torch.Tensor, n: int, bits: int, keep_exact: int,
+                   req: torch.Tensor, out: torch.Tensor = None, stream=None) -> torch.Tensor:
+        if out is None:
+            out = torch.empty(req.shape[0], dtype=self.sym_dtype, device=codes.device)
+        self._sym(out)
+        self._check(lib().fkv_lossy_read(self._h, _ptr(codes), _rows(codes), _ptr(tail), _rows(tail, 2),
+                                         codes.shape[0], n, int(bits), int(keep_exact), _ptr(req), req.shape[0],
+                                         _ptr(out), _stream(stream)))
+        return out
 
     def rvq_encode(self, kv: int, x: torch.Tensor, t0: int, t1: int, sym: torch.Tensor, rec0: int = 0, stream=None):
         """x: cache [layers, batch, heads, seq, dim]; sym: [batch*layers, >= (rec0+t1-t0)*R] of sym_dtype."""

@@ -399,6 +399,210 @@ k_append(double2 *__restrict__ pts, int64_t n_streams, int64_t pt_stride, int64_
 
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// ------------------------------------------------------------- lossy archive
+// Sec. 4: a span's stored point truncated to B bits per coordinate, the
+// B-bit two's complement code k = floor(x 2^(B-1)); the spans of a stream
+// older than its last keep_exact are kept as codes, packed into uint32 words
+// (span u's x code at stream bit 2uB, its y code at 2uB + B, least
+// significant bit first), the recent ones as exact points in a tail array.
+struct LossyArgs {
+    const uint32_t *codes;   // [n_streams][code_stride] words
+    int64_t code_stride;
+    int64_t words;           // words holding codes, per stream
+    const double2 *tail;     // [n_streams][tail_stride] exact points of spans T ..
+    int64_t tail_stride;
+    int64_t T;               // truncated spans per stream
+    int bits;
+    double scale;            // 2^-(B-1)
+};
+
+// B-bit code of one coordinate: floor(x 2^(B-1)) (exact scaling, floor conversion).
+__device__ __forceinline__ unsigned long long trunc_field(double x, double up, int bits)
+{
+    const long long k = __double2ll_rd(__dmul_rn(x, up));
+    return static_cast<unsigned long long>(k) & ((1ull << bits) - 1);
+}
+
+// Thread per (stream, output word): the word's 32 bits gathered from the codes
+// that overlap it.
+__global__ void __launch_bounds__(kThreads)
+k_truncate(const double *__restrict__ pts, int64_t pt_stride, int64_t n_streams, int64_t T, int bits,
+           uint32_t *__restrict__ codes, int64_t code_stride, int64_t words)
+{
+    const double up = static_cast<double>(1ull << (bits - 1));
+    const int64_t total = n_streams * words;
+    for (int64_t t = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const int64_t stream = t / words, w = t - stream * words;
+        const int64_t bit0 = 32 * w;
+        const int64_t c0 = bit0 / bits;
+        const int64_t c1 = min((bit0 + 31) / bits, 2 * T - 1);
+        uint32_t out = 0;
+        for (int64_t ci = c0; ci <= c1; ++ci) {
+            const double x = __ldg(pts + 2 * (stream * pt_stride + (ci >> 1)) + (ci & 1));
+            const unsigned long long f = trunc_field(x, up, bits);
+            const int64_t sh = ci * bits - bit0;
+            out |= static_cast<uint32_t>(sh >= 0 ? f << sh : f >> (-sh));
+        }
+        codes[stream * code_stride + w] = out;
+    }
+}
+
+// The B-bit field at stream bit `pos`, sign-extended.
+__device__ __forceinline__ long long read_field(const uint32_t *w, int64_t words, int64_t pos, int bits)
+{
+    const int64_t q = pos >> 5;
+    const int off = static_cast<int>(pos & 31);
+    unsigned long long v = __ldg(w + q);
+    if (q + 1 < words)
+        v |= static_cast<unsigned long long>(__ldg(w + q + 1)) << 32;
+    v >>= off;
+    if (off + bits > 64 && q + 2 < words)
+        v |= static_cast<unsigned long long>(__ldg(w + q + 2)) << (64 - off);
+    const int sh = 64 - bits;
+    return static_cast<long long>(v << sh) >> sh;
+}
+
+// The point a lossy archive keeps for span u of a stream.
+__device__ __forceinline__ double2 lossy_point(const LossyArgs &a, int64_t stream, int64_t u)
+{
+    if (u >= a.T)
+        return a.tail[stream * a.tail_stride + (u - a.T)];
+    const uint32_t *w = a.codes + stream * a.code_stride;
+    const int64_t pos = 2 * u * a.bits;
+    const long long kx = read_field(w, a.words, pos, a.bits);
+    const long long ky = read_field(w, a.words, pos + a.bits, a.bits);
+    return make_double2(__dmul_rn(static_cast<double>(kx), a.scale), __dmul_rn(static_cast<double>(ky), a.scale));
+}
+
+// Squared distance to a vertex as the paper's binary64 arithmetic forms it
+// (two products and a sum, no FMA).
+__device__ __forceinline__ double dist2(double2 v, double x, double y)
+{
+    const double dx = __dsub_rn(x, v.x), dy = __dsub_rn(y, v.y);
+    return __dadd_rn(__dmul_rn(dx, dx), __dmul_rn(dy, dy));
+}
+
+// Sec. 1 cell test in binary64 for a point that need not be a code point:
+// the vertex of least binary64 squared distance, lowest index on a tie.  The
+// nearest vertex is the angularly nearest, so for |p|^2 in [2^-40, 2^60] only
+// the three vertices around the fp32 angle are scored: every other vertex is
+// farther by at least 2|p|(cos(pi/N) - cos(3 pi/N)) (7.5e-5 |p| at N = 1024),
+// far above the rounding of the distances, so the choice equals a full scan's.
+// Other points (tiny, huge, not finite) take the full scan.
+__device__ __forceinline__ int nearest64(const double2 *sV, int N, double x, double y)
+{
+    const double rr = x * x + y * y;
+    if (rr >= 0x1p-40 && rr <= 0x1p60) {
+        const float a = atan2f(static_cast<float>(y), static_cast<float>(x)) *
+                        (static_cast<float>(N) * 0.15915494309189535f);
+        int c0 = static_cast<int>(rintf(a));
+        c0 = c0 < 0 ? c0 + N : (c0 >= N ? c0 - N : c0);
+        int best = -1;
+        double bd = 0.0;
+#pragma unroll
+        for (int k = -1; k <= 1; ++k) {
+            int c = c0 + k;
+            c = c < 0 ? c + N : (c >= N ? c - N : c);
+            const double d = dist2(sV[c], x, y);
+            if (best < 0 || d < bd || (d == bd && c < best)) {
+                bd = d;
+                best = c;
+            }
+        }
+        return best;
+    }
+    int best = 0;
+    double bd = INFINITY;
+    for (int c = 0; c < N; ++c) {
+        const double d = dist2(sV[c], x, y);
+        if (d < bd) {
+            bd = d;
+            best = c;
+        }
+    }
+    return best;
+}
+
+// Backward walk from (x, y) in the paper's arithmetic: the cell, then
+// p <- (p - w V(c)) / r with w = 1 - r (binary64 product, difference and
+// IEEE division).  emit(j, c) receives the symbol of step j.
+template <class Emit>
+__device__ __forceinline__ void walk64(const double2 *sV, int N, double w, double r, double x, double y, int steps,
+                                       Emit emit)
+{
+    for (int j = 0; j < steps; ++j) {
+        const int c = nearest64(sV, N, x, y);
+        emit(j, c);
+        const double2 v = sV[c];
+        x = __ddiv_rn(__dsub_rn(x, __dmul_rn(w, v.x)), r);
+        y = __ddiv_rn(__dsub_rn(y, __dmul_rn(w, v.y)), r);
+    }
+}
+
+// Bulk decode of a lossy archive: persistent blocks walk chunks of 256 spans
+// (one per thread) and write the symbols through shared memory.
+template <typename Sym>
+__global__ void __launch_bounds__(kThreads)
+k_lossy_decode(const LossyArgs a, int64_t n, int64_t spans, int bps, int64_t n_chunks, Sym *__restrict__ sym,
+               int64_t sym_stride, const double2 *__restrict__ V, int N, double w, double r, int L)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    double2 *sV = reinterpret_cast<double2 *>(dsm);
+    uint8_t *sbuf = dsm + N * 16;
+    for (int i = threadIdx.x; i < N; i += kThreads)
+        sV[i] = V[i];
+    __syncthreads();
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
+        const int64_t stream = ck / bps;
+        const int64_t s0 = (ck - stream * bps) * kThreads;
+        const int64_t b = s0 * L;
+        const int64_t e = min(n, (s0 + kThreads) * L);
+        uint8_t *dst = reinterpret_cast<uint8_t *>(sym + stream * sym_stride + b);
+        const int off = static_cast<int>(reinterpret_cast<uintptr_t>(dst) & 15);
+        const int64_t s = s0 + threadIdx.x;
+        if (s < spans) {
+            const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+            const double2 p = lossy_point(a, stream, s);
+            Sym *my = reinterpret_cast<Sym *>(sbuf + off) + threadIdx.x * L;
+            walk64(sV, N, w, r, p.x, p.y, m, [&](int j, int c) { my[m - 1 - j] = static_cast<Sym>(c); });
+        }
+        __syncthreads();
+        stage_out(dst, sbuf, static_cast<int>(e - b) * static_cast<int>(sizeof(Sym)), off);
+        __syncthreads();
+    }
+}
+
+// Random reads from a lossy archive: one request per thread.
+template <typename Sym>
+__global__ void __launch_bounds__(kThreads)
+k_lossy_read(const LossyArgs a, int64_t n_streams, int64_t n, const int64_t *__restrict__ req, int64_t n_req,
+             Sym *__restrict__ out, const double2 *__restrict__ V, int N, double w, double r, int L,
+             unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    double2 *sV = reinterpret_cast<double2 *>(dsm);
+    for (int i = threadIdx.x; i < N; i += kThreads)
+        sV[i] = V[i];
+    __syncthreads();
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; q < n_req;
+         q += static_cast<int64_t>(gridDim.x) * kThreads) {
+        const int64_t st = req[2 * q], pos = req[2 * q + 1];
+        if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
+            out[q] = static_cast<Sym>(~0u);
+            atomicOr(status, FKV_ST_CORRUPT);
+            continue;
+        }
+        const int64_t u = pos / L;
+        const int o = static_cast<int>(pos - u * L);
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+        const double2 p = lossy_point(a, st, u);
+        int c = 0;
+        walk64(sV, N, w, r, p.x, p.y, m - o, [&](int j, int cc) { c = cc; });
+        out[q] = static_cast<Sym>(c);
+    }
+}
+
 }  // namespace
 
 // Symbol width of a context: 1 byte for N <= 256, else 2.
@@ -629,3 +833,114 @@ cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int6
                         st);
     return append_t(c, pts, n_streams, pt_stride, n_old, static_cast<const uint8_t *>(sym), m, sym_stride, st);
 }
+
+// ------------------------------------------------------------ lossy launches
+namespace {
+
+LossyArgs lossy_args(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
+                     int64_t tail_stride, int64_t n, int bits, int64_t keep_exact)
+{
+    LossyArgs a;
+    const int64_t spans = cdiv(n, c->L);
+    a.T = spans > keep_exact ? spans - keep_exact : 0;
+    a.codes = codes;
+    a.code_stride = code_stride;
+    a.words = cdiv(2 * a.T * bits, 32);
+    a.tail = reinterpret_cast<const double2 *>(tail);
+    a.tail_stride = tail_stride;
+    a.bits = bits;
+    a.scale = ldexp(1.0, -(bits - 1));
+    return a;
+}
+
+template <typename Sym>
+cudaError_t lossy_decode_t(const fkv_ctx *c, const LossyArgs &a, int64_t n_streams, int64_t n, Sym *sym,
+                           int64_t sym_stride, cudaStream_t st)
+{
+    const int64_t spans = cdiv(n, c->L);
+    const int64_t bps = cdiv(spans, kThreads);
+    const int64_t n_chunks = n_streams * bps;
+    if (n_chunks == 0)
+        return cudaSuccess;
+    if (bps > 0x7FFFFFFF)
+        return cudaErrorInvalidConfiguration;
+    const int smem = c->N * 16 + ((kThreads * c->L * static_cast<int>(sizeof(Sym)) + 32 + 15) & ~15);
+    cudaError_t e = cudaFuncSetAttribute(k_lossy_decode<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_lossy_decode<Sym>), smem, n_chunks, &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_lossy_decode<Sym><<<grid, kThreads, smem, st>>>(a, n, spans, static_cast<int>(bps), n_chunks, sym, sym_stride,
+                                                      c->d_V, c->N, 1.0 - c->r, c->r, c->L);
+    return cudaGetLastError();
+}
+
+template <typename Sym>
+cudaError_t lossy_read_t(const fkv_ctx *c, const LossyArgs &a, int64_t n_streams, int64_t n, const int64_t *req,
+                         int64_t n_req, Sym *out, cudaStream_t st)
+{
+    const int64_t blocks = cdiv(n_req, kThreads);
+    if (blocks == 0)
+        return cudaSuccess;
+    const int smem = c->N * 16;
+    cudaError_t e = cudaFuncSetAttribute(k_lossy_read<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    unsigned grid = 0;
+    e = decode_grid(c, reinterpret_cast<const void *>(k_lossy_read<Sym>), smem, blocks, &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_lossy_read<Sym><<<grid, kThreads, smem, st>>>(a, n_streams, n, req, n_req, out, c->d_V, c->N, 1.0 - c->r,
+                                                    c->r, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_truncate(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
+                            int bits, int64_t keep_exact, uint32_t *codes, int64_t code_stride, double *tail,
+                            int64_t tail_stride, cudaStream_t st)
+{
+    const int64_t spans = cdiv(n, c->L);
+    const int64_t T = spans > keep_exact ? spans - keep_exact : 0;
+    const int64_t words = cdiv(2 * T * bits, 32);
+    if (n_streams > 0 && words > 0) {
+        int sms = 0;
+        cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+        if (e != cudaSuccess)
+            return e;
+        const int64_t blocks = min(cdiv(n_streams * words, kThreads), static_cast<int64_t>(sms) * 8);
+        k_truncate<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(pts, pt_stride, n_streams, T, bits, codes,
+                                                                        code_stride, words);
+        e = cudaGetLastError();
+        if (e != cudaSuccess)
+            return e;
+    }
+    if (tail && n_streams > 0 && spans > T)
+        return cudaMemcpy2DAsync(tail, tail_stride * 16, pts + 2 * T, pt_stride * 16, (spans - T) * 16, n_streams,
+                                 cudaMemcpyDeviceToDevice, st);
+    return cudaSuccess;
+}
+
+cudaError_t launch_lossy_decode(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
+                                int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                                void *sym, int64_t sym_stride, cudaStream_t st)
+{
+    const LossyArgs a = lossy_args(c, codes, code_stride, tail, tail_stride, n, bits, keep_exact);
+    if (wide(c))
+        return lossy_decode_t(c, a, n_streams, n, static_cast<uint16_t *>(sym), sym_stride, st);
+    return lossy_decode_t(c, a, n_streams, n, static_cast<uint8_t *>(sym), sym_stride, st);
+}
+
+cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
+                              int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                              const int64_t *req, int64_t n_req, void *out, cudaStream_t st)
+{
+    const LossyArgs a = lossy_args(c, codes, code_stride, tail, tail_stride, n, bits, keep_exact);
+    if (wide(c))
+        return lossy_read_t(c, a, n_streams, n, req, n_req, static_cast<uint16_t *>(out), st);
+    return lossy_read_t(c, a, n_streams, n, req, n_req, static_cast<uint8_t *>(out), st);
+}
+

@@ -525,6 +525,98 @@ int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, in
     return FKV_OK;
 }
 
+namespace {
+
+// Geometry of a lossy archive: truncated spans T and code words per stream.
+void lossy_geometry(const fkv_ctx *ctx, int64_t n, int bits, int64_t keep_exact, int64_t *T, int64_t *words,
+                    int64_t *tail_spans)
+{
+    const int64_t spans = (n + ctx->L - 1) / ctx->L;
+    *T = spans > keep_exact ? spans - keep_exact : 0;
+    *words = (2 * *T * bits + 31) / 32;
+    *tail_spans = spans - *T;
+}
+
+// Shared checks of the lossy calls; null on success, else the reason.
+const char *check_lossy(const fkv_ctx *ctx, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                        const void *codes, int64_t code_stride, const void *tail, int64_t tail_stride, bool need_tail)
+{
+    if (n_streams < 0 || n < 0 || keep_exact < 0)
+        return "negative size";
+    if (bits < 2 || bits > 53)
+        return "bits outside [2, 53]";
+    int64_t T, words, tail_spans;
+    lossy_geometry(ctx, n, bits, keep_exact, &T, &words, &tail_spans);
+    if (n_streams > 0 && words > 0 && (!codes || code_stride < words || reinterpret_cast<uintptr_t>(codes) % 4))
+        return "bad code buffer or stride";
+    if (n_streams > 0 && tail_spans > 0 && (need_tail || tail) &&
+        (!tail || tail_stride < tail_spans || reinterpret_cast<uintptr_t>(tail) % 16))
+        return "bad tail buffer or stride";
+    return nullptr;
+}
+
+}  // namespace
+
+int fkv_truncate(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride, int bits,
+                 int64_t keep_exact, uint32_t *codes_dev, int64_t code_stride, double *tail_dev, int64_t tail_stride,
+                 void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (const char *why = check_lossy(ctx, n_streams, n, bits, keep_exact, codes_dev, code_stride, tail_dev,
+                                      tail_stride, false))
+        return fail(ctx, FKV_EINVAL, why);
+    if (n_streams == 0 || n == 0)
+        return FKV_OK;
+    if (!pts_dev || pt_stride < (n + ctx->L - 1) / ctx->L || reinterpret_cast<uintptr_t>(pts_dev) % 16)
+        return fail(ctx, FKV_EINVAL, "bad point buffer or stride");
+    CK(launch_truncate(ctx, pts_dev, n_streams, n, pt_stride, bits, keep_exact, codes_dev, code_stride, tail_dev,
+                       tail_stride, as_stream(stream)),
+       "truncate launch");
+    return FKV_OK;
+}
+
+int fkv_lossy_decode(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride, const double *tail_dev,
+                     int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact, void *sym_dev,
+                     int64_t sym_stride, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (const char *why = check_lossy(ctx, n_streams, n, bits, keep_exact, codes_dev, code_stride, tail_dev,
+                                      tail_stride, true))
+        return fail(ctx, FKV_EINVAL, why);
+    if (n_streams == 0 || n == 0)
+        return FKV_OK;
+    if (!sym_dev || sym_stride < n || reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))
+        return fail(ctx, FKV_EINVAL, "bad symbol buffer or stride");
+    CK(launch_lossy_decode(ctx, codes_dev, code_stride, tail_dev, tail_stride, n_streams, n, bits, keep_exact,
+                           sym_dev, sym_stride, as_stream(stream)),
+       "lossy decode launch");
+    return FKV_OK;
+}
+
+int fkv_lossy_read(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride, const double *tail_dev,
+                   int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                   const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_req < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (const char *why = check_lossy(ctx, n_streams, n, bits, keep_exact, codes_dev, code_stride, tail_dev,
+                                      tail_stride, true))
+        return fail(ctx, FKV_EINVAL, why);
+    if (n_req == 0)
+        return FKV_OK;
+    if (!req_dev || !out_dev || reinterpret_cast<uintptr_t>(req_dev) % 8 ||
+        reinterpret_cast<uintptr_t>(out_dev) % sym_size(ctx))
+        return fail(ctx, FKV_EINVAL, "bad request or output buffer");
+    CK(launch_lossy_read(ctx, codes_dev, code_stride, tail_dev, tail_stride, n_streams, n, bits, keep_exact, req_dev,
+                         n_req, out_dev, as_stream(stream)),
+       "lossy read launch");
+    return FKV_OK;
+}
+
 int fkv_record_len(const fkv_ctx *ctx)
 {
     if (!ctx || !ctx->has_cb)

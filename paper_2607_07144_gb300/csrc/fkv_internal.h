@@ -89,6 +89,17 @@ cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_
 cudaError_t launch_append(const fkv_ctx *c, double *pts, int64_t n_streams, int64_t pt_stride,
                           int64_t n_old, const void *sym, int64_t m, int64_t sym_stride,
                           cudaStream_t st);
+// Sec. 4 lossy archive: B-bit codes of the spans older than the last
+// keep_exact, packed (words of uint32 per stream), plus the exact tail points.
+cudaError_t launch_truncate(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n, int64_t pt_stride,
+                            int bits, int64_t keep_exact, uint32_t *codes, int64_t code_stride, double *tail,
+                            int64_t tail_stride, cudaStream_t st);
+cudaError_t launch_lossy_decode(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
+                                int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                                void *sym, int64_t sym_stride, cudaStream_t st);
+cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
+                              int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                              const int64_t *req, int64_t n_req, void *out, cudaStream_t st);
 // rvq.cu
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
                               void *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
