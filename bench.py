@@ -309,6 +309,42 @@ def run_gpu(args, rank, world, local_rank):
                   "workload": "4 streams x 2^28 uniform symbols, N=256, span 6, one 6-symbol query"}
         del s_pts, sctx
 
+    # Sec. 4 lossy archive of this step's streams: spans older than the last
+    # 64 records truncated to 24 bits per coordinate (6 B instead of 16 B per
+    # span), the recent ones exact; truncation and the full lossy decode
+    lossy = None
+    if not args.no_lossy:
+        bits, keep = 24, 64 * R // ctx.L
+        step()
+        torch.cuda.synchronize()
+        lp = st.points()
+        n_sym = n_rec * R
+        T, words, ts = ctx.lossy_geometry(n_sym, bits, keep)
+        codes = torch.empty((ns, words), dtype=torch.int32, device=dev)
+        tail = torch.empty((ns, ts, 2), dtype=torch.float64, device=dev)
+        lsym = torch.empty((ns, n_sym), dtype=torch.uint8, device=dev)
+        evl = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        reps = 10
+        for _ in range(2):
+            ctx.truncate(lp, n_sym, bits, keep, codes=codes, tail=tail)
+            ctx.lossy_decode(codes, tail, n_sym, bits, keep, sym=lsym)
+        torch.cuda.synchronize()
+        evl[0].record(stream)
+        for _ in range(reps):                      # back to back: device time, not launch gaps
+            ctx.truncate(lp, n_sym, bits, keep, codes=codes, tail=tail)
+        evl[1].record(stream)
+        for _ in range(reps):
+            ctx.lossy_decode(codes, tail, n_sym, bits, keep, sym=lsym)
+        evl[2].record(stream)
+        torch.cuda.synchronize()
+        acc = np.array([evl[0].elapsed_time(evl[1]), evl[1].elapsed_time(evl[2])]) / reps
+        exact = ctx.span_decode(lp, n_sym)
+        err = (lsym[:, :T * ctx.L] != exact[:, :T * ctx.L]).float().mean().item()
+        lossy = {"truncate": acc[0], "decode": acc[1], "bits": bits, "keep": keep, "T": T, "spans": T + ts,
+                 "symbols": ns * n_sym, "code_bytes": ns * words * 4, "tail_bytes": ns * ts * 16,
+                 "point_bytes": ns * (T + ts) * 16, "sym_err_truncated": err, "ok": ctx.sync_status() == 0}
+        del codes, tail, lsym, exact
+
     # Table 2's pooled RVQ 1024 x 2 archive on the same GPT-2 shape: one
     # 1024-codeword codebook per layer and stage shared by the 12 heads,
     # uint16 symbols (N = 1024, r_1024, span 5); archive write and full read
@@ -357,7 +393,8 @@ def run_gpu(args, rank, world, local_rank):
 
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
-                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024)
+                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024,
+                lossy=lossy)
 
 
 def roofline(res, peaks, launches_traffic=None):
@@ -463,6 +500,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-suffix", action="store_true")
     ap.add_argument("--no-k1024", action="store_true")
+    ap.add_argument("--no-lossy", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -537,6 +575,19 @@ def main():
             "decode_kv_frac": dec_b / (kx["decode_kv"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
             "archived_positions_per_s": res["ns"] * kx["P"] / ((rvq_ms + kx["span_encode"]) * 1e-3),
             "status_ok": kx["ok"]}
+    if res["lossy"]:
+        lx = res["lossy"]
+        tb = lx["point_bytes"] + lx["code_bytes"]             # points read, codes written
+        kernels["lossy archive (Sec. 4)"] = {
+            "workload": "this step's 96 streams x 989 records x 72 symbols (N=256, span 6); spans older than the "
+                        "last %d truncated to %d bits per coordinate" % (lx["keep"], lx["bits"]),
+            "truncate_ms": lx["truncate"], "truncate_bound": "hbm",
+            "truncate_gbs": tb / (lx["truncate"] * 1e-3) / 1e9,
+            "truncate_frac": tb / (lx["truncate"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "decode_ms": lx["decode"], "decode_bound": "fp64 (binary64 walk with IEEE division, as the paper)",
+            "decode_symbols_per_s": lx["symbols"] / (lx["decode"] * 1e-3),
+            "archive_bytes": lx["code_bytes"] + lx["tail_bytes"], "exact_archive_bytes": lx["point_bytes"],
+            "symbol_error_rate_truncated_spans": lx["sym_err_truncated"], "status_ok": lx["ok"]}
     units = res["units"] * world
     value = units / (ms * 1e-3)
     cpu = None

@@ -186,8 +186,8 @@ int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, in
  * code k = floor(x * 2^(B-1)) (B = bits in [2, 53]; the kept value k 2^-(B-1)
  * is x with the bits below 2^-(B-1) dropped).  Truncation perturbs the point
  * by less than 2^-(B-1) and decoding amplifies that by 1/r per step, so a
- * truncated span keeps its last symbols exact and loses its first ones: about
- * (B - 1) / log2(1/r) trailing symbols survive.
+ * truncated span keeps its last symbols exact and loses its first ones:
+ * roughly (B - 1) / log2(1/r) - 1 trailing symbols survive on random data.
  * Layout: codes_dev is uint32 [n_streams][code_stride], code_stride >=
  * ceil(2 T B / 32) words; span u's x code occupies bits [2uB, 2uB + B) and its
  * y code bits [2uB + B, 2uB + 2B) of the stream's words (bit i of the stream is

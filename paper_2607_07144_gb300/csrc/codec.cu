@@ -423,28 +423,50 @@ __device__ __forceinline__ unsigned long long trunc_field(double x, double up, i
     return static_cast<unsigned long long>(k) & ((1ull << bits) - 1);
 }
 
-// Thread per (stream, output word): the word's 32 bits gathered from the codes
-// that overlap it.
+// Warp per group of 32 spans of one stream: the group's 64 codes fill exactly
+// 2B words (the group starts at stream bit 64 B g, a word boundary); each lane
+// computes its span's two codes, then assembles words lane, lane + 32, ... of
+// the group from the codes that overlap them, fetched by warp shuffles.
 __global__ void __launch_bounds__(kThreads)
 k_truncate(const double *__restrict__ pts, int64_t pt_stride, int64_t n_streams, int64_t T, int bits,
            uint32_t *__restrict__ codes, int64_t code_stride, int64_t words)
 {
     const double up = static_cast<double>(1ull << (bits - 1));
-    const int64_t total = n_streams * words;
-    for (int64_t t = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; t < total;
-         t += static_cast<int64_t>(gridDim.x) * kThreads) {
-        const int64_t stream = t / words, w = t - stream * words;
-        const int64_t bit0 = 32 * w;
-        const int64_t c0 = bit0 / bits;
-        const int64_t c1 = min((bit0 + 31) / bits, 2 * T - 1);
-        uint32_t out = 0;
-        for (int64_t ci = c0; ci <= c1; ++ci) {
-            const double x = __ldg(pts + 2 * (stream * pt_stride + (ci >> 1)) + (ci & 1));
-            const unsigned long long f = trunc_field(x, up, bits);
-            const int64_t sh = ci * bits - bit0;
-            out |= static_cast<uint32_t>(sh >= 0 ? f << sh : f >> (-sh));
+    const int lane = threadIdx.x & 31;
+    const int64_t gps = (T + 31) >> 5;                       // groups per stream
+    const int64_t n_groups = n_streams * gps;
+    const int64_t nw = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+    const int kmax = 32 / bits + 2;                          // codes overlapping one word, at most
+    const int wpg = 2 * bits;                                // words per group
+    for (int64_t g = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5; g < n_groups; g += nw) {
+        const int64_t stream = g / gps, grp = g - stream * gps;
+        const int64_t u = grp * 32 + lane;
+        unsigned long long fx = 0, fy = 0;
+        if (u < T) {
+            const double2 p = reinterpret_cast<const double2 *>(pts)[stream * pt_stride + u];
+            fx = trunc_field(p.x, up, bits);
+            fy = trunc_field(p.y, up, bits);
         }
-        codes[stream * code_stride + w] = out;
+        const int64_t w0 = grp * wpg;
+        const int64_t nwg = min(static_cast<int64_t>(wpg), words - w0);
+        for (int j0 = 0; j0 < wpg; j0 += 32) {
+            const int j = j0 + lane;
+            const int bit0 = 32 * j;                         // relative to the group
+            const int c0 = bit0 / bits;
+            uint32_t out = 0;
+            for (int k = 0; k < kmax; ++k) {
+                const int ci = c0 + k;                       // code of the group: span ci / 2, x or y
+                const int src = min(ci >> 1, 31);
+                const unsigned long long vx = __shfl_sync(0xFFFFFFFFu, fx, src);
+                const unsigned long long vy = __shfl_sync(0xFFFFFFFFu, fy, src);
+                const unsigned long long f = (ci & 1) ? vy : vx;
+                const int sh = ci * bits - bit0;
+                if (ci < 64 && sh < 32)
+                    out |= static_cast<uint32_t>(sh >= 0 ? f << sh : f >> (-sh));
+            }
+            if (j < nwg)
+                codes[stream * code_stride + w0 + j] = out;
+        }
     }
 }
 
@@ -911,7 +933,7 @@ cudaError_t launch_truncate(const fkv_ctx *c, const double *pts, int64_t n_strea
         cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
         if (e != cudaSuccess)
             return e;
-        const int64_t blocks = min(cdiv(n_streams * words, kThreads), static_cast<int64_t>(sms) * 8);
+        const int64_t blocks = min(cdiv(n_streams * cdiv(T, 32), kThreads / 32), static_cast<int64_t>(sms) * 8);
         k_truncate<<<static_cast<unsigned>(blocks), kThreads, 0, st>>>(pts, pt_stride, n_streams, T, bits, codes,
                                                                         code_stride, words);
         e = cudaGetLastError();
