@@ -400,20 +400,24 @@ k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
 // and a hi/lo operand tile of the scaled residual r'.
 //
 // A (group, stage) is scaled by a power of two 2^-e (max |c'| in [2^3, 2^9),
-// usually one e for all stages of a group), and an extra K = 16 MMA against a
-// constant operand adds the codeword norms, so
-//     acc_j = sum (r'_hi,lo) (-2 c'_hi,lo) + 2^10 sum_3 parts(||c'_j||^2 2^-10)
-//           = ||r' - c'_j||^2 - ||r'||^2
-// (hi*hi + hi*lo + lo*hi, ~22-bit operands; norms to ~33 bits).  The argmin
-// over the 256 columns is exact on the fp32 accumulators: tcgen05.ld.red
-// returns the minimum of every 16 columns with the load, which gives the
-// best value and its 16-column chunk, and an elementwise minimum across the
-// chunks gives its position inside the chunk; an exact tie (the minimum in two
-// chunks or two positions) is rescanned column by column.  A row whose scaled
-// residual reaches 2^14 (far outside the codebook) is scored exactly in fp32
-// from the stage buffer instead.  The fp32 residual r' lives in registers and
-// is updated with mixed-precision FMAs straight from the fp16 hi/lo codeword in
-// the buffer; the next pair's 16-bit input rows are prefetched into registers
+// usually one e for all stages of a group) and a row by a further 2^-er,
+// er >= 0 chosen when its pair starts so that the row's operand
+// t = r 2^-(e + er) starts below 2^12; an extra K = 16 MMA against the row's
+// norm operand (2^(10 - er) in columns 0..2) adds the codeword norms, so
+//     acc_j = sum (t_hi,lo) (-2 c'_hi,lo) + 2^(10-er) sum_3 parts(||c'_j||^2 2^-10)
+//           = 2^-er (||r' - c'_j||^2 - ||r'||^2)
+// (hi*hi + hi*lo + lo*hi, ~22-bit operands; norms to ~33 bits), whose argmin
+// over j is the nearest codeword for any input magnitude.  The argmin over
+// the 256 columns is exact on the fp32 accumulators: tcgen05.ld.red returns
+// the minimum of every 16 columns with the load (four loads in flight per
+// wait), which gives the best value and its 16-column chunk, and an
+// elementwise minimum across the chunks gives its position inside the chunk;
+// an exact tie (the minimum in two chunks or two positions) is rescanned
+// column by column.  The residual lives only in the operand tiles: each stage
+// adds the chosen codeword's fp16 hi/lo halves (from the stage buffer) to
+// hi + lo (exact in fp32) and splits the sum again, so |t| stays below
+// 2^12 + S 2^9 < 2^14 and fp16 never overflows; a change of the stage scale
+// e re-derives er.  The next pair's input rows are loaded into registers
 // during the last stage.  Both tiles of a pair share each stage's operands, so
 // one tile's epilogue overlaps the other's MMAs.
 namespace v2 {
@@ -421,20 +425,21 @@ constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epil
 constexpr int kThreads = kWarps * 32;
 constexpr int A_TILE = kRows * 128;          // 16 KB: 128 rows x 64 fp16 (128-byte swizzle)
 constexpr int A_SLOT = 2 * A_TILE;           // hi + lo
-constexpr int A_AUG = kRows * 32;            // 4 KB: 128 rows x 16 fp16 (core-matrix layout), constant
+constexpr int A_AUG = kRows * 32;            // 4 KB per slot: 128 rows x 16 fp16 (core-matrix layout)
 constexpr int B_TILE = kCodes * 128;         // 32 KB
 constexpr int B_AUG = kCodes * 32;           // 8 KB
 constexpr int B_BUF = 2 * B_TILE + B_AUG;    // 72 KB
 constexpr int OFF_A = 0;
 constexpr int OFF_AAUG = 2 * A_SLOT;
-constexpr int OFF_B = OFF_AAUG + A_AUG;      // 68 KB: 1024-aligned
+constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 72 KB: 1024-aligned
 constexpr int OFF_BAR = OFF_B + 2 * B_BUF;   // b_full[2], b_empty[2], a_ready[2], acc_full[2], drain
 constexpr int OFF_SLOT = OFF_BAR + 80;
 constexpr int OFF_LO = OFF_SLOT + 16;        // per slot: the pair whose first-stage lo operand is nonzero
 constexpr int OFF_ABORT = OFF_LO + 16;
 constexpr int END = OFF_ABORT + 16;
 constexpr int SMEM = END + 1024;
-constexpr float kFastLimit = 16384.0f;       // |r'| below 2^14: fp16 operands in range
+constexpr int kRowLog = 12;                  // a row's operand starts below 2^12
+constexpr int kAugMaxShift = 34;             // 2^(10 - er) stays an fp16 (2^-24 subnormal at most)
 }  // namespace v2
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar)
@@ -489,19 +494,6 @@ __device__ __forceinline__ float max3f(float a, float b, float c)
     return d;
 }
 
-// x0 += w.lo / 2, x1 += w.hi / 2 for the two fp16 halves of w, each one
-// mixed-precision FMA (exact product, one rounding).
-__device__ __forceinline__ void add_half2_halved(uint32_t w, float &x0, float &x1)
-{
-    asm("{\n\t.reg .b16 l, h, c;\n\t"
-        "mov.b32 {l, h}, %2;\n\t"
-        "mov.b16 c, 0x3800;\n\t"
-        "fma.rn.f32.f16 %0, l, c, %0;\n\t"
-        "fma.rn.f32.f16 %1, h, c, %1;\n\t}"
-        : "+f"(x0), "+f"(x1)
-        : "r"(w));
-}
-
 // hi = fp16(a) (packed pair), lo = fp16(a - hi); a - hi is exact in fp32.
 __device__ __forceinline__ void split_half2(float a0, float a1, uint32_t &hi, uint32_t &lo)
 {
@@ -529,153 +521,149 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t *r)
         : "memory");
 }
 
-// Columns [c, c + 32) of this thread's accumulator row as two 16-column
-// chunks a and b, with their minima ra and rb (tcgen05.ld.red), loads and
-// wait in one statement.
-__device__ __forceinline__ void tmem_red2x16(uint32_t taddr, float *a, float *b, float &ra, float &rb)
+// Columns [c, c + 64) of this thread's accumulator row as four 16-column
+// chunks with their minima (tcgen05.ld.red), all four loads in flight before
+// the one wait.
+__device__ __forceinline__ void tmem_red4x16(uint32_t taddr, float *a, float *b, float *c, float *d, float &ra,
+                                             float &rb, float &rc, float &rd)
 {
     asm volatile(
-        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, %32, [%34];\n\t"
-        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %33, [%34+16];\n\t"
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, %64, [%68+0];\n\t"
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %65, [%68+16];\n\t"
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, %66, [%68+32];\n\t"
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.min.f32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, %67, [%68+48];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
-        : "=f"(a[0]), "=f"(a[1]), "=f"(a[2]), "=f"(a[3]), "=f"(a[4]), "=f"(a[5]), "=f"(a[6]), "=f"(a[7]), "=f"(a[8]), "=f"(a[9]), "=f"(a[10]), "=f"(a[11]), "=f"(a[12]), "=f"(a[13]), "=f"(a[14]), "=f"(a[15]), "=f"(b[0]), "=f"(b[1]), "=f"(b[2]), "=f"(b[3]), "=f"(b[4]), "=f"(b[5]), "=f"(b[6]), "=f"(b[7]), "=f"(b[8]), "=f"(b[9]), "=f"(b[10]), "=f"(b[11]), "=f"(b[12]), "=f"(b[13]), "=f"(b[14]), "=f"(b[15]),
-          "=f"(ra), "=f"(rb)
+        : "=f"(a[0]), "=f"(a[1]), "=f"(a[2]), "=f"(a[3]), "=f"(a[4]), "=f"(a[5]), "=f"(a[6]), "=f"(a[7]), "=f"(a[8]), "=f"(a[9]), "=f"(a[10]), "=f"(a[11]), "=f"(a[12]), "=f"(a[13]), "=f"(a[14]), "=f"(a[15]), "=f"(b[0]), "=f"(b[1]), "=f"(b[2]), "=f"(b[3]), "=f"(b[4]), "=f"(b[5]), "=f"(b[6]), "=f"(b[7]), "=f"(b[8]), "=f"(b[9]), "=f"(b[10]), "=f"(b[11]), "=f"(b[12]), "=f"(b[13]), "=f"(b[14]), "=f"(b[15]), "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3]), "=f"(c[4]), "=f"(c[5]), "=f"(c[6]), "=f"(c[7]), "=f"(c[8]), "=f"(c[9]), "=f"(c[10]), "=f"(c[11]), "=f"(c[12]), "=f"(c[13]), "=f"(c[14]), "=f"(c[15]), "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3]), "=f"(d[4]), "=f"(d[5]), "=f"(d[6]), "=f"(d[7]), "=f"(d[8]), "=f"(d[9]), "=f"(d[10]), "=f"(d[11]), "=f"(d[12]), "=f"(d[13]), "=f"(d[14]), "=f"(d[15]), "=f"(ra), "=f"(rb), "=f"(rc), "=f"(rd)
         : "r"(taddr));
 }
 
-// Scale the residual row by a power of two.
-__device__ __forceinline__ void scale_row(float *r, float f)
+// Row shift er >= 0 that brings a row of magnitude m below 2^12 (0 when it
+// already is, or when m is not a number).
+__device__ __forceinline__ int row_shift(float m)
 {
-#pragma unroll
-    for (int i = 0; i < 64; ++i)
-        r[i] *= f;
+    if (!(m >= 4096.0f))
+        return 0;
+    if (isinf(m))
+        return 116;
+    int E;
+    frexpf(m, &E);                         // m < 2^E
+    return E - v2::kRowLog;
 }
 
-// Store the hi/lo split of the scaled residual r' into this row of the
-// operand tile.  *fast tells whether every |r'| stays below the fast-path
-// limit; with NZ the return value tells whether any lo is nonzero.
-template <bool NZ>
-__device__ __forceinline__ bool write_operands(uint8_t *ahi, uint8_t *alo, int row, const float *r, bool *fast)
+// The norm operand's row: columns 0..2 hold 2^(10 - er) (times the three
+// parts of ||c'||^2 2^-10 in B), the rest zero; far-out rows (er > 34), whose
+// norm term is below the accumulator's resolution, hold zero.
+__device__ __forceinline__ void write_aug_row(uint8_t *aaug, int row, int er)
 {
+    const float s = er <= v2::kAugMaxShift ? ldexpf(1024.0f, -er) : 0.0f;
+    *reinterpret_cast<uint4 *>(aaug + core16_off(row, 0)) =
+        make_uint4(pack_half2(s, s), pack_half2(s, 0.0f), 0u, 0u);
+    *reinterpret_cast<uint4 *>(aaug + core16_off(row, 1)) = make_uint4(0u, 0u, 0u, 0u);
+}
+
+// Store 8 values as chunk c of this row's hi/lo operand tiles; returns the
+// nonzero bits of the lo halves.
+__device__ __forceinline__ uint32_t store_chunk(uint8_t *ahi, uint8_t *alo, int row, int c, const float *v)
+{
+    uint4 hv, lv;
+    uint32_t *hw = &hv.x, *lw = &lv.x;
     uint32_t nz = 0;
-    float mx = 0.0f;
 #pragma unroll
-    for (int c = 0; c < 8; ++c) {
-        uint4 hv, lv;
-        uint32_t *hw = &hv.x, *lw = &lv.x;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float a0 = r[c * 8 + 2 * i], a1 = r[c * 8 + 2 * i + 1];
-            split_half2(a0, a1, hw[i], lw[i]);
-            mx = max3f(mx, fabsf(a0), fabsf(a1));
-            if (NZ)
-                nz |= lw[i] & 0x7FFF7FFFu;   // either sign of zero counts as zero
-        }
-        const uint32_t off = swz(row, c);
-        *reinterpret_cast<uint4 *>(ahi + off) = hv;
-        *reinterpret_cast<uint4 *>(alo + off) = lv;
+    for (int i = 0; i < 4; ++i) {
+        split_half2(v[2 * i], v[2 * i + 1], hw[i], lw[i]);
+        nz |= lw[i] & 0x7FFF7FFFu;       // either sign of zero counts as zero
     }
-    *fast = mx < v2::kFastLimit;
-    return nz != 0;
+    const uint32_t off = swz(row, c);
+    *reinterpret_cast<uint4 *>(ahi + off) = hv;
+    *reinterpret_cast<uint4 *>(alo + off) = lv;
+    return nz;
 }
 
+// Chunk c of this row's operand as 8 floats hi + lo (exact: lo lies at least
+// 11 bits below hi).
+__device__ __forceinline__ void load_chunk(const uint8_t *ahi, const uint8_t *alo, int row, int c, float *v)
+{
+    const uint32_t off = swz(row, c);
+    const uint4 hv = *reinterpret_cast<const uint4 *>(ahi + off);
+    const uint4 lv = *reinterpret_cast<const uint4 *>(alo + off);
+    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+    const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 h = __half22float2(*reinterpret_cast<const __half2 *>(&hw[i]));
+        const float2 l = __half22float2(*reinterpret_cast<const __half2 *>(&lw[i]));
+        v[2 * i] = h.x + l.x;
+        v[2 * i + 1] = h.y + l.y;
+    }
+}
+
+// v += (hi + lo) f for the 8 codeword halves of chunk hv/lv (hi + lo exact in
+// fp32, one rounding per element).
+__device__ __forceinline__ void add_codeword(uint4 hv, uint4 lv, float f, float *v)
+{
+    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+    const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 h = __half22float2(*reinterpret_cast<const __half2 *>(&hw[i]));
+        const float2 l = __half22float2(*reinterpret_cast<const __half2 *>(&lw[i]));
+        v[2 * i] = fmaf(h.x + l.x, f, v[2 * i]);
+        v[2 * i + 1] = fmaf(h.y + l.y, f, v[2 * i + 1]);
+    }
+}
+
+// Eight consecutive input elements (chunk c of the row) as floats.
 template <int ESZ>
-__device__ __forceinline__ void unpack_row64(const uint4 *xr, int dtype, float *r)
+__device__ __forceinline__ void unpack8(const uint4 *xr, int dtype, int c, float *v)
 {
     if (ESZ == 4) {
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-            r[4 * c] = __uint_as_float(xr[c].x);
-            r[4 * c + 1] = __uint_as_float(xr[c].y);
-            r[4 * c + 2] = __uint_as_float(xr[c].z);
-            r[4 * c + 3] = __uint_as_float(xr[c].w);
-        }
+        const uint4 a = xr[2 * c], b = xr[2 * c + 1];
+        v[0] = __uint_as_float(a.x); v[1] = __uint_as_float(a.y);
+        v[2] = __uint_as_float(a.z); v[3] = __uint_as_float(a.w);
+        v[4] = __uint_as_float(b.x); v[5] = __uint_as_float(b.y);
+        v[6] = __uint_as_float(b.z); v[7] = __uint_as_float(b.w);
     } else {
+        const uint32_t w[4] = {xr[c].x, xr[c].y, xr[c].z, xr[c].w};
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            const uint32_t w[4] = {xr[c].x, xr[c].y, xr[c].z, xr[c].w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                float2 f;
-                if (dtype == FKV_F16)
-                    f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
-                else
-                    f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
-                r[8 * c + 2 * i] = f.x;
-                r[8 * c + 2 * i + 1] = f.y;
-            }
+        for (int i = 0; i < 4; ++i) {
+            float2 f;
+            if (dtype == FKV_F16)
+                f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+            else
+                f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
         }
     }
 }
 
-// Exact fp32 scoring of one scaled row against the 256 codewords of a buffer
-// (c' = -(hi + lo) / 2), for rows outside the fast path.  Lowest index on ties;
-// *dmin receives the best squared distance.
-__device__ __forceinline__ int slow_argmin(const float *r, const uint8_t *bb, float *dmin)
-{
-    float best = INFINITY;
-    int bidx = 0;
-#pragma unroll 1
-    for (int j = 0; j < kCodes; ++j) {
-        float d = 0.0f;
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-            const uint32_t off = swz(j, c);
-            const uint4 hv = *reinterpret_cast<const uint4 *>(bb + off);
-            const uint4 lv = *reinterpret_cast<const uint4 *>(bb + v2::B_TILE + off);
-            const __half2 *hh = reinterpret_cast<const __half2 *>(&hv);
-            const __half2 *ll = reinterpret_cast<const __half2 *>(&lv);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 h = __half22float2(hh[i]), l = __half22float2(ll[i]);
-                const float t0 = r[c * 8 + 2 * i] + 0.5f * (h.x + l.x);
-                const float t1 = r[c * 8 + 2 * i + 1] + 0.5f * (h.y + l.y);
-                d = fmaf(t0, t0, d);
-                d = fmaf(t1, t1, d);
-            }
-        }
-        if (d < best) {
-            best = d;
-            bidx = j;
-        }
-    }
-    *dmin = best;
-    return bidx;
-}
-
-// Argmin of one accumulator row (warp-collective: every lane of the warp
-// calls it).  Returns bc * 16 + p, where bc is the first 16-column chunk whose
-// minimum (from tcgen05.ld.red) equals the row minimum and p the position at
-// which the elementwise minimum across chunks equals it.  When the row minimum
-// is held by exactly one chunk and one position, that column is the unique
-// argmin; otherwise (an exact tie, or no finite value) *amb is set and the
-// caller rescans.  *vmin receives the row minimum.
-__device__ __forceinline__ int argmin_row(uint32_t trow, bool *amb, float *vmin)
+// Argmin of one accumulator row as argmin_row, reading four 16-column chunks
+// per tensor-memory wait.
+__device__ __forceinline__ int argmin_row4(uint32_t trow, bool *amb, float *vmin)
 {
     float m[16];
     float best = INFINITY;
     int bc = 0;
     bool tie = false;
 #pragma unroll 1
-    for (int c = 0; c < kCodes / 16; c += 2) {
-        float a[16], b[16], ra, rb;
-        tmem_red2x16(trow + c * 16, a, b, ra, rb);
+    for (int c = 0; c < kCodes / 16; c += 4) {
+        float a[16], b[16], d[16], e[16], ra, rb, rd, re;
+        tmem_red4x16(trow + c * 16, a, b, d, e, ra, rb, rd, re);
 #pragma unroll
-        for (int p = 0; p < 16; ++p)
-            m[p] = c == 0 ? fminf(a[p], b[p]) : min3f(m[p], a[p], b[p]);
-        if (ra < best) {
-            best = ra;
-            bc = c;
-            tie = false;
-        } else if (ra == best) {
-            tie = true;
+        for (int p = 0; p < 16; ++p) {
+            const float t = fminf(min3f(a[p], b[p], d[p]), e[p]);
+            m[p] = c == 0 ? t : fminf(m[p], t);
         }
-        if (rb < best) {
-            best = rb;
-            bc = c + 1;
-            tie = false;
-        } else if (rb == best) {
-            tie = true;
+        const float rr[4] = {ra, rb, rd, re};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            if (rr[i] < best) {
+                best = rr[i];
+                bc = c + i;
+                tie = false;
+            } else if (rr[i] == best) {
+                tie = true;
+            }
         }
     }
     uint32_t pm = 0;
@@ -746,14 +734,6 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         fence_mbar_init();
         prefetch_tmap(&tmap);
     }
-    // the norm operand of A: columns 0..2 hold 2^10 (times the three parts of
-    // ||c'||^2 2^-10 in B), the rest zero
-    for (int i = tid; i < kRows; i += v2::kThreads) {
-        *reinterpret_cast<uint4 *>(base + OFF_AAUG + core16_off(i, 0)) =
-            make_uint4(pack_half2(1024.0f, 1024.0f), pack_half2(1024.0f, 0.0f), 0u, 0u);
-        *reinterpret_cast<uint4 *>(base + OFF_AAUG + core16_off(i, 1)) = make_uint4(0u, 0u, 0u, 0u);
-    }
-    fence_proxy_async_smem();
     if (warp == 1)
         tmem_alloc(sbase + OFF_SLOT, 512);
     tc_fence_before();
@@ -805,7 +785,6 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
-            const uint64_t daug = sdesc_core16(sbase + OFF_AAUG);
             int it = 0;
             uint32_t aph[2] = {0, 0};
             int pc = 0;
@@ -832,7 +811,8 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                             const uint32_t ab = sbase + OFF_A + k * A_SLOT;
                             const uint32_t acc = tmem + k * 256;
                             // codeword norms first (K = 16, no swizzle), then the split dot products
-                            umma_f16(acc, daug, sdesc_core16(bb + 2 * B_TILE), idesc, 0);
+                            umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(bb + 2 * B_TILE),
+                                     idesc, 0);
 #pragma unroll
                             for (int kk = 0; kk < 4; ++kk) {
                                 const uint64_t dah = sdesc_sw128(ab + kk * 32);
@@ -861,6 +841,7 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
         const uint32_t trow = tmem + k * 256 + (static_cast<uint32_t>(quad * 32) << 16);
         uint8_t *ahi = base + OFF_A + k * A_SLOT;
         uint8_t *alo = ahi + A_TILE;
+        uint8_t *aaug = base + OFF_AAUG + k * A_AUG;
         uint4 xr[XN];
         auto row_src = [&](int p, bool *in) -> const uint4 * {
             const int g = p / pairs_per_group, q = p - g * pairs_per_group;
@@ -911,14 +892,38 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             const int tile = 2 * q + k;
             const int64_t v = static_cast<int64_t>(tile) * kRows + row;
             const bool valid = tile < tiles && v < nvec;
-            float r[64];
-            unpack_row64<ESZ>(xr, a.dtype, r);
+            // the row's operand t = x 2^-(e + er): e the stage scale of the
+            // codebooks, er >= 0 the row shift keeping |t| below 2^12
             int e = __ldg(&a.escale_h[g * S]);
-            scale_row(r, pow2f(-e));
-            bool fast;
+            int er;
             ++pc;
-            if (write_operands<true>(ahi, alo, row, r, &fast))
-                lo_stamp[k] = pc;
+            {
+                const float se = pow2f(-e);
+                float mx = 0.0f;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    float f[8];
+                    unpack8<ESZ>(xr, a.dtype, c, f);
+#pragma unroll
+                    for (int i = 0; i < 8; i += 2)
+                        mx = max3f(mx, fabsf(f[i] * se), fabsf(f[i + 1] * se));
+                }
+                er = row_shift(mx);
+                const float sr = pow2f(-er);
+                uint32_t nz = 0;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    float f[8];
+                    unpack8<ESZ>(xr, a.dtype, c, f);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        f[i] = f[i] * se * sr;
+                    nz |= store_chunk(ahi, alo, row, c, f);
+                }
+                write_aug_row(aaug, row, er);
+                if (nz)
+                    lo_stamp[k] = pc;
+            }
             fence_proxy_async_smem();
             mbar_arrive(bar(4 + k));
             Sym idx[8];
@@ -943,15 +948,13 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                     __syncwarp();
                     bool amb;
                     float vu;
-                    int j = argmin_row(trow, &amb, &vu);
-                    if (__any_sync(0xFFFFFFFFu, fast && amb)) {   // warp-collective loads: every lane takes part
+                    int j = argmin_row4(trow, &amb, &vu);
+                    if (__any_sync(0xFFFFFFFFu, amb)) {   // warp-collective loads: every lane takes part
                         const int jj = exact_argmin_tmem(trow);
                         if (amb)
                             j = jj;
                     }
                     tc_fence_before();
-                    if (!fast)
-                        j = slow_argmin(r, bb, &vu);
                     if (NB == 1 || u == 0 || vu < bv) {
                         bv = vu;
                         bidx = u * kCodes + j;
@@ -967,17 +970,16 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                     break;
                 idx[s] = static_cast<Sym>(bidx);
                 if (s == S - 1 && has_next)
-                    load_row(p + gridDim.x);      // r is dead from here: the next input takes its registers
-                if (s + 1 < S) {
-                    // r' <- r' - c'_bidx = r' + (hi + lo) / 2, the codeword read from the
-                    // stage buffer (one block) or from its global copy
+                    load_row(p + gridDim.x);      // the next pair's input, while this pair finishes
+                if (s + 1 < S && valid) {
+                    // t <- t - c'_bidx 2^-er = t + (hi + lo) 2^(-1-er), the codeword read
+                    // from the stage buffer (one block) or from its global copy
+                    const float f = pow2f(-1 - er);
                     const uint4 *gh = nullptr;
                     if (NB > 1)
                         gh = reinterpret_cast<const uint4 *>(a.cb16 +
                                                              ((static_cast<int64_t>(cgroup(g) * S + s) * 2) * KC + bidx) * 64);
-#pragma unroll
-                    for (int c = 0; c < 8; ++c) {
-                        uint4 hv, lv;
+                    auto codeword = [&](int c, uint4 &hv, uint4 &lv) {
                         if (NB == 1) {
                             const uint32_t bo = swz(bidx, c);
                             hv = *reinterpret_cast<const uint4 *>(bb + bo);
@@ -986,27 +988,58 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
                             hv = __ldg(gh + c);
                             lv = __ldg(gh + KC * 8 + c);
                         }
-                        const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
-                        const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
+                    };
+                    if (e_next == e) {
+                        // |t| stays below 2^12 + S 2^9 < 2^14: the row shift holds
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            add_half2_halved(hw[i], r[8 * c + 2 * i], r[8 * c + 2 * i + 1]);
-                            add_half2_halved(lw[i], r[8 * c + 2 * i], r[8 * c + 2 * i + 1]);
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            uint4 hv, lv;
+                            load_chunk(ahi, alo, row, c, t);
+                            codeword(c, hv, lv);
+                            add_codeword(hv, lv, f, t);
+                            store_chunk(ahi, alo, row, c, t);
                         }
+                    } else {
+                        // the next stage has another codebook scale: rescale the row and
+                        // choose its shift again from the updated magnitude
+                        float mx = 0.0f;
+#pragma unroll 1
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            uint4 hv, lv;
+                            load_chunk(ahi, alo, row, c, t);
+                            codeword(c, hv, lv);
+                            add_codeword(hv, lv, f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; i += 2)
+                                mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
+                        }
+                        int E = 0;
+                        if (mx > 0.0f)
+                            frexpf(mx, &E);                      // |t| < 2^E in units 2^-(e + er)
+                        const int tot = E + er + e - e_next;     // |r| < 2^tot in units 2^-e_next
+                        const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
+                        const float gsc = pow2f(er + e - e_next - er2);
+#pragma unroll 1
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            uint4 hv, lv;
+                            load_chunk(ahi, alo, row, c, t);
+                            codeword(c, hv, lv);
+                            add_codeword(hv, lv, f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                t[i] *= gsc;
+                            store_chunk(ahi, alo, row, c, t);
+                        }
+                        er = er2;
+                        write_aug_row(aaug, row, er);
                     }
                 }
                 mbar_arrive(bar(2 + bi));         // this thread is done with the stage buffer
                 if (s + 1 < S) {
-                    if (e_next != e) {            // uniform: one group per CTA at a time
-                        scale_row(r, pow2f(e - e_next));
-                        e = e_next;
-                    }
-                    if (!valid) {
-#pragma unroll
-                        for (int i = 0; i < 64; ++i)
-                            r[i] = 0.0f;
-                    }
-                    write_operands<false>(ahi, alo, row, r, &fast);
+                    e = e_next;
                     fence_proxy_async_smem();
                     mbar_arrive(bar(4 + k));
                 }
