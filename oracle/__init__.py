@@ -78,6 +78,10 @@ def _load():
         lib.oracle_rvq_encode.restype = None
         lib.oracle_rvq_decode.argtypes = [P, I64, I, P, I, I, P]
         lib.oracle_rvq_decode.restype = None
+        lib.oracle_ac_encode.argtypes = [P, I64, I, I, P, I64]
+        lib.oracle_ac_encode.restype = I64
+        lib.oracle_ac_decode.argtypes = [P, I64, I64, I, I, P]
+        lib.oracle_ac_decode.restype = I
         lib.oracle_threads.argtypes = []
         lib.oracle_threads.restype = I
         _lib = lib
@@ -353,4 +357,48 @@ def lossy_decode(pts, n: int, N: int, r: float, L: int, bits: int, keep_exact: i
     so a span's last symbols stay exact and its first ones degrade.  int32 [n]."""
     sym, _, _ = span_decode(lossy_points(pts, bits, keep_exact), n, N, r, L)
     return sym
+
+
+# ------------------------------------------- probability-weighted maps ---
+def ac_capacity_words(n: int, N: int) -> int:
+    """Words that always hold the code of n symbols: a step emits at most
+    log2(T / count) + 1 <= ceil(log2(N + n)) + 1 bits, plus two final bits."""
+    per = int(np.ceil(np.log2(N + n))) + 1
+    return (int(n) * per + 2 + 31) // 32 + 1
+
+
+def ac_encode(sym, N: int, adaptive: bool = True):
+    """Sec. 6 eq. (1): arithmetic coding of one stream (oracle_ac_encode).
+    Returns (uint32 words, number of bits)."""
+    s = np.ascontiguousarray(sym, dtype=np.int32).ravel()
+    if s.size and (s.min() < 0 or s.max() >= N):
+        raise ValueError("symbol outside the alphabet")
+    cap = ac_capacity_words(s.size, N)
+    out = np.zeros(cap, np.uint32)
+    nb = _load().oracle_ac_encode(_ptr(s), s.size, int(N), int(bool(adaptive)), _ptr(out), cap)
+    if nb < 0:
+        raise RuntimeError("code longer than its bound")
+    return out[:(nb + 31) // 32].copy(), int(nb)
+
+
+def ac_decode(words, nbits: int, n: int, N: int, adaptive: bool = True) -> np.ndarray:
+    """The inverse of ac_encode: int32 [n]."""
+    w = np.ascontiguousarray(words, dtype=np.uint32)
+    sym = np.empty(int(n), np.int32)
+    _load().oracle_ac_decode(_ptr(w), int(nbits), int(n), int(N), int(bool(adaptive)), _ptr(sym))
+    return sym
+
+
+def ac_model_bits(sym, N: int, adaptive: bool = True) -> float:
+    """Sec. 6: the model's code length -sum_k log2 p(c_k) in bits (float64),
+    p from the same add-one counts the coder uses."""
+    s = np.asarray(sym, dtype=np.int64).ravel()
+    if not adaptive:
+        return float(s.size * np.log2(N))
+    cnt = np.ones(N, np.float64)
+    bits = 0.0
+    for k, c in enumerate(s):                      # pure-Python loop: small cases
+        bits -= np.log2(cnt[c] / (N + k))
+        cnt[c] += 1.0
+    return bits
 

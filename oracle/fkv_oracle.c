@@ -25,6 +25,10 @@
  *                            of the running residual at each stage.
  *   oracle_rvq_decode     -- Sec. 3 "Setup": the reconstruction is the sum of the
  *                            s selected centroids.
+ *   oracle_ac_encode/decode -- Sec. 6 eq. (1): probability-weighted maps, i.e.
+ *                            arithmetic coding: [lo, hi) shrinks to the symbol's
+ *                            sub-interval of width p(c) at offset F(c), with p from
+ *                            add-one counts (adaptive) or 1/N (the uniform code).
  * Parity pins for every function live in tests/test_oracle_*.py.
  */
 #include <math.h>
@@ -220,6 +224,141 @@ void oracle_rvq_decode(const int32_t *idx, int64_t n, int D, const float *cb,
                 y[i * D + k] += (double)C[k];
         }
     }
+}
+
+/* Sec. 6 eq. (1): the probability-weighted map.  Encoding keeps an interval
+ * [lo, hi] and replaces it, for symbol c, by lo' = lo + w F(c),
+ * hi' = lo + w (F(c) + p(c)) - 1 with w = hi - lo + 1 -- the paper's recursion
+ * in 32-bit integer arithmetic (the finite-precision arithmetic coder of
+ * Witten, Neal and Cleary, CACM 1987): F(c) and p(c) are the cumulative count
+ * and count of c over the total T, so w F(c) is floor(w cum(c) / T).
+ * Whenever the interval lies in one half of [0, 2^32), the half's bit is
+ * settled: it is emitted, followed by any pending opposite bits, and the
+ * interval doubles; an interval straddling the middle inside the middle half
+ * doubles around it and adds one pending bit.  After the last symbol two bits
+ * (plus the pending ones) single out a point inside the final interval.
+ * Model: counts start at 1 for all N symbols and, when adaptive, the coded
+ * symbol's count grows by one after each step (the prequential add-one model);
+ * otherwise every p(c) stays 1/N, which is the uniform code.  Bits are written
+ * most significant first: stream bit i is bit 31 - i % 32 of word i / 32.
+ * Returns the number of bits, or -1 when out (cap words) is too small. */
+#define AC_HALF 0x80000000ull
+#define AC_QTR 0x40000000ull
+#define AC_3QTR 0xC0000000ull
+
+static int ac_put(uint32_t *out, int64_t cap, int64_t *nb, int bit)
+{
+    if (*nb >= cap * 32)
+        return -1;
+    if (bit)
+        out[*nb >> 5] |= 1u << (31 - (*nb & 31));
+    *nb += 1;
+    return 0;
+}
+
+int64_t oracle_ac_encode(const int32_t *sym, int64_t n, int N, int adaptive, uint32_t *out, int64_t cap)
+{
+    uint64_t lo = 0, hi = 0xFFFFFFFFull, total = (uint64_t)N;
+    int64_t follow = 0, nb = 0;
+    uint32_t cnt[4096];
+    if (N > 4096)
+        return -1;
+    for (int c = 0; c < N; ++c)
+        cnt[c] = 1;
+    for (int64_t i = 0; i < cap; ++i)
+        out[i] = 0;
+    for (int64_t k = 0; k < n; ++k) {
+        int c = sym[k];
+        uint64_t cum = 0;
+        for (int j = 0; j < c; ++j)
+            cum += cnt[j];
+        uint64_t w = hi - lo + 1;
+        hi = lo + w * (cum + cnt[c]) / total - 1;
+        lo = lo + w * cum / total;
+        for (;;) {
+            if (hi < AC_HALF) {
+                if (ac_put(out, cap, &nb, 0)) return -1;
+                for (; follow > 0; --follow)
+                    if (ac_put(out, cap, &nb, 1)) return -1;
+            } else if (lo >= AC_HALF) {
+                if (ac_put(out, cap, &nb, 1)) return -1;
+                for (; follow > 0; --follow)
+                    if (ac_put(out, cap, &nb, 0)) return -1;
+                lo -= AC_HALF;
+                hi -= AC_HALF;
+            } else if (lo >= AC_QTR && hi < AC_3QTR) {
+                follow += 1;
+                lo -= AC_QTR;
+                hi -= AC_QTR;
+            } else {
+                break;
+            }
+            lo = 2 * lo;
+            hi = 2 * hi + 1;
+        }
+        if (adaptive) {
+            cnt[c] += 1;
+            total += 1;
+        }
+    }
+    follow += 1;
+    int b = lo >= AC_QTR;
+    if (ac_put(out, cap, &nb, b)) return -1;
+    for (; follow > 0; --follow)
+        if (ac_put(out, cap, &nb, !b)) return -1;
+    return nb;
+}
+
+/* The inverse of oracle_ac_encode: the decoder holds the 32 stream bits that
+ * follow its interval's origin (bits past the end read as zero), finds the
+ * symbol whose sub-interval holds them and applies the same interval steps. */
+int oracle_ac_decode(const uint32_t *in, int64_t nbits, int64_t n, int N, int adaptive, int32_t *sym)
+{
+    uint64_t lo = 0, hi = 0xFFFFFFFFull, total = (uint64_t)N, val = 0;
+    int64_t pos = 0;
+    uint32_t cnt[4096];
+    if (N > 4096)
+        return -1;
+    for (int c = 0; c < N; ++c)
+        cnt[c] = 1;
+    for (int i = 0; i < 32; ++i, ++pos)
+        val = 2 * val + (pos < nbits ? (in[pos >> 5] >> (31 - (pos & 31))) & 1 : 0);
+    for (int64_t k = 0; k < n; ++k) {
+        uint64_t w = hi - lo + 1;
+        uint64_t target = ((val - lo + 1) * total - 1) / w;
+        int c = 0;
+        uint64_t cum = 0;
+        while (cum + cnt[c] <= target) {
+            cum += cnt[c];
+            ++c;
+        }
+        sym[k] = c;
+        hi = lo + w * (cum + cnt[c]) / total - 1;
+        lo = lo + w * cum / total;
+        for (;;) {
+            if (hi < AC_HALF) {
+            } else if (lo >= AC_HALF) {
+                lo -= AC_HALF;
+                hi -= AC_HALF;
+                val -= AC_HALF;
+            } else if (lo >= AC_QTR && hi < AC_3QTR) {
+                lo -= AC_QTR;
+                hi -= AC_QTR;
+                val -= AC_QTR;
+            } else {
+                break;
+            }
+            lo = 2 * lo;
+            hi = 2 * hi + 1;
+            val = 2 * val + (pos < nbits ? (in[pos >> 5] >> (31 - (pos & 31))) & 1 : 0);
+            ++pos;
+        }
+        if (adaptive) {
+            cnt[c] += 1;
+            total += 1;
+        }
+    }
+    return 0;
 }
 
 /* Thread count the OpenMP runtime will use (reported beside CPU timings). */
