@@ -221,6 +221,38 @@ int fkv_lossy_read(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride,
                    int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
                    const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
 
+/* ------------------------------------------ probability-weighted maps --- */
+
+/* Sec. 6 eq. (1): the iterated map with maps sized by a source model, i.e.
+ * arithmetic coding.  Each of n_streams streams of n symbols (laid out as in
+ * fkv_span_encode) is coded on its own, the streams side by side (decoding is
+ * sequential within a stream: there is no random access, append or in-place
+ * search on this form).  Integer form: a 32-bit interval [lo, hi]; symbol c
+ * with cumulative count cum(c), count cnt(c) and count total T gives, with
+ * w = hi - lo + 1, lo' = lo + floor(w cum(c) / T) and
+ * hi' = lo + floor(w (cum(c) + cnt(c)) / T) - 1; whenever the interval lies in
+ * one half of [0, 2^32) that half's bit is emitted (followed by the bits held
+ * back for a middle straddle) and the interval doubles; an interval inside the
+ * middle half doubles around the middle and holds back one bit; after the last
+ * symbol two bits (plus those held back) pick a point inside the interval.
+ * Model: counts start at 1 for all N symbols; adaptive = 1 adds one to the
+ * coded symbol's count after each step (add-one prequential model, code
+ * length close to -sum log2 p(c_k)); adaptive = 0 keeps p(c) = 1/N, the
+ * uniform code (log2 N bits per symbol).  n < 2^29.
+ * Output: words_dev uint32 [n_streams][word_stride], word_stride >=
+ * fkv_ac_capacity_words(ctx, n); stream bit i is bit 31 - i % 32 of word
+ * i / 32 (most significant first); nbits_dev int64 [n_streams] receives each
+ * stream's bit count.  A symbol >= N is coded as N - 1 and sets FKV_ECORRUPT. */
+int64_t fkv_ac_capacity_words(const fkv_ctx *ctx, int64_t n);
+int fkv_ac_encode(fkv_ctx *ctx, const void *sym_dev, int64_t n_streams, int64_t n, int64_t sym_stride, int adaptive,
+                  uint32_t *words_dev, int64_t word_stride, int64_t *nbits_dev, void *stream);
+
+/* The inverse of fkv_ac_encode: n symbols per stream from the codes (bits past
+ * a stream's nbits read as zero).  Bits that no code produces decode to some
+ * symbols and set FKV_ECORRUPT. */
+int fkv_ac_decode(fkv_ctx *ctx, const uint32_t *words_dev, int64_t word_stride, const int64_t *nbits_dev,
+                  int64_t n_streams, int64_t n, int adaptive, void *sym_dev, int64_t sym_stride, void *stream);
+
 /* -------------------------------------------------- K/V archive path ---- */
 
 /* A K or V cache tensor on the device: head vectors of `dim` contiguous

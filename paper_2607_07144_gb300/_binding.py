@@ -62,6 +62,9 @@ SIGNATURES = {
     "fkv_truncate": (_I, [_P, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P, _I64, _P]),
     "fkv_lossy_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P]),
     "fkv_lossy_read": (_I, [_P, _P, _I64, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P, _P]),
+    "fkv_ac_capacity_words": (_I64, [_P, _I64]),
+    "fkv_ac_encode": (_I, [_P, _P, _I64, _I64, _I64, _I, _P, _I64, _P, _P]),
+    "fkv_ac_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I, _P, _I64, _P]),
     "fkv_record_len": (_I, [_P]),
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
@@ -259,6 +262,31 @@ class Context:
                                             _ptr(counts), _stream(stream)))
         c = counts.cpu().tolist()
         return match[:min(c[0], cap)], c[0], c[1]
+
+    # -- Sec. 6 probability-weighted maps (arithmetic coding)
+    def ac_encode(self, sym: torch.Tensor, adaptive: bool = True, words: torch.Tensor = None,
+                  nbits: torch.Tensor = None, stream=None):
+        """sym [n_streams, n] -> (words int32 [n_streams, capacity] holding the
+        uint32 code words, nbits int64 [n_streams])."""
+        ns, n = self._sym(sym).shape
+        cap = lib().fkv_ac_capacity_words(self._h, n)
+        if words is None:
+            words = torch.zeros((ns, cap), dtype=torch.int32, device=sym.device)
+        if nbits is None:
+            nbits = torch.empty(ns, dtype=torch.int64, device=sym.device)
+        self._check(lib().fkv_ac_encode(self._h, _ptr(sym), ns, n, _rows(sym), int(bool(adaptive)), _ptr(words),
+                                        _rows(words), _ptr(nbits), _stream(stream)))
+        return words, nbits
+
+    def ac_decode(self, words: torch.Tensor, nbits: torch.Tensor, n: int, adaptive: bool = True,
+                  sym: torch.Tensor = None, stream=None) -> torch.Tensor:
+        ns = words.shape[0]
+        if sym is None:
+            sym = torch.empty((ns, n), dtype=self.sym_dtype, device=words.device)
+        self._sym(sym)
+        self._check(lib().fkv_ac_decode(self._h, _ptr(words), _rows(words), _ptr(nbits), ns, n, int(bool(adaptive)),
+                                        _ptr(sym), _rows(sym), _stream(stream)))
+        return sym
 
     # -- Sec. 4 lossy archive
     def lossy_geometry(self, n: int, bits: int, keep_exact: int):

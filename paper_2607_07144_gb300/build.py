@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libfkv.so")
 INCLUDE = os.path.join(ROOT, "include")
-SOURCES = ["fkv_api.cu", "codec.cu", "rvq.cu", "gather.cu", "decode_static.cu"]
+SOURCES = ["fkv_api.cu", "codec.cu", "rvq.cu", "gather.cu", "decode_static.cu", "ac.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -617,6 +617,55 @@ int fkv_lossy_read(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride,
     return FKV_OK;
 }
 
+int64_t fkv_ac_capacity_words(const fkv_ctx *ctx, int64_t n)
+{
+    if (!ctx || n < 0)
+        return 0;
+    return ac_capacity_words(ctx->N, n);
+}
+
+int fkv_ac_encode(fkv_ctx *ctx, const void *sym_dev, int64_t n_streams, int64_t n, int64_t sym_stride, int adaptive,
+                  uint32_t *words_dev, int64_t word_stride, int64_t *nbits_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_streams < 0 || n < 0 || n >= (int64_t(1) << 29))
+        return fail(ctx, FKV_EINVAL, "size outside [0, 2^29)");
+    if (adaptive != 0 && adaptive != 1)
+        return fail(ctx, FKV_EINVAL, "adaptive must be 0 or 1");
+    if (n_streams == 0)
+        return FKV_OK;
+    if ((n > 0 && (!sym_dev || sym_stride < n || reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx))) ||
+        !words_dev || word_stride < ac_capacity_words(ctx->N, n) || reinterpret_cast<uintptr_t>(words_dev) % 4 ||
+        !nbits_dev || reinterpret_cast<uintptr_t>(nbits_dev) % 8)
+        return fail(ctx, FKV_EINVAL, "bad buffer, stride or alignment");
+    CK(launch_ac_encode(ctx, sym_dev, n_streams, n, sym_stride, adaptive, words_dev, word_stride, nbits_dev,
+                        as_stream(stream)),
+       "arithmetic encode launch");
+    return FKV_OK;
+}
+
+int fkv_ac_decode(fkv_ctx *ctx, const uint32_t *words_dev, int64_t word_stride, const int64_t *nbits_dev,
+                  int64_t n_streams, int64_t n, int adaptive, void *sym_dev, int64_t sym_stride, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_streams < 0 || n < 0 || n >= (int64_t(1) << 29))
+        return fail(ctx, FKV_EINVAL, "size outside [0, 2^29)");
+    if (adaptive != 0 && adaptive != 1)
+        return fail(ctx, FKV_EINVAL, "adaptive must be 0 or 1");
+    if (n_streams == 0 || n == 0)
+        return FKV_OK;
+    if (!sym_dev || sym_stride < n || reinterpret_cast<uintptr_t>(sym_dev) % sym_size(ctx) || !words_dev ||
+        word_stride < 1 || reinterpret_cast<uintptr_t>(words_dev) % 4 || !nbits_dev ||
+        reinterpret_cast<uintptr_t>(nbits_dev) % 8)
+        return fail(ctx, FKV_EINVAL, "bad buffer, stride or alignment");
+    CK(launch_ac_decode(ctx, words_dev, word_stride, nbits_dev, n_streams, n, adaptive, sym_dev, sym_stride,
+                        as_stream(stream)),
+       "arithmetic decode launch");
+    return FKV_OK;
+}
+
 int fkv_record_len(const fkv_ctx *ctx)
 {
     if (!ctx || !ctx->has_cb)

@@ -100,6 +100,13 @@ cudaError_t launch_lossy_decode(const fkv_ctx *c, const uint32_t *codes, int64_t
 cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
                               int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
                               const int64_t *req, int64_t n_req, void *out, cudaStream_t st);
+// ac.cu (Sec. 6 probability-weighted maps): words that always hold the code
+// of n symbols, and the warp-per-stream coder
+int64_t ac_capacity_words(int N, int64_t n);
+cudaError_t launch_ac_encode(const fkv_ctx *c, const void *sym, int64_t n_streams, int64_t n, int64_t sym_stride,
+                             int adaptive, uint32_t *words, int64_t word_stride, int64_t *nbits, cudaStream_t st);
+cudaError_t launch_ac_decode(const fkv_ctx *c, const uint32_t *words, int64_t word_stride, const int64_t *nbits,
+                             int64_t n_streams, int64_t n, int adaptive, void *sym, int64_t sym_stride, cudaStream_t st);
 // rvq.cu
 cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int64_t t0, int64_t t1,
                               void *sym, int64_t stream_stride, int64_t rec0, cudaStream_t st);
