@@ -345,6 +345,30 @@ def run_gpu(args, rank, world, local_rank):
                  "point_bytes": ns * (T + ts) * 16, "sym_err_truncated": err, "ok": ctx.sync_status() == 0}
         del codes, tail, lsym, exact
 
+    # Sec. 6 probability-weighted maps: this step's 96 archived index streams
+    # arithmetic-coded with the adaptive add-one model (one warp per stream;
+    # decoding is sequential within a stream), encode and decode
+    weighted = None
+    if not args.no_weighted:
+        words, nbits = ctx.ac_encode(sym)
+        wsym = torch.empty_like(sym)
+        ctx.ac_decode(words, nbits, sym.shape[1], sym=wsym)
+        torch.cuda.synchronize()
+        evw = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        reps = 3
+        evw[0].record(stream)
+        for _ in range(reps):
+            ctx.ac_encode(sym, words=words, nbits=nbits)
+        evw[1].record(stream)
+        for _ in range(reps):
+            ctx.ac_decode(words, nbits, sym.shape[1], sym=wsym)
+        evw[2].record(stream)
+        torch.cuda.synchronize()
+        weighted = {"encode": evw[0].elapsed_time(evw[1]) / reps, "decode": evw[1].elapsed_time(evw[2]) / reps,
+                    "symbols": sym.numel(), "bits": int(nbits.sum().item()), "exact": bool(torch.equal(wsym, sym)),
+                    "ok": ctx.sync_status() == 0}
+        del words, nbits, wsym
+
     # Table 2's pooled RVQ 1024 x 2 archive on the same GPT-2 shape: one
     # 1024-codeword codebook per layer and stage shared by the 12 heads,
     # uint16 symbols (N = 1024, r_1024, span 5); archive write and full read
@@ -394,7 +418,7 @@ def run_gpu(args, rank, world, local_rank):
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
                 R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024,
-                lossy=lossy)
+                lossy=lossy, weighted=weighted)
 
 
 def roofline(res, peaks, launches_traffic=None):
@@ -501,6 +525,7 @@ def main():
     ap.add_argument("--no-suffix", action="store_true")
     ap.add_argument("--no-k1024", action="store_true")
     ap.add_argument("--no-lossy", action="store_true")
+    ap.add_argument("--no-weighted", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -588,6 +613,16 @@ def main():
             "decode_symbols_per_s": lx["symbols"] / (lx["decode"] * 1e-3),
             "archive_bytes": lx["code_bytes"] + lx["tail_bytes"], "exact_archive_bytes": lx["point_bytes"],
             "symbol_error_rate_truncated_spans": lx["sym_err_truncated"], "status_ok": lx["ok"]}
+    if res["weighted"]:
+        wx = res["weighted"]
+        kernels["probability-weighted maps (Sec. 6)"] = {
+            "workload": "this step's 96 archived RVQ index streams (989 records x 72 symbols, N=256), adaptive "
+                        "add-one model, one warp per stream",
+            "encode_ms": wx["encode"], "decode_ms": wx["decode"], "bound": "latency (sequential within a stream)",
+            "encode_symbols_per_s": wx["symbols"] / (wx["encode"] * 1e-3),
+            "decode_symbols_per_s": wx["symbols"] / (wx["decode"] * 1e-3),
+            "bits_per_symbol": wx["bits"] / wx["symbols"], "uniform_bits_per_symbol": 8.0,
+            "lossless": wx["exact"], "status_ok": wx["ok"]}
     units = res["units"] * world
     value = units / (ms * 1e-3)
     cpu = None
