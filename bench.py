@@ -54,10 +54,10 @@ def load_peaks():
 
 
 # DRAM bytes (read + write) per k_rvq64 launch of this workload, the mean of
-# the key launch (197,753,856) and the value launch (171,147,008) from one ncu
+# the key launch (197,526,272) and the value launch (171,083,008) from one ncu
 # capture of the current kernel (profiles/k_rvq64_gpt2_full_cache.md); set it
 # to None whenever that kernel changes until it is captured again.
-RVQ_DRAM_BYTES_PER_LAUNCH = None
+RVQ_DRAM_BYTES_PER_LAUNCH = 184304640
 
 # FP64 add/mul issue rate measured on this machine's GB300 (1.6 per clock per SM,
 # 504 Gop/s at the clock of that run); the span encoder is bound by it.
