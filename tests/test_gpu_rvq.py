@@ -6,6 +6,8 @@ earlier stages agreed); closer ties are counted and reported.  Rebuilt K/V:
 float32 sums within 1e-3 of the oracle's float64 sums, and fp16/bf16 outputs
 equal to the oracle sum rounded to nearest-even except where the float32
 summation error bound straddles a rounding boundary."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -198,6 +200,39 @@ def test_edge_vectors(fkv, oracle_mod, dim):
         assert idx[0, 0] == 9
         if n > 5:
             assert idx[1, 0] == 77 and idx[5, 0] == 3
+
+
+@pytest.mark.parametrize("k1024", [False, True])
+def test_extreme_magnitudes_and_stage_scale_change(fkv, oracle_mod, k1024):
+    """Rows far outside the codebook (1e20, 1e30), far inside it (1e-30,
+    subnormal), and a second stage 1e4 times smaller than the first (its
+    codebook takes another power-of-two scale, so every row is rescaled and its
+    shift chosen again between the stages), with 256 and 1024 codewords."""
+    dim, K = 64, (1024 if k1024 else 256)
+    rng = np.random.default_rng(11 + k1024)
+    cbk = rng.normal(size=(1, 1, 2, K, dim)).astype(np.float32)
+    cbk[0, 0, 1] *= 1e-4
+    cbv = rng.normal(size=(1, 1, 1, K, dim)).astype(np.float32)
+    n = 400
+    x = rng.normal(size=(n, dim))
+    x[:50] += cbk[0, 0, 0, rng.integers(0, K, 50)] * 3.0
+    x[50:60] *= 1e20
+    x[60:70] *= 1e30
+    x[70:80] *= 1e-30
+    x[80:90] *= 1e-40                                   # float32 subnormals
+    x[90:200] = cbk[0, 0, 0, rng.integers(0, K, 110)] + 0.5 * cbk[0, 0, 1, rng.integers(0, K, 110)]
+    cfg = dataclasses.replace(_one_group_cfg(dim, "f32", n), N=K)
+    X = torch.from_numpy(x.astype(np.float32)).reshape(1, 1, 1, n, dim).cuda()
+    ctx = fkv.Context(K, codebooks=(cbk, cbv))
+    sym = torch.zeros((1, n * 3), dtype=ctx.sym_dtype, device="cuda")
+    ctx.rvq_encode(0, X, 0, n, sym)
+    ctx.rvq_encode(1, X, 0, n, sym)
+    assert ctx.sync_status() == 0
+    idx = sym.cpu().numpy().astype(np.int32).reshape(n, 3)
+    assert idx.max() < K
+    oi, gap = oracle_mod.rvq_encode(x.astype(np.float32).astype(np.float64), cbk[0, 0])
+    hard, near, seen = compare_rvq(idx[:, :2], oi, gap)
+    assert hard == 0, hard
 
 
 def test_strided_cache_view(fkv, oracle_mod):
