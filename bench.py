@@ -244,8 +244,9 @@ def run_gpu(args, rank, world, local_rank):
                     s_in.wait_event(after)
                 if free[b] is not None:
                     s_in.wait_event(free[b])
-                Kd[b].copy_(Kh, non_blocking=True)
-                Vd[b].copy_(Vh, non_blocking=True)
+                # only the positions that leave the exact window travel
+                ctx.cache_upload(Kh, Kd[b], t0, t1 + 1, stream=s_in)
+                ctx.cache_upload(Vh, Vd[b], t0, t1 + 1, stream=s_in)
                 ev_in = torch.cuda.Event()
                 ev_in.record(s_in)
             stream.wait_event(ev_in)
@@ -276,7 +277,7 @@ def run_gpu(args, rank, world, local_rank):
         t2.record(stream)
         torch.cuda.synchronize()
         e2e_ms = s2.elapsed_time(t2) / args.steps
-        h2d = Kh.numel() * Kh.element_size() * 2
+        h2d = Kh[:, :, :, t0:t1 + 1].numel() * Kh.element_size() * 2
         d2h = ptsh[0].numel() * 8 + outh[0].numel() * outh[0].element_size()
         e2e = {"ms": e2e_ms, "h2d": h2d, "d2h": d2h}
 

@@ -328,6 +328,19 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
 int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
                          fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream);
 
+/* Host-to-device transfer of the positions that leave the exact window:
+ * copies positions [t0, t1) of every (layer, sequence, head) of src_host (a
+ * cache view of HOST memory, pinned for full speed) into the same positions
+ * of dst_dev (device), n_layers and n_heads from the context, asynchronously
+ * on `stream`; both views hold positions contiguously (stride_pos = dim) and
+ * share dtype and batch.  The archive path reads only these positions
+ * (Sec. 3 "Setup": the 4 sinks and the 32 recent positions stay exact), so an
+ * archive write need not move the rest of the cache.  One 2-D copy when the
+ * (layer, sequence, head) rows share one pitch on both sides, else one per
+ * (layer, sequence). */
+int fkv_cache_upload(fkv_ctx *ctx, const fkv_cache *src_host, const fkv_cache *dst_dev, int64_t t0, int64_t t1,
+                     void *stream);
+
 /* Sec. 2 random access at record granularity: for each request q,
  * req_dev[2q] = stream (b * n_layers + l), req_dev[2q + 1] = record index,
  * decode only the spans of that record and write its K and V head vectors to

@@ -71,6 +71,7 @@ SIGNATURES = {
     "fkv_decode_kv": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
     "fkv_decode_kv_static": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
     "fkv_read_kv": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _I, _P]),
+    "fkv_cache_upload": (_I, [_P, _P, _P, _I64, _I64, _P]),
     "fkv_streams_create": (_I, [_P, _I64, _I64, ctypes.POINTER(_P)]),
     "fkv_streams_destroy": (_I, [_P]),
     "fkv_streams_reset": (_I, [_P]),
@@ -123,11 +124,13 @@ def max_span_len(r: float) -> int:
     return lib().fkv_max_span_len(float(r))
 
 
-def cache_view(t: torch.Tensor) -> _Cache:
-    """fkv_cache view of a CUDA tensor shaped [n_layers, batch, n_heads, seq, dim]
-    (any strides with a contiguous last dimension)."""
-    if t.dim() != 5 or t.stride(4) != 1 or not t.is_cuda:
-        raise ValueError("cache must be a CUDA tensor [layers, batch, heads, seq, dim] with contiguous dim")
+def cache_view(t: torch.Tensor, host: bool = False) -> _Cache:
+    """fkv_cache view of a tensor shaped [n_layers, batch, n_heads, seq, dim]
+    (any strides with a contiguous last dimension): a CUDA tensor, or with
+    host=True a CPU tensor (pinned for full transfer speed)."""
+    if t.dim() != 5 or t.stride(4) != 1 or t.is_cuda == host:
+        raise ValueError("cache must be a %s tensor [layers, batch, heads, seq, dim] with contiguous dim"
+                         % ("CPU" if host else "CUDA"))
     c = _Cache()
     c.data = t.data_ptr()
     c.dtype = _DTYPE[t.dtype]
@@ -364,6 +367,12 @@ class Context:
         self._check(lib().fkv_decode_kv_static(self._h, _ptr(pts), n_rec, _rows(pts, 2),
                                                ctypes.byref(ck) if ck else None, ctypes.byref(cv) if cv else None,
                                                t0, _stream(stream)))
+
+    def cache_upload(self, src_host: torch.Tensor, dst: torch.Tensor, t0: int, t1: int, stream=None):
+        """Copy positions [t0, t1) of a host cache (CPU tensor, pinned) into a device cache."""
+        cs, cd = cache_view(src_host, host=True), cache_view(dst)
+        self._check(lib().fkv_cache_upload(self._h, ctypes.byref(cs), ctypes.byref(cd), t0, t1, _stream(stream)))
+        return dst
 
     def read_kv(self, pts: torch.Tensor, n_rec: int, req: torch.Tensor, out: torch.Tensor, stream=None):
         """req int64 [n_req, 2] = (stream, record) -> out [n_req, 2, heads, dim]."""

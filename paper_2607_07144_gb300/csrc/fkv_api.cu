@@ -758,6 +758,49 @@ int fkv_decode_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt
                           as_stream(stream));
 }
 
+int fkv_cache_upload(fkv_ctx *ctx, const fkv_cache *src_host, const fkv_cache *dst_dev, int64_t t0, int64_t t1,
+                     void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!ctx->has_cb)
+        return fail(ctx, FKV_EINVAL, "context has no codebooks");
+    if (!src_host || !dst_dev || !src_host->data || !dst_dev->data || src_host->dtype != dst_dev->dtype ||
+        src_host->batch != dst_dev->batch || src_host->batch <= 0)
+        return fail(ctx, FKV_EINVAL, "bad cache views");
+    if (t0 < 0 || t1 < t0 || t1 > src_host->seq || t1 > dst_dev->seq)
+        return fail(ctx, FKV_EINVAL, "bad position range");
+    const int64_t D = ctx->D;
+    if (src_host->stride_pos != D || dst_dev->stride_pos != D)
+        return fail(ctx, FKV_EINVAL, "positions must be contiguous (stride_pos = dim)");
+    if (t1 == t0)
+        return FKV_OK;
+    const int64_t esz = src_host->dtype == FKV_F32 ? 4 : 2;
+    const int64_t L = ctx->Ly, B = src_host->batch, H = ctx->H;
+    const int64_t width = (t1 - t0) * D * esz;
+    const uint8_t *s = static_cast<const uint8_t *>(src_host->data);
+    uint8_t *d = static_cast<uint8_t *>(dst_dev->data);
+    auto uniform = [&](const fkv_cache *c) {
+        return c->stride_batch == H * c->stride_head && c->stride_layer == B * c->stride_batch;
+    };
+    if (uniform(src_host) && uniform(dst_dev)) {
+        // every (layer, sequence, head) row at one pitch: a single 2-D copy
+        CK(cudaMemcpy2DAsync(d + t0 * D * esz, dst_dev->stride_head * esz, s + t0 * D * esz,
+                             src_host->stride_head * esz, width, L * B * H, cudaMemcpyHostToDevice,
+                             as_stream(stream)),
+           "cache upload");
+        return FKV_OK;
+    }
+    for (int64_t l = 0; l < L; ++l)
+        for (int64_t b = 0; b < B; ++b)
+            CK(cudaMemcpy2DAsync(d + (l * dst_dev->stride_layer + b * dst_dev->stride_batch + t0 * D) * esz,
+                                 dst_dev->stride_head * esz,
+                                 s + (l * src_host->stride_layer + b * src_host->stride_batch + t0 * D) * esz,
+                                 src_host->stride_head * esz, width, H, cudaMemcpyHostToDevice, as_stream(stream)),
+               "cache upload");
+    return FKV_OK;
+}
+
 int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
                 const int64_t *req_dev, int64_t n_req, void *out_dev, int dtype, void *stream)
 {

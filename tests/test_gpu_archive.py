@@ -76,6 +76,28 @@ def test_archive_round_trip(fkv, oracle_mod, base, cid):
     assert torch.equal(out[:, 1], Vr[ti(l), ti(b), :, ti(t)])
 
 
+def test_cache_upload_moves_only_the_archived_positions(fkv):
+    cfg = synth.small_config(synth.CFG1, 306, n_layers=2, batch=3, seq=36 + 50)
+    ctx = fkv.Context(256, codebooks=(synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)))
+    K = torch.from_numpy(synth.kv_cache(cfg, 0)).pin_memory()
+    dst = torch.full(cfg.cache_shape(), 7.0, dtype=K.dtype, device="cuda")
+    ctx.cache_upload(K, dst, cfg.t0, cfg.t1)
+    torch.cuda.synchronize()
+    want = torch.full(cfg.cache_shape(), 7.0, dtype=K.dtype)
+    want[:, :, :, cfg.t0:cfg.t1] = K[:, :, :, cfg.t0:cfg.t1]
+    assert torch.equal(dst.cpu(), want)
+    # a layout whose rows do not share one pitch: one copy per (layer, sequence)
+    big = torch.zeros((cfg.n_layers, cfg.batch + 1) + cfg.cache_shape()[2:], dtype=K.dtype).pin_memory()
+    big[:, 1:] = K
+    src = big[:, 1:]
+    dst2 = torch.zeros(cfg.cache_shape(), dtype=K.dtype, device="cuda")
+    ctx.cache_upload(src, dst2, 0, cfg.seq)
+    torch.cuda.synchronize()
+    assert torch.equal(dst2.cpu(), K)
+    with pytest.raises(fkv.FkvError):
+        ctx.cache_upload(K, dst, 10, 5)
+
+
 def test_decode_time_streaming(fkv, oracle_mod):
     """Config-4 pattern at reduced size: a prefilled archive, then steps that
     each append the token leaving the recent window (RVQ + tail append) and
