@@ -261,6 +261,38 @@ int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n
     return FKV_OK;
 }
 
+namespace {
+
+// Geometry of a lossy archive: truncated spans T and code words per stream.
+void lossy_geometry(const fkv_ctx *ctx, int64_t n, int bits, int64_t keep_exact, int64_t *T, int64_t *words,
+                    int64_t *tail_spans)
+{
+    const int64_t spans = (n + ctx->L - 1) / ctx->L;
+    *T = spans > keep_exact ? spans - keep_exact : 0;
+    *words = (2 * *T * bits + 31) / 32;
+    *tail_spans = spans - *T;
+}
+
+// Shared checks of the lossy calls; null on success, else the reason.
+const char *check_lossy(const fkv_ctx *ctx, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
+                        const void *codes, int64_t code_stride, const void *tail, int64_t tail_stride, bool need_tail)
+{
+    if (n_streams < 0 || n < 0 || keep_exact < 0)
+        return "negative size";
+    if (bits < 2 || bits > 53)
+        return "bits outside [2, 53]";
+    int64_t T, words, tail_spans;
+    lossy_geometry(ctx, n, bits, keep_exact, &T, &words, &tail_spans);
+    if (n_streams > 0 && words > 0 && (!codes || code_stride < words || reinterpret_cast<uintptr_t>(codes) % 4))
+        return "bad code buffer or stride";
+    if (n_streams > 0 && tail_spans > 0 && (need_tail || tail) &&
+        (!tail || tail_stride < tail_spans || reinterpret_cast<uintptr_t>(tail) % 16))
+        return "bad tail buffer or stride";
+    return nullptr;
+}
+
+}  // namespace
+
 extern "C" {
 
 double fkv_packing_ratio(int N)
@@ -525,37 +557,6 @@ int fkv_suffix_search(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, in
     return FKV_OK;
 }
 
-namespace {
-
-// Geometry of a lossy archive: truncated spans T and code words per stream.
-void lossy_geometry(const fkv_ctx *ctx, int64_t n, int bits, int64_t keep_exact, int64_t *T, int64_t *words,
-                    int64_t *tail_spans)
-{
-    const int64_t spans = (n + ctx->L - 1) / ctx->L;
-    *T = spans > keep_exact ? spans - keep_exact : 0;
-    *words = (2 * *T * bits + 31) / 32;
-    *tail_spans = spans - *T;
-}
-
-// Shared checks of the lossy calls; null on success, else the reason.
-const char *check_lossy(const fkv_ctx *ctx, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
-                        const void *codes, int64_t code_stride, const void *tail, int64_t tail_stride, bool need_tail)
-{
-    if (n_streams < 0 || n < 0 || keep_exact < 0)
-        return "negative size";
-    if (bits < 2 || bits > 53)
-        return "bits outside [2, 53]";
-    int64_t T, words, tail_spans;
-    lossy_geometry(ctx, n, bits, keep_exact, &T, &words, &tail_spans);
-    if (n_streams > 0 && words > 0 && (!codes || code_stride < words || reinterpret_cast<uintptr_t>(codes) % 4))
-        return "bad code buffer or stride";
-    if (n_streams > 0 && tail_spans > 0 && (need_tail || tail) &&
-        (!tail || tail_stride < tail_spans || reinterpret_cast<uintptr_t>(tail) % 16))
-        return "bad tail buffer or stride";
-    return nullptr;
-}
-
-}  // namespace
 
 int fkv_truncate(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride, int bits,
                  int64_t keep_exact, uint32_t *codes_dev, int64_t code_stride, double *tail_dev, int64_t tail_stride,
