@@ -142,8 +142,12 @@ class KVConfig:
 CFG0 = KVConfig(0, "gpt2-1layer-b1-t1024-f32", 1, 1, 12, 64, 1024, "f32", 2, 1, 4, 8.0, 0.0)
 CFG1 = KVConfig(1, "gpt2-12layer-b8-t1024-f16", 12, 8, 12, 64, 1024, "f16", 4, 2, 4, 8.0, 0.0)
 CFG3 = KVConfig(3, "llama3-8b-32layer-b4-t32768-bf16", 32, 4, 8, 128, 32768, "bf16", 4, 2, 3, 10.0, 0.5)
-# Decode-time streaming (Llama-3-8B shape, 64 sequences x 131072 prefilled).
-CFG4 = KVConfig(4, "llama3-8b-stream-b64-t131072-bf16", 32, 64, 8, 128, 131072 + 36, "bf16", 4, 2, 3, 10.0, 0.5)
+# Decode-time streaming (Llama-3-8B shape, 64 sequences): 131072 archived
+# positions prefilled, then 512 steps that each archive one more position; the
+# cache holds all of them plus the 4 + 32 exact window.
+CFG4 = KVConfig(4, "llama3-8b-stream-b64-t131072-bf16", 32, 64, 8, 128, 131072 + 512 + 36, "bf16", 4, 2, 3, 10.0,
+                0.5)
+CFG4_PREFILL, CFG4_STEPS = 131072, 512
 # Table 2's pooled rows at k = 1024 on the GPT-2 shape: RVQ 1024 x 2 and VQ 1024.
 CFG5 = KVConfig(5, "gpt2-12layer-b8-t1024-f16-pooled-rvq1024x2", 12, 8, 12, 64, 1024, "f16", 2, 2, 4, 8.0, 0.0,
                 N=1024, pooled=True)
@@ -319,24 +323,27 @@ def _gpu():
         if _syn is None:
             L = _ct.CDLL(build())
             i64, u32, u64, p = _ct.c_int64, _ct.c_uint32, _ct.c_uint64, _ct.c_void_p
-            L.synth_gen_kv.argtypes = [p, _ct.c_int, i64, i64, i64, i64, i64, u32, u32, u32, p, p]
+            L.synth_gen_kv.argtypes = [p, _ct.c_int, i64, i64, i64, i64, i64, i64, i64, u32, u32, u32, p, p]
             L.synth_gen_symbols.argtypes = [p, i64, u64, u32, u32, _ct.c_int, p, u32, u32, p]
             L.synth_gen_positions.argtypes = [p, i64, u64, u32, u64, u32, u32, i64, i64, p]
             _syn = L
         return _syn
 
 
-def gpu_kv_cache(cfg: KVConfig, kv: int, device="cuda", out=None):
+def gpu_kv_cache(cfg: KVConfig, kv: int, device="cuda", out=None, t0: int = 0, count: int = None):
     """The cache [Ly, B, H, T, D] generated on the device (torch tensor),
-    element for element equal to kv_cache()/kv_elements()."""
+    element for element equal to kv_cache()/kv_elements(); with t0/count only
+    positions [t0, t0 + count) of it, as [Ly, B, H, count, D] (for caches too
+    large to hold whole)."""
     import torch
     tdt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[cfg.dtype]
+    Ly, B, H, T, D = cfg.cache_shape()
+    C = T - t0 if count is None else int(count)
     if out is None:
-        out = torch.empty(cfg.cache_shape(), dtype=tdt, device=device)
+        out = torch.empty((Ly, B, H, C, D), dtype=tdt, device=device)
     scale = torch.from_numpy(channel_scale32(cfg, kv)).to(device)
     k0, k1 = seed_key(cfg.cfg_id)
-    Ly, B, H, T, D = cfg.cache_shape()
-    rc = _gpu().synth_gen_kv(out.data_ptr(), {"f32": 0, "f16": 1, "bf16": 2}[cfg.dtype], Ly, B, H, T, D,
+    rc = _gpu().synth_gen_kv(out.data_ptr(), {"f32": 0, "f16": 1, "bf16": 2}[cfg.dtype], Ly, B, H, T, D, int(t0), C,
                              TID_K if kv == 0 else TID_V, k0, k1, scale.data_ptr(),
                              torch.cuda.current_stream().cuda_stream)
     if rc != 0:

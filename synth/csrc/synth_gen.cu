@@ -41,16 +41,20 @@ __device__ __forceinline__ int irwin_hall(uint64_t e, uint32_t tid, uint32_t k0,
     return z - 262140;
 }
 
-// cache [Ly][B][H][T][D]; scale [Ly][H][D] float32.
-__global__ void k_gen_kv(void *out, int dtype, int64_t B, int64_t H, int64_t T, int64_t D, int64_t total,
-                         uint32_t tid, uint32_t k0, uint32_t k1, const float *scale)
+// Positions [t0, t0 + C) of the cache [Ly][B][H][T][D] into out [Ly][B][H][C][D];
+// every element keeps its flat index in the whole cache; scale [Ly][H][D] float32.
+__global__ void k_gen_kv(void *out, int dtype, int64_t B, int64_t H, int64_t T, int64_t D, int64_t t0, int64_t C,
+                         int64_t total, uint32_t tid, uint32_t k0, uint32_t k1, const float *scale)
 {
     for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < total;
          e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const int64_t d = e % D;
-        const int64_t h = (e / (D * T)) % H;
-        const int64_t l = e / (D * T * H * B);
-        const float x = __fmul_rn(static_cast<float>(irwin_hall(static_cast<uint64_t>(e), tid, k0, k1)),
+        const int64_t t = (e / D) % C;
+        const int64_t row = e / (D * C);               // (l * B + b) * H + h
+        const int64_t h = row % H;
+        const int64_t l = row / (H * B);
+        const int64_t ef = (row * T + t0 + t) * D + d; // flat index in the whole cache
+        const float x = __fmul_rn(static_cast<float>(irwin_hall(static_cast<uint64_t>(ef), tid, k0, k1)),
                                   scale[(l * H + h) * D + d]);
         if (dtype == 0)
             static_cast<float *>(out)[e] = x;
@@ -112,12 +116,12 @@ unsigned grid_for(int64_t n)
 
 extern "C" {
 
-int synth_gen_kv(void *out, int dtype, int64_t Ly, int64_t B, int64_t H, int64_t T, int64_t D, uint32_t tid,
-                 uint32_t k0, uint32_t k1, const float *scale, void *stream)
+int synth_gen_kv(void *out, int dtype, int64_t Ly, int64_t B, int64_t H, int64_t T, int64_t D, int64_t t0,
+                 int64_t C, uint32_t tid, uint32_t k0, uint32_t k1, const float *scale, void *stream)
 {
-    const int64_t total = Ly * B * H * T * D;
-    k_gen_kv<<<grid_for(total), 256, 0, static_cast<cudaStream_t>(stream)>>>(out, dtype, B, H, T, D, total, tid,
-                                                                             k0, k1, scale);
+    const int64_t total = Ly * B * H * C * D;
+    k_gen_kv<<<grid_for(total), 256, 0, static_cast<cudaStream_t>(stream)>>>(out, dtype, B, H, T, D, t0, C, total,
+                                                                             tid, k0, k1, scale);
     return static_cast<int>(cudaGetLastError());
 }
 
