@@ -370,6 +370,51 @@ def run_gpu(args, rank, world, local_rank):
                     "ok": ctx.sync_status() == 0}
         del words, nbits, wsym
 
+    # Llama-3-8B-shaped archive (32 layers x batch 4 x 8 KV heads x 32768
+    # positions x 128 dims, bf16, K 4 / V 2 stages): the same write and read
+    # path as the step above, on 128-dimensional heads
+    llama = None
+    if not args.no_llama:
+        c3 = synth.CFG3
+        lctx = fkv.Context(256, codebooks=(synth.codebooks(c3, 0), synth.codebooks(c3, 1)))
+        K3 = synth.gpu_kv_cache(c3, 0, device=dev)
+        V3 = synth.gpu_kv_cache(c3, 1, device=dev)
+        R3, P3, ns3 = lctx.record_len(), c3.n_archived, c3.batch * c3.n_layers
+        sym3 = torch.empty((ns3, P3 * R3), dtype=torch.uint8, device=dev)
+        pts3 = torch.empty((ns3, lctx.n_spans(P3 * R3), 2), dtype=torch.float64, device=dev)
+        K3r, V3r = torch.zeros_like(K3), torch.zeros_like(V3)
+        g3 = torch.Generator().manual_seed(9)
+        req3 = torch.stack([torch.randint(0, ns3, (N_READS,), generator=g3),
+                            torch.randint(0, P3, (N_READS,), generator=g3)], dim=1).to(dev)
+        out3 = torch.empty((N_READS, 2, c3.n_heads, c3.dim), dtype=K3.dtype, device=dev)
+        ev3 = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+
+        def step3(record=False):
+            r_ = (lambda i: ev3[i].record(stream)) if record else (lambda i: None)
+            r_(0)
+            lctx.rvq_encode(0, K3, c3.t0, c3.t1, sym3)
+            r_(1)
+            lctx.rvq_encode(1, V3, c3.t0, c3.t1, sym3)
+            r_(2)
+            lctx.span_encode(sym3, pts3)
+            r_(3)
+            lctx.decode_kv(pts3, P3, K3r, V3r, t0=c3.t0)
+            r_(4)
+            lctx.read_kv(pts3, P3, req3, out3)
+            r_(5)
+        step3()
+        acc = np.zeros(5)
+        reps = 3
+        for _ in range(reps):
+            step3(record=True)
+            torch.cuda.synchronize()
+            acc += np.array([ev3[i].elapsed_time(ev3[i + 1]) for i in range(5)])
+        acc /= reps
+        llama = {"phase": acc.tolist(), "records": ns3 * P3, "nvec": ns3 * P3 * c3.n_heads,
+                 "stages": (c3.stages_k, c3.stages_v), "R": R3, "L": lctx.L, "spans": ns3 * lctx.n_spans(P3 * R3),
+                 "out_bytes": 2 * ns3 * P3 * c3.n_heads * c3.dim * 2, "ok": lctx.sync_status() == 0}
+        del K3, V3, K3r, V3r, sym3, pts3, out3, lctx
+
     # Table 2's pooled RVQ 1024 x 2 archive on the same GPT-2 shape: one
     # 1024-codeword codebook per layer and stage shared by the 12 heads,
     # uint16 symbols (N = 1024, r_1024, span 5); archive write and full read
@@ -419,7 +464,7 @@ def run_gpu(args, rank, world, local_rank):
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
                 R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024,
-                lossy=lossy, weighted=weighted)
+                lossy=lossy, weighted=weighted, llama=llama)
 
 
 def roofline(res, peaks, launches_traffic=None):
@@ -527,6 +572,7 @@ def main():
     ap.add_argument("--no-k1024", action="store_true")
     ap.add_argument("--no-lossy", action="store_true")
     ap.add_argument("--no-weighted", action="store_true")
+    ap.add_argument("--no-llama", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -614,6 +660,24 @@ def main():
             "decode_symbols_per_s": lx["symbols"] / (lx["decode"] * 1e-3),
             "archive_bytes": lx["code_bytes"] + lx["tail_bytes"], "exact_archive_bytes": lx["point_bytes"],
             "symbol_error_rate_truncated_spans": lx["sym_err_truncated"], "status_ok": lx["ok"]}
+    if res["llama"]:
+        lx = res["llama"]
+        ph3 = lx["phase"]
+        rvq3 = ph3[0] + ph3[1]
+        tf3 = lx["nvec"] * sum(lx["stages"]) * 2 * 128 * 256 / (rvq3 * 1e-3) / 1e12
+        sym3 = lx["records"] * lx["R"]
+        dec3 = sym3 + lx["spans"] * 16 + lx["out_bytes"]
+        kernels["llama3-8b-shaped archive (config 3)"] = {
+            "workload": "32 layers x batch 4 x 8 KV heads x 32768 tok x 128 dims, bf16; 4+32 exact window; K 4 / V 2 "
+                        "RVQ stages x 256; N=256, r=r_256, L=6",
+            "records_per_s": lx["records"] / (sum(ph3) * 1e-3), "step_ms": sum(ph3),
+            "rvq_ms": rvq3, "rvq_tflops": tf3, "rvq_frac": tf3 / peaks["bf16_tflops"],
+            "rvq_kernel": "k_rvq128 (persistent, two tile slots, codebook streamed in 64-dim K blocks)",
+            "span_encode_ms": ph3[2], "span_encode_frac_fp64": sym3 * 6 / (ph3[2] * 1e-3) /
+            (FP64_OPS_PER_CLK_SM * 152 * (res["clocks"].get("sm_mhz") or 1900.0) * 1e6),
+            "decode_kv_ms": ph3[3], "decode_kv_gbs": dec3 / (ph3[3] * 1e-3) / 1e9,
+            "decode_kv_frac": dec3 / (ph3[3] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+            "read_kv_ms_4096": ph3[4], "status_ok": lx["ok"]}
     if res["weighted"]:
         wx = res["weighted"]
         kernels["probability-weighted maps (Sec. 6)"] = {

@@ -66,7 +66,6 @@ int sym_size(const fkv_ctx *c)
 void destroy_cbset(fkv_cbset &s)
 {
     cudaFree(s.cb32);
-    cudaFree(s.cnorm);
     cudaFree(s.cb16);
     cudaFree(s.escale);
     cudaFree(s.escale_h);
@@ -113,9 +112,8 @@ void split3(double v, __half *out)
 }
 
 // Upload one K-or-V half of the codebooks: float32 copy, squared norms and
-// the fp16 operands of the tensor-core RVQ kernels with their TMA map.
-//   D = 128 (k_rvq<128>): hi/lo split of c 2^-e, max |c 2^-e| in [2^14, 2^15).
-//   D = 64 (k_rvq64): hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^3, 2^9)
+// the fp16 operands of the tensor-core RVQ kernels with their TMA map:
+//   hi/lo split of -2 c 2^-e, max |c 2^-e| in [2^3, 2^9)
 //   (in [2^8, 2^9) at a group's first stage; later stages keep the previous
 //   e while they can), and a K x 16 norm operand per (group, stage):
 //   columns 0-2 hold three fp16 parts of ||c 2^-e||^2 2^-10, the rest zero.
@@ -125,12 +123,10 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
     fkv_cbset &s = ctx->cb[kv];
     s.stages = stages;
     const int G = ctx->Ly * (ctx->pooled ? 1 : ctx->H), D = ctx->D, K = ctx->KC;
-    const bool d64 = D == 64;
     const size_t ncode = static_cast<size_t>(G) * stages * K;
-    std::vector<float> cn(ncode);
     std::vector<int> es(static_cast<size_t>(G) * stages);
     std::vector<__half> c16(ncode * 2 * D);
-    std::vector<__half> caug(d64 ? ncode * 16 : 0, __float2half(0.0f));
+    std::vector<__half> caug(ncode * 16, __float2half(0.0f));
     for (int gs = 0; gs < G * stages; ++gs) {
         const float *cb = host + static_cast<size_t>(gs) * K * D;
         float m = 0.0f;
@@ -142,24 +138,22 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         int E = 0;
         if (m > 0.0f)
             frexpf(m, &E);
-        int e = m > 0.0f ? (d64 ? E - 9 : E - 15) : 0;
-        if (d64 && gs % stages != 0) {
-            // 64-dim heads: keep the previous stage's scale while this stage's
-            // max |c| 2^-e stays in [2^3, 2^9), so the kernel rescales the
-            // residual only between stages of very different magnitude
+        int e = m > 0.0f ? E - 9 : 0;
+        if (gs % stages != 0) {
+            // keep the previous stage's scale while this stage's max |c| 2^-e
+            // stays in [2^3, 2^9), so the kernels rescale the residual only
+            // between stages of very different magnitude
             const int prev = es[gs - 1];
             const float q = ldexpf(m, -prev);
             if (q >= 8.0f && q < 512.0f)
                 e = prev;
         }
         es[gs] = e;
-        const float mul = d64 ? -2.0f : 1.0f;
+        const float mul = -2.0f;
         for (int j = 0; j < K; ++j) {
-            double nn = 0.0, ns = 0.0;
+            double ns = 0.0;
             for (int d = 0; d < D; ++d) {
-                const double v = cb[j * D + d];
-                nn += v * v;
-                const double vs = ldexp(v, -e);
+                const double vs = ldexp(static_cast<double>(cb[j * D + d]), -e);
                 ns += vs * vs;
                 const float sv = mul * ldexpf(cb[j * D + d], -e);
                 const __half hi = __float2half_rn(sv);
@@ -167,25 +161,20 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
                 c16[((static_cast<size_t>(gs) * 2 + 0) * K + j) * D + d] = hi;
                 c16[((static_cast<size_t>(gs) * 2 + 1) * K + j) * D + d] = lo;
             }
-            cn[static_cast<size_t>(gs) * K + j] = static_cast<float>(nn);
-            if (d64) {
-                // K rows in the core-matrix layout: 256-row blocks of 8 KB, back to back
-                __half *blk = caug.data() + static_cast<size_t>(gs) * K * 16;
-                __half parts[3];
-                split3(ldexp(ns, -10), parts);
-                for (int k = 0; k < 16; ++k) {
-                    const __half val = k < 3 ? parts[k] : __float2half(0.0f);
-                    blk[core16_offset(j, k) / 2] = val;
-                }
+            // K rows in the core-matrix layout: 256-row blocks of 8 KB, back to back
+            __half *blk = caug.data() + static_cast<size_t>(gs) * K * 16;
+            __half parts[3];
+            split3(ldexp(ns, -10), parts);
+            for (int k = 0; k < 16; ++k) {
+                const __half val = k < 3 ? parts[k] : __float2half(0.0f);
+                blk[core16_offset(j, k) / 2] = val;
             }
         }
     }
     CK(cudaMalloc(&s.cb32, ncode * D * sizeof(float)), "codebook alloc");
-    CK(cudaMalloc(&s.cnorm, ncode * sizeof(float)), "codebook alloc");
     CK(cudaMalloc(&s.cb16, ncode * 2 * D * sizeof(__half)), "codebook alloc");
     CK(cudaMalloc(&s.escale, es.size() * sizeof(int)), "codebook alloc");
     CK(cudaMemcpy(s.cb32, host, ncode * D * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
-    CK(cudaMemcpy(s.cnorm, cn.data(), ncode * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.cb16, c16.data(), c16.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMemcpy(s.escale, es.data(), es.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
     {
@@ -198,10 +187,8 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         CK(cudaMalloc(&s.escale_h, eh.size() * sizeof(int)), "codebook alloc");
         CK(cudaMemcpy(s.escale_h, eh.data(), eh.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
     }
-    if (d64) {
-        CK(cudaMalloc(&s.cbaug, caug.size() * sizeof(__half)), "codebook alloc");
-        CK(cudaMemcpy(s.cbaug, caug.data(), caug.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
-    }
+    CK(cudaMalloc(&s.cbaug, caug.size() * sizeof(__half)), "codebook alloc");
+    CK(cudaMemcpy(s.cbaug, caug.data(), caug.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
     EncodeTiledFn enc = encode_tiled();
     if (!enc)
         return fail(ctx, FKV_ECUDA, "cuTensorMapEncodeTiled unavailable");

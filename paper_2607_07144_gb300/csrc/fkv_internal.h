@@ -20,7 +20,6 @@
 struct fkv_cbset {
     int stages = 0;
     float *cb32 = nullptr;    // [G][S][K][D] float32 (gather, residual update)
-    float *cnorm = nullptr;   // [G][S][K] float32 squared norms
     __half *cb16 = nullptr;   // [G][S][2][K][D] fp16 hi/lo split, scaled by 2^-e
     int *escale = nullptr;    // [G][S] exponent e of the fp16 split
     int *escale_h = nullptr;  // [Ly*H][S] the same per head (its group's), for k_rvq64

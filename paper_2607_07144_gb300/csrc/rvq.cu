@@ -1,24 +1,16 @@
-// Per-head residual-VQ assignment on the 5th-generation tensor cores.
+// Residual-VQ assignment on the 5th-generation tensor cores.
 //
 // Sec. 3 "Setup": each archived head vector is quantised stage by stage to
-// the nearest of 256 codewords of its (layer, head, K/V, stage) codebook, the
-// residual dropping the chosen codeword after each stage.
+// the nearest codeword of its (layer, head or pooled layer, K/V, stage)
+// codebook, the residual dropping the chosen codeword after each stage.
 //
-// One CTA owns a tile of 128 vectors of one codebook group and walks all of
-// its stages:
-//   * the residual tile lives in shared memory as two fp16 operands, hi and
-//     lo (r * 2^-e_row = hi + lo), in the tcgen05 K-major 128-byte-swizzle
-//     layout; e_row is a per-row power of two that keeps the row in range;
-//   * the stage codebook arrives by TMA as fp16 hi/lo (scaled by 2^-e_stage);
-//   * one elected thread issues tcgen05.mma (M = 128, N = 256, K = 16 per
-//     instruction) for hi*hi + hi*lo + lo*hi into a 128 x 256 fp32
-//     accumulator in tensor memory -- the dot products r . c_j to ~2^-21
-//     relative, so the score ||c_j||^2 - 2 r . c_j is certain to well below
-//     the 1e-4 ||r||^2 tie band;
-//   * the four epilogue warps read their 32 lanes of tensor memory
-//     (tcgen05.ld), form the scores, take the running argmin (lowest index on
-//     ties), subtract the chosen float32 codeword and re-split the residual
-//     into the operand tiles for the next stage.
+// Two persistent, warp-specialised kernels, one CTA per SM: k_rvq64 for
+// 64-dimensional heads (256 or 1024 codewords per stage) and k_rvq128 for
+// 128-dimensional heads (256).  Warp 0 streams the stage codebook by TMA, warp
+// 1 issues tcgen05.mma (M = 128, N = 256, K = 16) into fp32 accumulators in
+// tensor memory, and two 4-warp epilogue groups each walk one 128-vector tile
+// through the stages: exact argmin read out of tensor memory with
+// tcgen05.ld.red, then the residual update in the fp16 hi/lo operand tiles.
 #include <type_traits>
 
 #include "fkv_internal.h"
@@ -28,9 +20,7 @@ using namespace fkvd;
 namespace {
 
 constexpr int kRows = 128;          // vectors per tile (MMA M)
-constexpr int kCodes = 256;         // codewords per stage (MMA N)
-constexpr int kThreads = 128;       // 4 warps: one TMEM lane quadrant each
-constexpr uint32_t kTmemCols = 256; // fp32 accumulator columns
+constexpr int kCodes = 256;         // codewords per block (MMA N)
 
 struct RvqArgs {
     const void *x;
@@ -39,7 +29,6 @@ struct RvqArgs {
     int64_t s_layer, s_batch, s_head, s_pos;
     int n_layers, n_heads, S;
     const float *cb32;
-    const float *cnorm;
     const int *escale;
     const int *escale_h;   // [Ly*H][S] escale of each head's codebook group
     const __half *cbaug;
@@ -53,23 +42,6 @@ struct RvqArgs {
     unsigned *status;
 };
 
-template <int D>
-struct Layout {
-    static constexpr int KB = D / 64;                 // 64-element K blocks
-    static constexpr int A_BYTES = KB * kRows * 128;  // one of hi / lo
-    static constexpr int B_BYTES = KB * kCodes * 128;
-    static constexpr int AHI = 0;
-    static constexpr int ALO = A_BYTES;
-    static constexpr int BHI = 2 * A_BYTES;
-    static constexpr int BLO = 2 * A_BYTES + B_BYTES;
-    static constexpr int CN = 2 * A_BYTES + 2 * B_BYTES;   // 256 float
-    static constexpr int BAR = CN + kCodes * 4;            // 2 mbarriers
-    static constexpr int SLOT = BAR + 16;                  // tmem address
-    static constexpr int FLAG = SLOT + 16;                 // abort flag
-    static constexpr int END = FLAG + 16;
-    static constexpr int SMEM = END + 1024;                // + alignment slack
-};
-
 // Byte offset of 16-byte chunk `kk` (0..7) of row `row` inside one
 // 128-row-per-atom K block in the 128-byte swizzle layout.
 __device__ __forceinline__ uint32_t swz(int row, int kk)
@@ -77,96 +49,11 @@ __device__ __forceinline__ uint32_t swz(int row, int kk)
     return static_cast<uint32_t>((row >> 3) * 1024 + (row & 7) * 128 + ((kk ^ (row & 7)) << 4));
 }
 
-// Eight consecutive elements of a head vector as float.
-__device__ __forceinline__ void load8(const uint8_t *p, int dtype, float *o)
-{
-    if (dtype == FKV_F32) {
-        const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
-        const float4 b = __ldg(reinterpret_cast<const float4 *>(p + 16));
-        o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
-        o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
-    } else {
-        const uint4 u = __ldg(reinterpret_cast<const uint4 *>(p));
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            float2 f;
-            if (dtype == FKV_F16)
-                f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
-            else
-                f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
-            o[2 * i] = f.x;
-            o[2 * i + 1] = f.y;
-        }
-    }
-}
-
 // 2^e as a float for e in [-126, 127] (clamped), built from its exponent bits.
 __device__ __forceinline__ float pow2f(int e)
 {
     e = e < -126 ? -126 : (e > 127 ? 127 : e);
     return __int_as_float((e + 127) << 23);
-}
-
-// Power-of-two exponent e such that m * 2^-e lies in [2^14, 2^15) (0 for m = 0).
-__device__ __forceinline__ int row_exp(float m)
-{
-    if (!(m > 0.0f))
-        return 0;
-    int E;
-    frexpf(m, &E);      // m = f * 2^E, f in [0.5, 1)
-    return E - 15;
-}
-
-// Split 8 scaled values into fp16 hi and lo and store them as chunk kk of
-// K block kb of this row's operand tiles.  Returns whether any lo is nonzero.
-__device__ __forceinline__ bool store_split8(uint8_t *ahi, uint8_t *alo, int row, int chunk,
-                                             const float *v)
-{
-    __align__(16) __half hi[8];
-    __align__(16) __half lo[8];
-    bool nz = false;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        hi[i] = __float2half_rn(v[i]);
-        lo[i] = __float2half_rn(v[i] - __half2float(hi[i]));
-        nz |= __half2float(lo[i]) != 0.0f;
-    }
-    const int kb = chunk >> 3, kk = chunk & 7;
-    const uint32_t off = static_cast<uint32_t>(kb * kRows * 128) + swz(row, kk);
-    *reinterpret_cast<uint4 *>(ahi + off) = *reinterpret_cast<const uint4 *>(hi);
-    *reinterpret_cast<uint4 *>(alo + off) = *reinterpret_cast<const uint4 *>(lo);
-    return nz;
-}
-
-// hi + lo of chunk `chunk` of this row, unscaled by 2^e.
-__device__ __forceinline__ void load_split8(const uint8_t *ahi, const uint8_t *alo, int row, int chunk,
-                                            int e, float *o)
-{
-    const int kb = chunk >> 3, kk = chunk & 7;
-    const uint32_t off = static_cast<uint32_t>(kb * kRows * 128) + swz(row, kk);
-    const uint4 h = *reinterpret_cast<const uint4 *>(ahi + off);
-    const uint4 l = *reinterpret_cast<const uint4 *>(alo + off);
-    const __half *hh = reinterpret_cast<const __half *>(&h);
-    const __half *ll = reinterpret_cast<const __half *>(&l);
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-        o[i] = ldexpf(__half2float(hh[i]) + __half2float(ll[i]), e);
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *r)
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 // Bounded wait that also gives up once another thread has flagged an abort.
@@ -187,206 +74,6 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uns
             return false;
         }
     }
-}
-
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
-k_rvq(const __grid_constant__ CUtensorMap tmap, const RvqArgs a)
-{
-    using Lay = Layout<D>;
-    constexpr int CHUNKS = D / 8;
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t *ahi = base + Lay::AHI;
-    uint8_t *alo = base + Lay::ALO;
-    float *cn = reinterpret_cast<float *>(base + Lay::CN);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(base + Lay::FLAG);
-    const uint32_t sbase = smem_u32(base);
-    const uint32_t bar_b = sbase + Lay::BAR;
-    const uint32_t bar_mma = sbase + Lay::BAR + 8;
-
-    const int tid = threadIdx.x;
-    const int warp = tid >> 5;
-    const int g = blockIdx.x / a.tiles_per_group;
-    const int tile = blockIdx.x % a.tiles_per_group;
-    const int l = g / a.n_heads, h = g % a.n_heads;
-    const int cg = a.pooled ? l : g;          // codebook group
-    const int S = a.S;
-    const int64_t nvec = a.batch * a.n_pos;
-    const int64_t v = static_cast<int64_t>(tile) * kRows + tid;
-    const bool valid = v < nvec;
-    const int64_t b = valid ? v / a.n_pos : 0;
-    const int64_t t = valid ? a.t0 + (v - b * a.n_pos) : 0;
-
-    if (tid == 0) {
-        mbar_init(bar_b, 1);
-        mbar_init(bar_mma, 1);
-        *abort_flag = 0;
-        fence_mbar_init();
-        prefetch_tmap(&tmap);
-    }
-    if (warp == 0)
-        tmem_alloc(sbase + Lay::SLOT, kTmemCols);
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(base + Lay::SLOT);
-
-    auto issue_codebook = [&](int s) {
-        const int row0 = (cg * S + s) * 2 * kCodes;
-        mbar_arrive_expect_tx(bar_b, 2u * Lay::KB * kCodes * 128u);
-#pragma unroll
-        for (int kb = 0; kb < Lay::KB; ++kb) {
-            tma_load_2d(sbase + Lay::BHI + kb * kCodes * 128, &tmap, kb * 64, row0, bar_b);
-            tma_load_2d(sbase + Lay::BLO + kb * kCodes * 128, &tmap, kb * 64, row0 + kCodes, bar_b);
-        }
-    };
-    if (tid == 0)
-        issue_codebook(0);
-
-    // Stage-0 residual = the input vector, split into the operand tiles.
-    const uint8_t *xr = nullptr;
-    const int esz = a.dtype == FKV_F32 ? 4 : 2;
-    if (valid)
-        xr = static_cast<const uint8_t *>(a.x) +
-             (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * esz;
-    float rmax = 0.0f;
-    if (valid) {
-        for (int c = 0; c < CHUNKS; ++c) {
-            float f[8];
-            load8(xr + c * 8 * esz, a.dtype, f);
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                rmax = fmaxf(rmax, fabsf(f[i]));
-        }
-    }
-    int ea = row_exp(rmax);
-    bool lo_nz = false;
-    for (int c = 0; c < CHUNKS; ++c) {
-        float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        if (valid) {
-            load8(xr + c * 8 * esz, a.dtype, f);
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                f[i] = ldexpf(f[i], -ea);
-        }
-        lo_nz |= store_split8(ahi, alo, tid, c, f);
-    }
-    const float *cn_g = a.cnorm + static_cast<int64_t>(cg) * S * kCodes;
-    cn[tid] = cn_g[tid];
-    cn[tid + kThreads] = cn_g[tid + kThreads];
-    fence_proxy_async_smem();
-    int lo_any = __syncthreads_or(lo_nz);
-
-    uint8_t idx[8];
-    const float *cb_g = a.cb32 + static_cast<int64_t>(cg) * S * kCodes * D;
-    const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
-
-    for (int s = 0; s < S; ++s) {
-        // --- MMA: acc[row][j] = sum_k (hi*hi + hi*lo + lo*hi), all K blocks
-        if (tid == 0) {
-            if (wait_or_abort(bar_b, s & 1, a.status, abort_flag)) {
-                tc_fence_after();
-                uint32_t accum = 0;
-#pragma unroll
-                for (int kb = 0; kb < Lay::KB; ++kb) {
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const uint32_t ka = kb * kRows * 128 + k * 32;
-                        const uint32_t kbb = kb * kCodes * 128 + k * 32;
-                        const uint64_t dah = sdesc_sw128(sbase + Lay::AHI + ka);
-                        const uint64_t dal = sdesc_sw128(sbase + Lay::ALO + ka);
-                        const uint64_t dbh = sdesc_sw128(sbase + Lay::BHI + kbb);
-                        const uint64_t dbl = sdesc_sw128(sbase + Lay::BLO + kbb);
-                        umma_f16(tmem, dah, dbh, idesc, accum);
-                        accum = 1;
-                        umma_f16(tmem, dah, dbl, idesc, 1);
-                        if (lo_any)
-                            umma_f16(tmem, dal, dbh, idesc, 1);
-                    }
-                }
-                umma_commit(bar_mma);
-            }
-        }
-        const bool ok = wait_or_abort(bar_mma, s & 1, a.status, abort_flag);
-        if (!__syncthreads_and(ok))
-            break;
-        tc_fence_after();
-
-        // --- epilogue: scores ||c||^2 - 2 r.c, argmin over this row's 256 columns
-        const int eb = a.escale[cg * S + s];
-        const float sc = -ldexpf(1.0f, ea + eb + 1);
-        float best = INFINITY;
-        int bi = 0;
-        const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-#pragma unroll 1
-        for (int ch = 0; ch < kCodes / 32; ++ch) {
-            uint32_t r[32];
-            tmem_ld32(trow + ch * 32, r);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                const float score = fmaf(sc, __uint_as_float(r[j]), cn[ch * 32 + j]);
-                if (score < best) {
-                    best = score;
-                    bi = ch * 32 + j;
-                }
-            }
-        }
-        idx[s] = static_cast<uint8_t>(bi);
-        tc_fence_before();
-        __syncthreads();   // TMEM read, operand tiles and codebook buffers free
-
-        if (s + 1 < S) {
-            if (tid == 0)
-                issue_codebook(s + 1);
-            // residual update: r <- r - C_s[bi], re-split with a fresh row exponent
-            const float *crow = cb_g + (static_cast<int64_t>(s) * kCodes + bi) * D;
-            float m2 = 0.0f;
-            if (valid) {
-                for (int c = 0; c < CHUNKS; ++c) {
-                    float f[8];
-                    load_split8(ahi, alo, tid, c, ea, f);
-                    const float4 c0 = __ldg(reinterpret_cast<const float4 *>(crow + c * 8));
-                    const float4 c1 = __ldg(reinterpret_cast<const float4 *>(crow + c * 8 + 4));
-                    const float cc[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-#pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        m2 = fmaxf(m2, fabsf(f[i] - cc[i]));
-                }
-            }
-            const int ea2 = row_exp(m2);
-            lo_nz = false;
-            for (int c = 0; c < CHUNKS; ++c) {
-                float f[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                if (valid) {
-                    load_split8(ahi, alo, tid, c, ea, f);
-                    const float4 c0 = __ldg(reinterpret_cast<const float4 *>(crow + c * 8));
-                    const float4 c1 = __ldg(reinterpret_cast<const float4 *>(crow + c * 8 + 4));
-                    const float cc[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-#pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        f[i] = ldexpf(f[i] - cc[i], -ea2);
-                }
-                lo_nz |= store_split8(ahi, alo, tid, c, f);
-            }
-            ea = ea2;
-            cn[tid] = cn_g[(s + 1) * kCodes + tid];
-            cn[tid + kThreads] = cn_g[(s + 1) * kCodes + tid + kThreads];
-            fence_proxy_async_smem();
-            lo_any = __syncthreads_or(lo_nz);
-        }
-    }
-
-    if (valid && !*abort_flag) {
-        uint8_t *dst = static_cast<uint8_t *>(a.sym) + (b * a.n_layers + l) * a.stream_stride +
-                       (a.rec0 + (t - a.t0)) * a.R + a.kv_off + h * S;
-        for (int s = 0; s < S; ++s)
-            dst[s] = idx[s];
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0)
-        tmem_dealloc(tmem, kTmemCols);
 }
 
 // ===================================================================
@@ -1064,6 +751,347 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
     }
 }
 
+
+// ===================================================================
+// Persistent kernel for 128-dimensional heads.
+//
+// The k_rvq64 scheme (two tile slots, split-fp16 operands of -2 c', a per-row
+// shift, the residual in the operand tiles, exact ld.red argmin) with the
+// head dimension in two 64-wide K blocks.  A slot's hi and lo operand tiles
+// take 64 KB, so the stage codebook does not fit twice: it streams through
+// one buffer a K block at a time (hi and lo of 256 codewords x 64 dimensions,
+// 64 KB, with the 256 x 16 norm operand beside the first block).  Per stage
+// the MMA warp runs block 0 for both slots (the norm MMA plus 12), releases
+// the buffer with a commit once those MMAs are done, then block 1 for both
+// slots, committing each slot's accumulator; so the buffer is the MMAs' alone
+// and the epilogue reads the chosen codeword's hi/lo rows from their global
+// (L2-resident) copy.  One slot's epilogue overlaps the other slot's MMAs and
+// the next block's load.
+namespace v3 {
+constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups
+constexpr int kThreads = kWarps * 32;
+constexpr int A_KB = kRows * 128;            // 16 KB: 128 rows x 64 fp16 (128-byte swizzle)
+constexpr int A_HALF = 2 * A_KB;             // hi (or lo): both K blocks
+constexpr int A_SLOT = 2 * A_HALF;           // 64 KB
+constexpr int A_AUG = kRows * 32;            // 4 KB per slot
+constexpr int B_TILE = kCodes * 128;         // 32 KB: 256 codewords x 64 fp16
+constexpr int B_BUF = 2 * B_TILE;            // hi + lo of one K block
+constexpr int B_AUG = kCodes * 32;           // 8 KB
+constexpr int OFF_A = 0;
+constexpr int OFF_AAUG = 2 * A_SLOT;         // 128 KB
+constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 136 KB: 1024-aligned
+constexpr int OFF_BAUG = OFF_B + B_BUF;
+constexpr int OFF_BAR = OFF_BAUG + B_AUG;    // b_full, b_empty, a_ready[2], acc_full[2], drain
+constexpr int OFF_SLOT = OFF_BAR + 64;
+constexpr int OFF_LO = OFF_SLOT + 16;
+constexpr int OFF_ABORT = OFF_LO + 16;
+constexpr int END = OFF_ABORT + 16;
+constexpr int SMEM = END + 1024;
+static_assert(SMEM <= 232448, "shared memory");
+}  // namespace v3
+
+template <int ESZ>
+__global__ void __launch_bounds__(v3::kThreads, 1)
+k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per_group, int n_pairs)
+{
+    using namespace v3;
+    constexpr int D = 128;
+    constexpr int XC = D * ESZ / 16;             // 16-byte chunks per input row
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t sbase = smem_u32(base);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(base + OFF_ABORT);
+    volatile int *lo_stamp = reinterpret_cast<volatile int *>(base + OFF_LO);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    // barrier i: 0 b_full; 1 b_empty; 2,3 a_ready; 4,5 acc_full; 6 drain (MMA completion at exit)
+    auto bar = [&](int i) { return sbase + OFF_BAR + 8u * i; };
+    if (tid == 0) {
+        mbar_init(bar(0), 1);
+        mbar_init(bar(1), 1);
+        mbar_init(bar(2), 128);
+        mbar_init(bar(3), 128);
+        mbar_init(bar(4), 1);
+        mbar_init(bar(5), 1);
+        mbar_init(bar(6), 1);
+        lo_stamp[0] = 0;
+        lo_stamp[1] = 0;
+        *abort_flag = 0;
+        fence_mbar_init();
+        prefetch_tmap(&tmap);
+    }
+    if (warp == 1)
+        tmem_alloc(sbase + OFF_SLOT, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(base + OFF_SLOT);
+    const int S = a.S;
+    const int64_t nvec = a.batch * a.n_pos;
+    const int tiles = a.tiles_per_group;
+    auto cgroup = [&](int g) { return a.pooled ? g / a.n_heads : g; };
+
+    if (warp == 0) {
+        // ---------------------------------------------------- TMA producer
+        if (lane == 0) {
+            int it = 0, last = -1;
+            bool ok = true;
+            for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
+                const int cg = cgroup(p / pairs_per_group);
+                for (int s = 0; s < S && ok; ++s) {
+                    for (int kb = 0; kb < 2; ++kb, ++it) {
+                        if (!wait_or_abort(bar(1), (it & 1) ^ 1, a.status, abort_flag)) {
+                            ok = false;
+                            break;
+                        }
+                        const int row0 = (cg * S + s) * 2 * kCodes;
+                        const uint32_t bb = sbase + OFF_B;
+                        mbar_arrive_expect_tx(bar(0), B_BUF + (kb == 0 ? B_AUG : 0));
+                        tma_load_2d(bb, &tmap, kb * 64, row0, bar(0));
+                        tma_load_2d(bb + B_TILE, &tmap, kb * 64, row0 + kCodes, bar(0));
+                        if (kb == 0)
+                            bulk_load(sbase + OFF_BAUG, a.cbaug + static_cast<int64_t>(cg * S + s) * kCodes * 16,
+                                      B_AUG, bar(0));
+                        last = it;
+                    }
+                }
+            }
+            // no copy may still be landing in shared memory when the CTA exits
+            if (last >= 0)
+                mbar_wait(bar(0), last & 1, a.status);
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
+            int it = 0;
+            uint32_t aph[2] = {0, 0};
+            int pc = 0;
+            bool ok = true;
+            for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
+                ++pc;
+                for (int s = 0; s < S && ok; ++s) {
+                    for (int kb = 0; kb < 2 && ok; ++kb, ++it) {
+                        ok = wait_or_abort(bar(0), it & 1, a.status, abort_flag);
+                        if (!ok)
+                            break;
+                        const uint32_t bb = sbase + OFF_B;
+                        for (int k = 0; k < 2; ++k) {
+                            if (kb == 0) {
+                                ok = wait_or_abort(bar(2 + k), aph[k], a.status, abort_flag);
+                                if (!ok)
+                                    break;
+                                aph[k] ^= 1;
+                            }
+                            tc_fence_after();
+                            const bool lo = s > 0 || lo_stamp[k] == pc;
+                            const uint32_t ab = sbase + OFF_A + k * A_SLOT + kb * A_KB;
+                            const uint32_t acc = tmem + k * 256;
+                            if (kb == 0)   // codeword norms first (K = 16, no swizzle)
+                                umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(sbase + OFF_BAUG),
+                                         idesc, 0);
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk) {
+                                const uint64_t dah = sdesc_sw128(ab + kk * 32);
+                                const uint64_t dal = sdesc_sw128(ab + A_HALF + kk * 32);
+                                const uint64_t dbh = sdesc_sw128(bb + kk * 32);
+                                const uint64_t dbl = sdesc_sw128(bb + B_TILE + kk * 32);
+                                umma_f16(acc, dah, dbh, idesc, 1);
+                                umma_f16(acc, dah, dbl, idesc, 1);
+                                if (lo)
+                                    umma_f16(acc, dal, dbh, idesc, 1);
+                            }
+                            if (kb == 1)
+                                umma_commit(bar(4 + k));
+                        }
+                        if (ok)
+                            umma_commit(bar(1));          // the buffer is free once these MMAs are done
+                    }
+                }
+            }
+            // every MMA has completed before tensor memory is released
+            umma_commit(bar(6));
+            mbar_wait(bar(6), 0, a.status);
+        }
+    } else {
+        // ---------------------------------------------------- epilogue groups
+        const int k = (warp - 2) >> 2;           // tile slot 0 or 1
+        const int quad = warp & 3;                // TMEM lane quadrant of this warp
+        const int row = quad * 32 + lane;
+        const uint32_t trow = tmem + k * 256 + (static_cast<uint32_t>(quad * 32) << 16);
+        uint8_t *ahi = base + OFF_A + k * A_SLOT;
+        uint8_t *alo = ahi + A_HALF;
+        uint8_t *aaug = base + OFF_AAUG + k * A_AUG;
+        auto row_src = [&](int p, bool *in) -> const uint4 * {
+            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
+            const int tile = 2 * q + k;
+            const int64_t v = static_cast<int64_t>(tile) * kRows + row;
+            *in = tile < tiles && v < nvec;
+            if (!*in)
+                return nullptr;
+            const int l = g / a.n_heads, h = g - l * a.n_heads;
+            const int64_t b = v / a.n_pos;
+            const int64_t t = a.t0 + (v - b * a.n_pos);
+            return reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(a.x) +
+                                                   (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * ESZ);
+        };
+        int it = 0;
+        uint32_t fph = 0;
+        int pc = 0;
+        for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
+            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
+            const int l = g / a.n_heads, h = g - l * a.n_heads;
+            const int tile = 2 * q + k;
+            const int64_t v = static_cast<int64_t>(tile) * kRows + row;
+            const bool valid = tile < tiles && v < nvec;
+            bool in;
+            const uint4 *src = row_src(p, &in);
+            // the row's operand t = x 2^-(e + er), er >= 0 keeping |t| below 2^12
+            int e = __ldg(&a.escale_h[g * S]);
+            int er;
+            ++pc;
+            {
+                const float se = pow2f(-e);
+                float mx = 0.0f;
+#pragma unroll 4
+                for (int c = 0; c < 16; ++c) {
+                    float f[8];
+                    uint4 xr[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+                    if (in) {
+                        xr[0] = __ldg(src + c * (ESZ / 2));
+                        if (ESZ == 4)
+                            xr[1] = __ldg(src + c * 2 + 1);
+                    }
+                    unpack8<ESZ>(xr, a.dtype, 0, f);
+#pragma unroll
+                    for (int i = 0; i < 8; i += 2)
+                        mx = max3f(mx, fabsf(f[i] * se), fabsf(f[i + 1] * se));
+                }
+                er = row_shift(mx);
+                const float sr = pow2f(-er);
+                uint32_t nz = 0;
+#pragma unroll 4
+                for (int c = 0; c < 16; ++c) {
+                    float f[8];
+                    uint4 xr[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+                    if (in) {
+                        xr[0] = __ldg(src + c * (ESZ / 2));
+                        if (ESZ == 4)
+                            xr[1] = __ldg(src + c * 2 + 1);
+                    }
+                    unpack8<ESZ>(xr, a.dtype, 0, f);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        f[i] = f[i] * se * sr;
+                    nz |= store_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7, f);
+                }
+                write_aug_row(aaug, row, er);
+                if (nz)
+                    lo_stamp[k] = pc;
+            }
+            fence_proxy_async_smem();
+            mbar_arrive(bar(2 + k));
+            if (p + static_cast<int>(gridDim.x) < n_pairs) {
+                // the next pair's input row into L2 while this pair runs
+                bool nin;
+                const uint4 *nsrc = row_src(p + gridDim.x, &nin);
+                if (nin)
+                    for (int c = 0; c < XC; c += 8)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(nsrc + c));
+            }
+            uint8_t idx[8];
+            bool ok = true;
+            for (int s = 0; s < S; ++s, ++it) {
+                const int e_next = s + 1 < S ? __ldg(&a.escale_h[g * S + s + 1]) : e;
+                ok = wait_or_abort(bar(4 + k), fph, a.status, abort_flag);
+                // the tensor-memory loads below are warp-collective: the warp
+                // goes on, or leaves, as one
+                ok = __all_sync(0xFFFFFFFFu, ok);
+                if (!ok)
+                    break;
+                fph ^= 1;
+                tc_fence_after();
+                __syncwarp();
+                bool amb;
+                float vu;
+                int bidx = argmin_row4(trow, &amb, &vu);
+                if (__any_sync(0xFFFFFFFFu, amb)) {   // warp-collective loads: every lane takes part
+                    const int jj = exact_argmin_tmem(trow);
+                    if (amb)
+                        bidx = jj;
+                }
+                tc_fence_before();
+                idx[s] = static_cast<uint8_t>(bidx);
+                if (s + 1 < S) {
+                    // t <- t + (hi + lo) 2^(-1-er) from the codeword's global hi/lo rows
+                    const float f = pow2f(-1 - er);
+                    const uint4 *gh = reinterpret_cast<const uint4 *>(
+                        a.cb16 + ((static_cast<int64_t>(cgroup(g) * S + s) * 2) * kCodes + bidx) * D);
+                    constexpr int LO = kCodes * D / 8;   // uint4 from a hi row to its lo row
+                    if (e_next == e) {
+#pragma unroll 4
+                        for (int c = 0; c < 16; ++c) {
+                            float t[8];
+                            uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
+                            load_chunk(hp, lp, row, c & 7, t);
+                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+                            store_chunk(hp, lp, row, c & 7, t);
+                        }
+                    } else {
+                        float mx = 0.0f;
+#pragma unroll 1
+                        for (int c = 0; c < 16; ++c) {
+                            float t[8];
+                            load_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7, t);
+                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; i += 2)
+                                mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
+                        }
+                        int E = 0;
+                        if (mx > 0.0f)
+                            frexpf(mx, &E);
+                        const int tot = E + er + e - e_next;
+                        const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
+                        const float gsc = pow2f(er + e - e_next - er2);
+#pragma unroll 1
+                        for (int c = 0; c < 16; ++c) {
+                            float t[8];
+                            uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
+                            load_chunk(hp, lp, row, c & 7, t);
+                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                t[i] *= gsc;
+                            store_chunk(hp, lp, row, c & 7, t);
+                        }
+                        er = er2;
+                        write_aug_row(aaug, row, er);
+                    }
+                    e = e_next;
+                    fence_proxy_async_smem();
+                    mbar_arrive(bar(2 + k));
+                }
+            }
+            if (!ok)
+                break;
+            if (valid) {
+                const int64_t b = v / a.n_pos;
+                const int64_t t = a.t0 + (v - b * a.n_pos);
+                uint8_t *dst = static_cast<uint8_t *>(a.sym) + (b * a.n_layers + l) * a.stream_stride +
+                               (a.rec0 + (t - a.t0)) * a.R + a.kv_off + h * S;
+                for (int s = 0; s < S; ++s)
+                    dst[s] = idx[s];
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
 }  // namespace
 
 template <int ESZ, int NB>
@@ -1095,7 +1123,6 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
     a.n_heads = c->H;
     a.S = cb.stages;
     a.cb32 = cb.cb32;
-    a.cnorm = cb.cnorm;
     a.escale = cb.escale;
     a.escale_h = cb.escale_h;
     a.cbaug = cb.cbaug;
@@ -1133,15 +1160,28 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
         return x->dtype == FKV_F32 ? launch_rvq64<4, 1>(cb.tmap, a, pp, np, grid, st)
                                    : launch_rvq64<2, 1>(cb.tmap, a, pp, np, grid, st);
     } else {
-        static bool attr = false;
-        if (!attr) {
-            cudaError_t e = cudaFuncSetAttribute(k_rvq<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 Layout<128>::SMEM);
+        // 128-dimensional heads: 256 codewords per stage
+        const int64_t ppg = (tiles + 1) / 2;
+        const int64_t n_pairs = ppg * c->Ly * c->H;
+        if (n_pairs > 0x7FFFFFFF)
+            return cudaErrorInvalidConfiguration;
+        int sms = 0;
+        cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+        if (e != cudaSuccess)
+            return e;
+        const unsigned grid = static_cast<unsigned>(n_pairs < sms ? n_pairs : sms);
+        const int pp = static_cast<int>(ppg), np = static_cast<int>(n_pairs);
+        if (x->dtype == FKV_F32) {
+            e = cudaFuncSetAttribute(k_rvq128<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, v3::SMEM);
             if (e != cudaSuccess)
                 return e;
-            attr = true;
+            k_rvq128<4><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, pp, np);
+        } else {
+            e = cudaFuncSetAttribute(k_rvq128<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, v3::SMEM);
+            if (e != cudaSuccess)
+                return e;
+            k_rvq128<2><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, pp, np);
         }
-        k_rvq<128><<<static_cast<unsigned>(blocks), kThreads, Layout<128>::SMEM, st>>>(cb.tmap, a);
     }
     return cudaGetLastError();
 }
