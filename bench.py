@@ -375,7 +375,8 @@ def run_gpu(args, rank, world, local_rank):
     # path as the step above, on 128-dimensional heads
     llama = None
     if not args.no_llama:
-        c3 = synth.CFG3
+        c3 = synth.CFG3 if args.llama_seq == synth.CFG3.seq else synth.small_config(
+            synth.CFG3, synth.CFG3.cfg_id, n_layers=synth.CFG3.n_layers, batch=synth.CFG3.batch, seq=args.llama_seq)
         lctx = fkv.Context(256, codebooks=(synth.codebooks(c3, 0), synth.codebooks(c3, 1)))
         K3 = synth.gpu_kv_cache(c3, 0, device=dev)
         V3 = synth.gpu_kv_cache(c3, 1, device=dev)
@@ -573,6 +574,8 @@ def main():
     ap.add_argument("--no-lossy", action="store_true")
     ap.add_argument("--no-weighted", action="store_true")
     ap.add_argument("--no-llama", action="store_true")
+    ap.add_argument("--llama-seq", type=int, default=synth.CFG3.seq,
+                    help="positions of the Llama-shaped cache (a shorter one for profiling captures)")
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()
@@ -668,8 +671,8 @@ def main():
         sym3 = lx["records"] * lx["R"]
         dec3 = sym3 + lx["spans"] * 16 + lx["out_bytes"]
         kernels["llama3-8b-shaped archive (config 3)"] = {
-            "workload": "32 layers x batch 4 x 8 KV heads x 32768 tok x 128 dims, bf16; 4+32 exact window; K 4 / V 2 "
-                        "RVQ stages x 256; N=256, r=r_256, L=6",
+            "workload": "32 layers x batch 4 x 8 KV heads x %d tok x 128 dims, bf16; 4+32 exact window; K 4 / V 2 "
+                        "RVQ stages x 256; N=256, r=r_256, L=6" % args.llama_seq,
             "records_per_s": lx["records"] / (sum(ph3) * 1e-3), "step_ms": sum(ph3),
             "rvq_ms": rvq3, "rvq_tflops": tf3, "rvq_frac": tf3 / peaks["bf16_tflops"],
             "rvq_kernel": "k_rvq128 (persistent, two tile slots, codebook streamed in 64-dim K blocks)",
