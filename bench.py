@@ -59,7 +59,7 @@ def load_peaks():
 # to None whenever that kernel changes until it is captured again.
 RVQ_DRAM_BYTES_PER_LAUNCH = 184304640
 
-# FP64 add/mul issue rate measured on this machine's GB300 (1.6 per clock per SM,
+# FP64 add/mul issue rate measured on a GB300 (1.6 per clock per SM,
 # 504 Gop/s at the clock of that run); the span encoder is bound by it.
 FP64_OPS_PER_CLK_SM = 1.6
 
@@ -310,6 +310,41 @@ def run_gpu(args, rank, world, local_rank):
                   "workload": "4 streams x 2^28 uniform symbols, N=256, span 6, one 6-symbol query"}
         del s_pts, sctx
 
+    # The span codec on the symbol-stress workload: per alphabet N in
+    # {3, 4, 16, 256} (spans 44, 44, 16, 6), four streams of 2^28 seeded
+    # uniform symbols encoded to points, decoded whole, and 2^20 seeded random
+    # positions per stream read back; every result checked against the input
+    codec = None
+    if not args.no_codec:
+        codec = {}
+        n = 1 << 28
+        for N in (3, 4, 16, 256):
+            cc = fkv.Context(N)
+            c_sym = synth.gpu_symbols(N, "uniform", 4, n, device=dev)
+            c_pts = cc.span_encode(c_sym)
+            c_dec = torch.empty_like(c_sym)
+            req = torch.cat([torch.stack([torch.full((1 << 20,), s_, dtype=torch.int64, device=dev),
+                                          synth.gpu_positions(n, 1 << 20, s_, device=dev)], 1) for s_ in range(4)])
+            c_out = torch.empty(req.shape[0], dtype=c_sym.dtype, device=dev)
+            ops = (lambda: cc.span_encode(c_sym, c_pts), lambda: cc.span_decode(c_pts, n, c_dec),
+                   lambda: cc.read(c_pts, n, req, c_out))
+            for op in ops:
+                op()
+            reps = 3
+            ms_ = []
+            for op in ops:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for _ in range(reps):
+                    op()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                ms_.append(e0.elapsed_time(e1) / reps)
+            exact = bool(torch.equal(c_dec, c_sym)) and bool(torch.equal(c_out, c_sym[req[:, 0], req[:, 1]]))
+            codec[N] = {"L": cc.L, "spans": c_pts.shape[1], "encode_ms": ms_[0], "decode_ms": ms_[1],
+                        "read_ms": ms_[2], "reads": req.shape[0], "exact": exact, "ok": cc.sync_status() == 0}
+            del c_sym, c_pts, c_dec, req, c_out, cc
+
     # Sec. 4 lossy archive of this step's streams: spans older than the last
     # 64 records truncated to 24 bits per coordinate (6 B instead of 16 B per
     # span), the recent ones exact; truncation and the full lossy decode
@@ -464,7 +499,7 @@ def run_gpu(args, rank, world, local_rank):
 
     units = ns * n_rec
     return dict(cfg=cfg, ms=ms, phase=dict(zip(names, phase.tolist())), clocks=clk, ok=ok, e2e=e2e, units=units,
-                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, k1024=k1024,
+                R=R, ns=ns, P=P, n_rec=n_rec, spans=ctx.n_spans(n_rec * R), L=ctx.L, suffix=suffix, codec=codec, k1024=k1024,
                 lossy=lossy, weighted=weighted, llama=llama)
 
 
@@ -572,6 +607,7 @@ def main():
     ap.add_argument("--no-suffix", action="store_true")
     ap.add_argument("--no-k1024", action="store_true")
     ap.add_argument("--no-lossy", action="store_true")
+    ap.add_argument("--no-codec", action="store_true")
     ap.add_argument("--no-weighted", action="store_true")
     ap.add_argument("--no-llama", action="store_true")
     ap.add_argument("--llama-seq", type=int, default=synth.CFG3.seq,
@@ -634,6 +670,25 @@ def main():
         kernels["suffix_search (Sec. 5)"] = {"bound": "hbm", "ms": sx["ms"], "achieved_gbs": gbs,
                                              "frac": gbs / peaks["hbm_gbs"], "matches": sx["matches"],
                                              "candidates": sx["candidates"], "workload": sx["workload"]}
+    if res["codec"]:
+        fp64_peak = FP64_OPS_PER_CLK_SM * 152 * (res["clocks"].get("sm_mhz") or 1900.0) * 1e6
+        per_n = {}
+        for N, cx in res["codec"].items():
+            syms = 4 * (1 << 28)
+            nbytes = syms + 4 * cx["spans"] * 16          # 1 B per symbol + one 16 B point per span
+            per_n["N=%d" % N] = {
+                "L": cx["L"],
+                "encode_ms": cx["encode_ms"], "encode_symbols_per_s": syms / (cx["encode_ms"] * 1e-3),
+                "encode_frac_hbm": nbytes / (cx["encode_ms"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                "encode_frac_fp64": syms * 6 / (cx["encode_ms"] * 1e-3) / fp64_peak,
+                "decode_ms": cx["decode_ms"], "decode_symbols_per_s": syms / (cx["decode_ms"] * 1e-3),
+                "decode_frac_hbm": nbytes / (cx["decode_ms"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                "read_ms": cx["read_ms"], "reads_per_s": cx["reads"] / (cx["read_ms"] * 1e-3),
+                "exact": cx["exact"], "status_ok": cx["ok"]}
+        kernels["span codec, symbol stress"] = {
+            "workload": "4 streams x 2^28 seeded uniform symbols per N; full encode, full decode, 2^20 seeded "
+                        "random reads per stream; all decoded and read symbols checked equal to the input",
+            "encode_bound": "fp64", "decode_bound": "integer ALU", "read_bound": "latency", "per_N": per_n}
     if res["k1024"]:
         kx = res["k1024"]
         rvq_ms = kx["rvq_k"] + kx["rvq_v"]
