@@ -59,9 +59,10 @@ def load_peaks():
 # to None whenever that kernel changes until it is captured again.
 RVQ_DRAM_BYTES_PER_LAUNCH = 184304640
 
-# FP64 add/mul issue rate measured on a GB300 (1.6 per clock per SM,
-# 504 Gop/s at the clock of that run); the span encoder is bound by it.
-FP64_OPS_PER_CLK_SM = 1.6
+# FP64 add/mul peak: GB300's nominal 1.25 TFLOP/s of FP64 FMA is 625 G add or
+# mul instructions per second at the 2070 MHz boost clock, 1.99 per clock per SM
+# (a dependent-chain probe reached 1.6, the span encoder 1.67)
+FP64_OPS_PER_CLK_SM = 1.25e12 / 2 / (152 * 2070e6)
 
 
 class ClockSampler:
