@@ -22,6 +22,8 @@
 //     neighbouring sectors are decided by the exact sign of Q . (V(a) - V(b)).
 #pragma once
 
+#include <climits>
+
 #include "fkv_internal.h"
 
 namespace fkvdec {
@@ -77,6 +79,23 @@ static __device__ __noinline__ int classify_exact_all(const Tables &t, long long
     return best;
 }
 
+// fp32 image (qx, qy) of the direction of (X, Y): both scaled by one power of
+// two that puts the larger magnitude's top bit at bit 62, then their high
+// 32-bit words converted.  Relative to the larger magnitude the image is off
+// by at most 2^-30 (the dropped low word) plus one fp32 rounding, like a
+// direct conversion; only integer ops and 32-bit conversions are used,
+// because 64-bit integer conversions issue at the FP64 rate on this GPU.
+__device__ __forceinline__ void direction(long long X, long long Y, float &qx, float &qy)
+{
+    const unsigned long long ax = X < 0 ? 0ull - static_cast<unsigned long long>(X) : static_cast<unsigned long long>(X);
+    const unsigned long long ay = Y < 0 ? 0ull - static_cast<unsigned long long>(Y) : static_cast<unsigned long long>(Y);
+    const int sh = max(__clzll(static_cast<long long>(ax | ay)) - 1, 0);
+    const unsigned long long xs = static_cast<unsigned long long>(X) << sh;
+    const unsigned long long ys = static_cast<unsigned long long>(Y) << sh;
+    qx = __int2float_rn(static_cast<int>(static_cast<unsigned>(xs >> 32)));
+    qy = __int2float_rn(static_cast<int>(static_cast<unsigned>(ys >> 32)));
+}
+
 __device__ __forceinline__ int classify(const Tables &t, long long X, long long Y)
 {
     const int N = t.N;
@@ -86,7 +105,8 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
             return X >= 0 ? 0 : 2;
         return Y >= 0 ? 1 : 3;
     }
-    const float qx = __ll2float_rn(X), qy = __ll2float_rn(Y);
+    float qx, qy;
+    direction(X, Y, qx, qy);
     if (N <= 8) {
         float b1 = -INFINITY, b2 = -INFINITY;
         int bi = 0;
@@ -127,9 +147,35 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
     return c0 < c1 ? c0 : c1;
 }
 
+// round(v * 2^62) to nearest, ties to even, saturated to int64 (NaN gives
+// INT64_MIN), from the binary64 fields with integer ops: v = m 2^(e - 1075),
+// so v 2^62 = m 2^(e - 1013), a left shift or a rounded right shift of m.
 __device__ __forceinline__ long long to_q62(double v)
 {
-    return __double2ll_rn(v * 4611686018427387904.0);   // v * 2^62, exact scaling
+    const unsigned long long b = static_cast<unsigned long long>(__double_as_longlong(v));
+    const int e = static_cast<int>((b >> 52) & 0x7FF);
+    const unsigned long long frac = b & 0xFFFFFFFFFFFFFull;
+    const bool neg = (b >> 63) != 0;
+    if (e >= 1024) {                           // |v| >= 2, infinity or NaN
+        if (e == 2047 && frac)
+            return LLONG_MIN;
+        return neg ? LLONG_MIN : LLONG_MAX;
+    }
+    if (e == 0)                                // zero or subnormal: |v 2^62| < 2^-960
+        return 0;
+    const unsigned long long m = frac | (1ull << 52);
+    const int s = e - 1013;
+    unsigned long long mag;
+    if (s >= 0) {
+        mag = m << s;                          // s <= 10: below 2^63
+    } else if (s > -54) {
+        const int k = -s;
+        const unsigned long long q = m >> k, rem = m & ((1ull << k) - 1), half = 1ull << (k - 1);
+        mag = q + ((rem > half || (rem == half && (q & 1))) ? 1 : 0);
+    } else {
+        mag = 0;                               // below half a unit
+    }
+    return neg ? -static_cast<long long>(mag) : static_cast<long long>(mag);
 }
 
 // Decode `steps` symbols backward from Q (the span's stored point in Q1.62):

@@ -7,15 +7,17 @@
 // block holds the float32 codebooks of one group and one slice of the head
 // dimension (all stages) in shared memory while it works on that slice, so
 // HBM sees only the indices in and the rebuilt K/V out.  Codebooks of 256
-// codewords take uint8 indices, of 1024 codewords uint16.  A thread rebuilds four dimensions (one
-// 16-byte granule of a slice row) of a vector.  Sums run in float32, stage
+// codewords take uint8 indices, of 1024 codewords uint16.  A thread rebuilds eight dimensions
+// (two 16-byte granules of a slice row) of a vector, four in 16-float slices.  Sums run in float32, stage
 // order, then round to nearest-even into the cache dtype.
 //
 // Shared-memory reads are conflict-free for any indices: a slice row spans a
-// multiple of 128 bytes, so its granule g lies in bank group g % 8, and the
-// eight threads of a quarter warp read the eight consecutive granules of one
-// row.  A 16-float slice (two rows per bank line, for more than four stages)
-// permutes its granules by an XOR of the row instead.
+// multiple of 128 bytes, so its granule g lies in bank group g % 8.  A thread
+// owns granules 2q and 2q + 1; lanes 0-3 of a quarter warp read the even one
+// first and lanes 4-7 the odd one, so each read covers the eight bank groups
+// once (32-float rows: two vectors per quarter warp; 64-float rows: one).  A
+// 16-float slice (two rows per bank line, for more than four stages) gives a
+// thread one granule and permutes granules by an XOR of the row instead.
 #include <type_traits>
 
 #include "decode_core.cuh"
@@ -23,7 +25,6 @@
 namespace {
 
 constexpr int kThreads = 1024;
-constexpr int kDT = 4;                   // dimensions a thread rebuilds
 
 struct GatherArgs {
     const void *sym;       // the S indices of (b, l, h, rec) at sym + b ib + l il + h ih + rec ir + ioff (symbols)
@@ -58,6 +59,20 @@ __device__ __forceinline__ uint32_t pack2(int dtype, float a, float b)
     }
     const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// Eight consecutive elements at `elem` (16-byte aligned): lo then hi.
+__device__ __forceinline__ void store8(void *out, int dtype, int64_t elem, float4 lo, float4 hi)
+{
+    if (dtype == FKV_F32) {
+        float4 *p = reinterpret_cast<float4 *>(static_cast<float *>(out) + elem);
+        p[0] = lo;
+        p[1] = hi;
+        return;
+    }
+    *reinterpret_cast<uint4 *>(static_cast<uint16_t *>(out) + elem) =
+        make_uint4(pack2(dtype, lo.x, lo.y), pack2(dtype, lo.z, lo.w), pack2(dtype, hi.x, hi.y),
+                   pack2(dtype, hi.z, hi.w));
 }
 
 // Four consecutive elements at `elem` (aligned to their size).
@@ -122,9 +137,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
     const int D = a.D, parts = a.parts;
     constexpr int q4 = Dp / 4;               // 16-byte granules per slice row
     constexpr bool xor_rows = Dp < 32;       // 16-float rows: XOR-permuted granules
+    constexpr int kDT = Dp >= 32 ? 8 : 4;    // dimensions a thread rebuilds
     constexpr int tpv = Dp / kDT;            // threads per vector
     constexpr int vpi = kThreads / tpv;      // vectors per pass
-    const int dq = threadIdx.x % tpv;        // this thread's granule of the slice row
+    const int dq = threadIdx.x % tpv;        // this thread's granule (pair) of the slice row
+    // Two granules per thread: the upper four lanes of each quarter warp read
+    // their pair in the opposite order, so each read instruction's quarter
+    // warp covers the eight bank groups once whatever rows it reads
+    const int ph = kDT == 8 ? (threadIdx.x >> 2) & 1 : 0;
     const int64_t n_rec = a.n_rec;
     // advancing by vpi vectors: step_r records and step_b sequences, plus one
     // more sequence when the record wraps
@@ -177,11 +197,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
         // kU vectors per round: their index loads are all issued before any is used
         constexpr int kU = 4;
         for (; n_it > 0; n_it -= kU) {
-            uint64_t ids[kU];
+            using Ids = typename std::conditional<S * kBits <= 32, uint32_t, uint64_t>::type;
+            Ids ids[kU];
             int64_t off[kU];
 #pragma unroll
             for (int u = 0; u < kU; ++u) {
-                ids[u] = u < n_it ? load_ids<S, WIDE>(ip) : 0;
+                ids[u] = u < n_it ? static_cast<Ids>(load_ids<S, WIDE>(ip)) : 0;
                 off[u] = oe;
                 rec += step_r;
                 ip += di_step;
@@ -196,16 +217,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
             for (int u = 0; u < kU; ++u) {
                 if (u >= n_it)
                     break;
-                float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+                if constexpr (kDT == 8) {
+                    float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f), y = x;
+                    const int ga = 2 * dq + ph, gb = 2 * dq + 1 - ph;
 #pragma unroll
-                for (int s = 0; s < S; ++s) {
-                    const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
-                    const int xq = xor_rows ? (row >> 1) & 3 : 0;
-                    const float4 c = row0[row * q4 + (dq ^ xq)];
-                    add2(x.x, x.y, c.x, c.y);
-                    add2(x.z, x.w, c.z, c.w);
+                    for (int s = 0; s < S; ++s) {
+                        const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
+                        const float4 c = row0[row * q4 + ga];
+                        const float4 e = row0[row * q4 + gb];
+                        add2(x.x, x.y, c.x, c.y);
+                        add2(x.z, x.w, c.z, c.w);
+                        add2(y.x, y.y, e.x, e.y);
+                        add2(y.z, y.w, e.z, e.w);
+                    }
+                    store8(a.out, a.dtype, off[u], ph ? y : x, ph ? x : y);
+                } else {
+                    float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+                    for (int s = 0; s < S; ++s) {
+                        const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
+                        const int xq = xor_rows ? (row >> 1) & 3 : 0;
+                        const float4 c = row0[row * q4 + (dq ^ xq)];
+                        add2(x.x, x.y, c.x, c.y);
+                        add2(x.z, x.w, c.z, c.w);
+                    }
+                    store4(a.out, a.dtype, off[u], x);
                 }
-                store4(a.out, a.dtype, off[u], x);
             }
         }
     }
