@@ -181,7 +181,7 @@ def test_edge_vectors(fkv, oracle_mod, dim):
     cbk[0, 0, 1] *= 0.5
     cbk[0, 0, 0, 200] = cbk[0, 0, 0, 9]                  # duplicate codeword
     cbv = rng.normal(size=(1, 1, 1, 256, dim)).astype(np.float32)
-    for n in [1, 127, 129, 300]:
+    for n in [1, 6, 16, 127, 129, 300]:
         x = rng.normal(size=(n, dim))
         x[0] = cbk[0, 0, 0, 9]                            # equal to a (duplicated) codeword
         if n > 5:
@@ -200,6 +200,52 @@ def test_edge_vectors(fkv, oracle_mod, dim):
         assert idx[0, 0] == 9
         if n > 5:
             assert idx[1, 0] == 77 and idx[5, 0] == 3
+
+
+@pytest.mark.parametrize("dim,dtype,K,pooled", [(64, "f16", 256, False), (64, "f32", 256, False),
+                                                (64, "bf16", 1024, True), (128, "bf16", 256, False)])
+def test_small_batch(fkv, oracle_mod, dim, dtype, K, pooled):
+    """At most 16 vectors per codebook group (a decode step's appended
+    position: tiles with 1 to 16 live rows of 128): every index equals the
+    oracle's outside near ties, for several (batch, positions) shapes, with
+    rows far outside and far inside the codebooks' scale, codeword-equal rows
+    and zero rows, per-head and pooled codebooks."""
+    rng = np.random.default_rng(dim + K + len(dtype))
+    L, H = 2, 3
+    Hc = 1 if pooled else H
+    SK = 2 if K == 1024 else 3                          # 1024-codeword codebooks: two stages at most
+    cbk = rng.normal(size=(L, Hc, SK, K, dim)).astype(np.float32)
+    cbk[:, :, 1] *= 0.3
+    cbk[:, :, SK - 1] *= 1e-3                           # another power-of-two scale
+    cbv = rng.normal(size=(L, Hc, 2, K, dim)).astype(np.float32)
+    big, small = (1e3, 1e-3) if dtype == "f16" else (1e30, 1e-30)
+    ctx = fkv.Context(K, codebooks=(cbk, cbv), pooled=pooled, n_heads=H if pooled else None)
+    R = ctx.record_len()
+    for batch, npos in [(1, 1), (8, 1), (3, 5), (2, 8), (1, 16)]:
+        t0, seq = 3, npos + 7
+        x = rng.normal(size=(L, batch, H, seq, dim))
+        x[0, 0, 0, t0] *= big
+        x[1, 0, 1, t0] *= small
+        x[0, 0, 2, t0] = 0.0
+        x[1, 0, 0, t0] = cbk[1, 0, 0, 17]
+        X = torch.from_numpy(x).to(TORCH_DT[dtype]).cuda()
+        x64 = X.double().cpu().numpy()
+        sym = torch.zeros((batch * L, npos * R), dtype=ctx.sym_dtype, device="cuda")
+        ctx.rvq_encode(0, X, t0, t0 + npos, sym)
+        ctx.rvq_encode(1, X, t0, t0 + npos, sym)
+        assert ctx.sync_status() == 0
+        s = sym.cpu().numpy().astype(np.int32).reshape(batch, L, npos * R)
+        assert s.max() < K
+        for b in range(batch):
+            for l in range(L):
+                ik, iv = oracle_mod.indices_from_records(s[b, l], H, SK, 2)
+                for h in range(H):
+                    for gidx, cb in ((ik, cbk), (iv, cbv)):
+                        oi, gap = oracle_mod.rvq_encode(x64[l, b, h, t0:t0 + npos], cb[l, 0 if pooled else h])
+                        hard, near, seen = compare_rvq(gidx[h], oi, gap)
+                        assert hard == 0, (batch, npos, b, l, h, hard)
+        ik, _ = oracle_mod.indices_from_records(s[0, 1], H, SK, 2)
+        assert ik[0, 0, 0] == 17                        # the codeword-equal row
 
 
 @pytest.mark.parametrize("k1024", [False, True])
