@@ -318,17 +318,17 @@ def run_gpu(args, rank, world, local_rank):
     codec = None
     if not args.no_codec:
         codec = {}
-        n = 1 << 28
-        for N in (3, 4, 16, 256):
-            cc = fkv.Context(N)
-            c_sym = synth.gpu_symbols(N, "uniform", 4, n, device=dev)
+        c_n = 1 << 28
+        for c_N in (3, 4, 16, 256):
+            cc = fkv.Context(c_N)
+            c_sym = synth.gpu_symbols(c_N, "uniform", 4, c_n, device=dev)
             c_pts = cc.span_encode(c_sym)
             c_dec = torch.empty_like(c_sym)
-            req = torch.cat([torch.stack([torch.full((1 << 20,), s_, dtype=torch.int64, device=dev),
-                                          synth.gpu_positions(n, 1 << 20, s_, device=dev)], 1) for s_ in range(4)])
-            c_out = torch.empty(req.shape[0], dtype=c_sym.dtype, device=dev)
-            ops = (lambda: cc.span_encode(c_sym, c_pts), lambda: cc.span_decode(c_pts, n, c_dec),
-                   lambda: cc.read(c_pts, n, req, c_out))
+            c_req = torch.cat([torch.stack([torch.full((1 << 20,), s_, dtype=torch.int64, device=dev),
+                                          synth.gpu_positions(c_n, 1 << 20, s_, device=dev)], 1) for s_ in range(4)])
+            c_out = torch.empty(c_req.shape[0], dtype=c_sym.dtype, device=dev)
+            ops = (lambda: cc.span_encode(c_sym, c_pts), lambda: cc.span_decode(c_pts, c_n, c_dec),
+                   lambda: cc.read(c_pts, c_n, c_req, c_out))
             for op in ops:
                 op()
             reps = 3
@@ -341,10 +341,10 @@ def run_gpu(args, rank, world, local_rank):
                 e1.record(stream)
                 torch.cuda.synchronize()
                 ms_.append(e0.elapsed_time(e1) / reps)
-            exact = bool(torch.equal(c_dec, c_sym)) and bool(torch.equal(c_out, c_sym[req[:, 0], req[:, 1]]))
-            codec[N] = {"L": cc.L, "spans": c_pts.shape[1], "encode_ms": ms_[0], "decode_ms": ms_[1],
-                        "read_ms": ms_[2], "reads": req.shape[0], "exact": exact, "ok": cc.sync_status() == 0}
-            del c_sym, c_pts, c_dec, req, c_out, cc
+            exact = bool(torch.equal(c_dec, c_sym)) and bool(torch.equal(c_out, c_sym[c_req[:, 0], c_req[:, 1]]))
+            codec[c_N] = {"L": cc.L, "spans": c_pts.shape[1], "encode_ms": ms_[0], "decode_ms": ms_[1],
+                        "read_ms": ms_[2], "reads": c_req.shape[0], "exact": exact, "ok": cc.sync_status() == 0}
+            del c_sym, c_pts, c_dec, c_req, c_out, cc
 
     # Sec. 4 lossy archive of this step's streams: spans older than the last
     # 64 records truncated to 24 bits per coordinate (6 B instead of 16 B per
