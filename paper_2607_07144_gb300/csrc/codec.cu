@@ -133,6 +133,51 @@ __host__ __device__ inline int tables_bytes(int N, int L)
     return (fkvdec::smem_bytes(N, L) + 15) & ~15;
 }
 
+// Decode span s of `stream` (one per thread): the walk's symbols go through
+// `put(j, c)`, j = 0 .. m-1 from the span's last symbol back to its first,
+// straight from registers to their place; a point whose walk does not end at
+// the anchor sets the corrupt status.
+template <class Put>
+__device__ __forceinline__ void decode_span(const fkvdec::Tables &t, const double2 *__restrict__ pts, int64_t n,
+                                            int64_t pt_stride, int64_t stream, int64_t s,
+                                            const fkv_decconst *__restrict__ dc, int L, unsigned *status, Put put,
+                                            int &m)
+{
+    m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+    const double2 p = pts[stream * pt_stride + s];
+    long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+    fkvdec::walk(t, X, Y, m, put);
+    const long long lim = __ldg(&dc->alim[m]);
+    if (X > lim || X < -lim || Y > lim || Y < -lim)
+        atomicOr(status, FKV_ST_CORRUPT);
+}
+
+// Persistent: a block loads the decoder tables once and walks chunks of
+// dec_threads spans (chunk = stream * bps + span block), blockIdx.x,
+// + gridDim.x, ...; each thread stores its span's symbols directly, so the
+// chunks need no block barrier.
+template <typename Sym>
+__global__ void __launch_bounds__(dec_threads<Sym>())
+k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
+              int64_t n_chunks, Sym *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
+              const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    __syncthreads();
+    constexpr int TPB = dec_threads<Sym>();
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
+        const int64_t stream = ck / bps;
+        const int64_t s = (ck - stream * bps) * TPB + threadIdx.x;
+        if (s >= spans)
+            continue;
+        Sym *dst = sym + stream * sym_stride + s * L;
+        int m = 0;
+        decode_span(t, pts, n, pt_stride, stream, s, dc, L, status,
+                    [&](int j, int c) { dst[m - 1 - j] = static_cast<Sym>(c); }, m);
+    }
+}
+
 // Decode 256 spans of one stream (chunk `ck` of the n_streams * bps chunks)
 // into sbuf (one span per thread, symbol i of the chunk at sbuf[i]).
 template <typename Sym>
@@ -154,11 +199,14 @@ __device__ __forceinline__ void decode_chunk(const fkvdec::Tables &t, const doub
     }
 }
 
-// Persistent: a block loads the decoder tables once and walks chunks of 256
-// spans (chunk = stream * bps + span block), blockIdx.x, + gridDim.x, ...
+// The stream decode for long spans (more than 8 symbols): a chunk's symbols
+// are staged in shared memory and written out with aligned 16-byte stores,
+// since a thread's own span would otherwise be a run of scattered byte
+// stores.  Persistent: chunk = stream * bps + span block, blockIdx.x,
+// + gridDim.x, ...
 template <typename Sym>
 __global__ void __launch_bounds__(dec_threads<Sym>())
-k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
+k_span_decode_staged(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int64_t spans, int bps,
               int64_t n_chunks, Sym *__restrict__ sym, int64_t sym_stride, const fkv_decconst *__restrict__ dc,
               const longlong2 *__restrict__ T, int N, int L, unsigned *status)
 {
@@ -184,9 +232,10 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
 // The same decode for a whole archive of token records, written out in the
 // planar layout the archive gather reads: per stream, the H key planes
 // (n_rec x S_K indices each, one plane per head) and then the H value planes
-// (n_rec x S_V).  A chunk's records are written plane by plane, a thread per
-// (record, stage) slot of the run, consecutive threads on consecutive bytes; a
-// record cut by the chunk boundary is completed by the neighbouring chunk.
+// (n_rec x S_V).  A thread places each symbol of its span as the walk yields
+// it, last to first, stepping a (record, K or V, head, stage) position back
+// by one per symbol from the one of the span's last symbol (one division per
+// span).
 template <typename Sym>
 __global__ void __launch_bounds__(dec_threads<Sym>())
 k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
@@ -196,38 +245,50 @@ k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    Sym *sbuf = reinterpret_cast<Sym *>(dsm + tables_bytes(N, L));
     __syncthreads();
     const int R = H * (SK + SV);
     const int nk = H * SK;
     const int64_t n = n_rec * R;
+    const int64_t vplanes = static_cast<int64_t>(nk) * n_rec;     // offset of the value planes
     constexpr int TPB = dec_threads<Sym>();
     for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
         const int64_t stream = ck / bps;
-        const int64_t s0 = (ck - stream * bps) * TPB;
-        const int64_t q0 = s0 * L;
-        const int64_t q1 = min(n, (s0 + TPB) * L);
-        decode_chunk(t, pts, n, pt_stride, spans, stream, s0, sbuf, dc, L, status);
-        __syncthreads();
-        // records [rec_lo, rec_lo + nrb) overlap this chunk's symbols [q0, q1)
-        const int64_t rec_lo = q0 / R;
-        const int nrb = static_cast<int>((q1 - 1) / R - rec_lo + 1);
+        const int64_t s = (ck - stream * bps) * TPB + threadIdx.x;
+        if (s >= spans)
+            continue;
         Sym *base = out + stream * n;
-        for (int kv = 0; kv < 2; ++kv) {
-            const int S = kv == 0 ? SK : SV;
-            const int o0 = kv == 0 ? 0 : nk;                       // first offset of this half in a record
-            Sym *pl = base + (kv == 0 ? 0 : static_cast<int64_t>(nk) * n_rec) + rec_lo * S;
-            for (int i = threadIdx.x; i < nrb * S; i += TPB) {
-                const int j = i / S, st = i - j * S;               // record j of the chunk, stage st
-                const int64_t qj = (rec_lo + j) * R + o0 + st - q0; // symbol of head 0, relative to q0
-                for (int h = 0; h < H; ++h) {
-                    const int64_t q = qj + h * S;
-                    if (q >= 0 && q < q1 - q0)
-                        pl[static_cast<int64_t>(h) * n_rec * S + i] = sbuf[q];
-                }
-            }
-        }
-        __syncthreads();
+        // position of the span's last symbol
+        const int64_t q = min(s * L + L, n) - 1;
+        int64_t rec = q / R;
+        int o = static_cast<int>(q - rec * R);
+        int seg = o < nk ? 0 : 1;
+        if (seg)
+            o -= nk;
+        const int S0 = seg ? SV : SK;
+        int h = o / S0, st = o - h * S0;
+        int m = 0;
+        decode_span(t, pts, n, pt_stride, stream, s, dc, L, status,
+                    [&](int, int c) {
+                        const int Sg = seg ? SV : SK;
+                        base[(seg ? vplanes : 0) + static_cast<int64_t>(h) * n_rec * Sg + rec * Sg + st] =
+                            static_cast<Sym>(c);
+                        if (st > 0) {
+                            --st;
+                        } else if (h > 0) {
+                            --h;
+                            st = Sg - 1;
+                        } else if (seg) {
+                            seg = 0;
+                            h = H - 1;
+                            st = SK - 1;
+                        } else {
+                            seg = 1;
+                            h = H - 1;
+                            st = SV - 1;
+                            --rec;
+                        }
+                    },
+                    m);
     }
 }
 
@@ -691,17 +752,26 @@ cudaError_t span_decode_t(const fkv_ctx *c, const double *pts, int64_t n_streams
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + dec_stage_bytes<Sym>(c->L);
-    cudaError_t e = cudaFuncSetAttribute(k_span_decode<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    // spans of up to 8 symbols: each thread stores its own; longer ones: staged
+    const bool direct = c->L <= 8;
+    const void *kern = direct ? reinterpret_cast<const void *>(k_span_decode<Sym>)
+                              : reinterpret_cast<const void *>(k_span_decode_staged<Sym>);
+    const int smem = tables_bytes(c->N, c->L) + (direct ? 0 : dec_stage_bytes<Sym>(c->L));
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
     unsigned grid = 0;
-    e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode<Sym>), smem, n_chunks, &grid, TPB);
+    e = decode_grid(c, kern, smem, n_chunks, &grid, TPB);
     if (e != cudaSuccess)
         return e;
-    k_span_decode<Sym><<<grid, TPB, smem, st>>>(reinterpret_cast<const double2 *>(pts), n, pt_stride, spans,
-                                                     static_cast<int>(bps), n_chunks, sym, sym_stride, c->d_dec,
-                                                     c->d_T, c->N, c->L, c->d_status);
+    const double2 *p2 = reinterpret_cast<const double2 *>(pts);
+    if (direct)
+        k_span_decode<Sym><<<grid, TPB, smem, st>>>(p2, n, pt_stride, spans, static_cast<int>(bps), n_chunks, sym,
+                                                         sym_stride, c->d_dec, c->d_T, c->N, c->L, c->d_status);
+    else
+        k_span_decode_staged<Sym><<<grid, TPB, smem, st>>>(p2, n, pt_stride, spans, static_cast<int>(bps), n_chunks,
+                                                                sym, sym_stride, c->d_dec, c->d_T, c->N, c->L,
+                                                                c->d_status);
     return cudaGetLastError();
 }
 
@@ -727,7 +797,7 @@ cudaError_t span_decode_planar_t(const fkv_ctx *c, const double *pts, int64_t n_
         return cudaSuccess;
     if (bps > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L) + dec_stage_bytes<Sym>(c->L);
+    const int smem = tables_bytes(c->N, c->L);
     cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          smem);
     if (e != cudaSuccess)
