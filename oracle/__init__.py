@@ -13,9 +13,22 @@ and adds the bookkeeping the paper states in words:
 * the token-record order of the archived index stream (a reading: the paper
   does not state it), and
 * the round-to-nearest-even cast of a float64 reconstruction to fp16/bf16/fp32,
-* the in-place suffix retrieval of Sec. 5, and
+* the in-place suffix retrieval of Sec. 5,
 * the lossy truncation of Sec. 4 (B-bit codes of the stored points, their
-  packed layout, recency allocation across spans).
+  packed layout, recency allocation across spans), and
+* the probability-weighted maps of Sec. 6 eq. (1) (integer arithmetic coding
+  with an add-one adaptive or a uniform model).
+
+Pins (tests/test_oracle_*.py): r_N = 1/2 at N = 3, 4 and a brute-force
+disjointness bisection for other N; the N = 3 and N = 4 midpoint closed forms
+and exact rational evaluation of the map (tests/golden/); exhaustive round
+trips of tiny streams and the 44/log2(1/r) capacity; the 2 r^s suffix decay;
+RVQ against brute force and codeword-equal inputs; the storage identities of
+Sec. 3; hand-computed lossy codes and layouts with the lossless limit; the
+uniform arithmetic code's plain-binary pattern and the code-length bound.
+Parity unpinned: the paper's printed byte counts of Table 2, Table 3's lossy
+rates and Table 4's bits per character (they need the paper's corpus and
+trained codebooks; the functions computing them are pinned as above).
 """
 from __future__ import annotations
 
