@@ -21,7 +21,8 @@ and adds the bookkeeping the paper states in words:
 
 Pins (tests/test_oracle_*.py): r_N = 1/2 at N = 3, 4 and a brute-force
 disjointness bisection for other N; the N = 3 and N = 4 midpoint closed forms
-and exact rational evaluation of the map (tests/golden/); exhaustive round
+(hand-worked points in tests/golden/) and exact rational evaluation of the
+map's closed form; exhaustive round
 trips of tiny streams and the 44/log2(1/r) capacity; the 2 r^s suffix decay;
 RVQ against brute force and codeword-equal inputs; the storage identities of
 Sec. 3; hand-computed lossy codes and layouts with the lossless limit; the
