@@ -16,6 +16,17 @@ One step is one pass of the whole archive path over that cache:
   6. 4096 random record reads (K and V of all heads of one position).
 value = archived KV positions (sequence x layer x position records) per second
 over the whole step.  Inputs (302 MB) are larger than L2, so no flush is needed.
+`e2e` times the same step through the public API with the caches in pinned host
+memory (host -> device copies and the result read-back inside the timed region).
+
+After the timed steps the line also reports, under "kernels", secondary
+workloads, each measured on its own (a --no-<name> flag skips it):
+  suffix    Sec. 5 retrieval over 4 streams x 2^28 symbols;
+  codec     the span codec on the symbol-stress streams (N = 3, 4, 16, 256);
+  k1024     Table 2's pooled RVQ 1024 x 2 archive of the same cache;
+  lossy     Sec. 4 truncation and lossy decode of this step's streams;
+  llama     the Llama-3-8B-shaped archive (--llama-seq sets its cache length);
+  weighted  Sec. 6 probability-weighted maps of this step's index streams.
 
 --impl reference times the float64 CPU oracle on a bounded sample of the same
 workload (the paper ships no GPU implementation; the oracle is the reference).
