@@ -787,6 +787,9 @@ def main():
         "kernels": kernels,
         "cpu_baseline": cpu,
         "e2e": e2e,
+        # per step: k_rvq64 x4 (K and V archive, K and V of the appended
+        # position), k_span_encode x2 (archive, tail append),
+        # k_span_decode_planar, k_gather x2, k_read_kv (profiles' launch list)
         "gpu_launches": 10 * args.steps,
         "clocks": res["clocks"],
         "status_ok": res["ok"],
