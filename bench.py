@@ -65,9 +65,10 @@ def load_peaks():
 
 
 # DRAM bytes (read + write) per k_rvq64 launch of this workload, the mean of
-# the key launch (197,526,272) and the value launch (171,083,008) from one ncu
-# capture of the current kernel (profiles/k_rvq64_gpt2_full_cache.md); set it
-# to None whenever that kernel changes until it is captured again.
+# the key launch (197,526,272) and the value launch (171,083,008) in one ncu
+# capture (dram__bytes_read.sum + dram__bytes_write.sum) of the current
+# kernel; set it to None whenever that kernel changes until it is captured
+# again.
 RVQ_DRAM_BYTES_PER_LAUNCH = 184304640
 
 # FP64 add/mul peak: GB300's nominal 1.25 TFLOP/s of FP64 FMA is 625 G add or
@@ -789,7 +790,7 @@ def main():
         "e2e": e2e,
         # per step: k_rvq64 x4 (K and V archive, K and V of the appended
         # position), k_span_encode x2 (archive, tail append),
-        # k_span_decode_planar, k_gather x2, k_read_kv (profiles' launch list)
+        # k_span_decode_planar, k_gather x2, k_read_kv (as the ncu launch list shows)
         "gpu_launches": 10 * args.steps,
         "clocks": res["clocks"],
         "status_ok": res["ok"],
