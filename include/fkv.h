@@ -119,7 +119,9 @@ int fkv_symbol_bytes(const fkv_ctx *ctx);
 const char *fkv_last_error(const fkv_ctx *ctx);
 
 /* Wait for `stream`, then return and clear the device status word:
- * FKV_OK, FKV_ECORRUPT or FKV_ETIMEOUT. */
+ * FKV_OK, or the first of FKV_ETIMEOUT (a bounded device wait ran out),
+ * FKV_ECORRUPT (a corrupt point or symbol) and FKV_ERANGE (a request named a
+ * position, record or stream outside the archive) that was recorded. */
 int fkv_sync_status(fkv_ctx *ctx, void *stream);
 
 /* -------------------------------------------------- bulk symbol codec --- */
@@ -153,9 +155,35 @@ int fkv_span_decode(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int6
  * (at most span_len backward steps).  Points laid out as in fkv_span_encode.
  * out_dev holds symbols of the context's width.  A request outside
  * [0, n_streams) x [0, n) writes all ones (0xFF or 0xFFFF) to out_dev[q] and
- * sets FKV_ECORRUPT. */
+ * sets FKV_ERANGE in the status word. */
 int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, int64_t pt_stride,
              const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
+
+/* The same three calls for a ragged batch: streams of different lengths in
+ * one call, as the sequences of a serving batch are (Sec. 2 applies the code
+ * per sequence; nothing in it ties the streams' lengths together).
+ *   sym_off_dev: int64 [n_streams + 1], DEVICE memory, caller-owned: stream
+ *                i's symbols are sym_dev[sym_off_dev[i] .. sym_off_dev[i+1])
+ *                (symbols of the context's width), len_i their count;
+ *   pt_off_dev:  int64 [n_streams + 1], DEVICE memory, caller-owned: stream
+ *                i's points occupy point slots [pt_off_dev[i],
+ *                pt_off_dev[i+1]) of pts_dev (slot g at pts_dev[2 g]), at
+ *                least ceil(len_i / span_len) of them; slots past the
+ *                stream's last span are left untouched.
+ * Both arrays must be nondecreasing.  The host checks pointers and alignment
+ * (FKV_EINVAL, nothing launched); the offsets are read on the device, where a
+ * stream with a negative length or too few point slots is skipped and sets
+ * FKV_ERANGE in the status word.  Span contents, arithmetic and the corrupt
+ * status are those of fkv_span_encode / fkv_span_decode.  fkv_read_ragged
+ * takes requests req_dev[2q] = stream, req_dev[2q + 1] = position within
+ * that stream; a request outside [0, n_streams) x [0, len_i) writes all ones
+ * to out_dev[q] and sets FKV_ERANGE. */
+int fkv_span_encode_ragged(fkv_ctx *ctx, const void *sym_dev, const int64_t *sym_off_dev, int64_t n_streams,
+                           double *pts_dev, const int64_t *pt_off_dev, void *stream);
+int fkv_span_decode_ragged(fkv_ctx *ctx, const double *pts_dev, const int64_t *pt_off_dev, int64_t n_streams,
+                           void *sym_dev, const int64_t *sym_off_dev, void *stream);
+int fkv_read_ragged(fkv_ctx *ctx, const double *pts_dev, const int64_t *pt_off_dev, const int64_t *sym_off_dev,
+                    int64_t n_streams, const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
 
 /* Sec. 5: in-place suffix retrieval over the stored points, with no
  * decompression of the archive.  query (host memory, the context's symbol
@@ -215,8 +243,9 @@ int fkv_lossy_decode(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_strid
                      int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
                      void *sym_dev, int64_t sym_stride, void *stream);
 
-/* Sec. 2 random access into a lossy archive: requests as in fkv_read, each
- * decoded from its span's kept point as fkv_lossy_decode does. */
+/* Sec. 2 random access into a lossy archive: requests as in fkv_read (an
+ * out-of-range request writes all ones and sets FKV_ERANGE), each decoded
+ * from its span's kept point as fkv_lossy_decode does. */
 int fkv_lossy_read(fkv_ctx *ctx, const uint32_t *codes_dev, int64_t code_stride, const double *tail_dev,
                    int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
                    const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream);
@@ -252,6 +281,15 @@ int fkv_ac_encode(fkv_ctx *ctx, const void *sym_dev, int64_t n_streams, int64_t 
  * symbols and set FKV_ECORRUPT. */
 int fkv_ac_decode(fkv_ctx *ctx, const uint32_t *words_dev, int64_t word_stride, const int64_t *nbits_dev,
                   int64_t n_streams, int64_t n, int adaptive, void *sym_dev, int64_t sym_stride, void *stream);
+
+/* Measurement utility (no counterpart in the paper): binary64 add and
+ * multiply instructions per second of the current device, measured by
+ * independent chains of round-to-nearest multiplies and adds (no FMA), the
+ * operation mix of the span encoder (Sec. 1: six such operations per
+ * symbol).  It is the measured denominator of span encoding's roofline on a
+ * GPU whose FP64 rate, not memory, bounds it.  Launches about 30 ms of work
+ * on `stream` and waits for it; writes the rate to *ops_per_s (host). */
+int fkv_measure_fp64_rate(double *ops_per_s, void *stream);
 
 /* -------------------------------------------------- K/V archive path ---- */
 
@@ -346,7 +384,7 @@ int fkv_cache_upload(fkv_ctx *ctx, const fkv_cache *src_host, const fkv_cache *d
  * decode only the spans of that record and write its K and V head vectors to
  * out_dev, laid out [n_req][2 (K, V)][n_heads][dim] in `dtype`.  Streams hold
  * n_rec records each, points as in fkv_decode_kv.  Out-of-range requests
- * write zeros and set FKV_ECORRUPT. */
+ * write zeros and set FKV_ERANGE. */
 int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec,
                 int64_t pt_stride, const int64_t *req_dev, int64_t n_req, void *out_dev,
                 int dtype, void *stream);

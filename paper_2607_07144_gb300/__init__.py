@@ -5,7 +5,7 @@ this package is its thin Python binding.  Build with
 ``paper_2607_07144_gb300.build.build()`` or ``__graft_entry__.build()``.
 """
 from ._binding import (BF16, F16, F32, Context, FkvError, Streams, cache_view, lib,  # noqa: F401
-                       max_span_len, packing_ratio)
+                       max_span_len, measure_fp64_rate, packing_ratio)
 
-__all__ = ["Context", "Streams", "FkvError", "lib", "packing_ratio", "max_span_len", "cache_view",
+__all__ = ["Context", "Streams", "FkvError", "lib", "packing_ratio", "max_span_len", "cache_view", "measure_fp64_rate",
            "F32", "F16", "BF16"]

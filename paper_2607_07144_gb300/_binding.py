@@ -58,6 +58,9 @@ SIGNATURES = {
     "fkv_span_encode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
     "fkv_span_decode": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P]),
     "fkv_read": (_I, [_P, _P, _I64, _I64, _I64, _P, _I64, _P, _P]),
+    "fkv_span_encode_ragged": (_I, [_P, _P, _P, _I64, _P, _P, _P]),
+    "fkv_span_decode_ragged": (_I, [_P, _P, _P, _I64, _P, _P, _P]),
+    "fkv_read_ragged": (_I, [_P, _P, _P, _P, _I64, _P, _I64, _P, _P]),
     "fkv_suffix_search": (_I, [_P, _P, _I64, _I64, _I64, _P, _I, _P, _I64, _P, _P]),
     "fkv_truncate": (_I, [_P, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P, _I64, _P]),
     "fkv_lossy_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I64, _I, _I64, _P, _I64, _P]),
@@ -65,6 +68,7 @@ SIGNATURES = {
     "fkv_ac_capacity_words": (_I64, [_P, _I64]),
     "fkv_ac_encode": (_I, [_P, _P, _I64, _I64, _I64, _I, _P, _I64, _P, _P]),
     "fkv_ac_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I, _P, _I64, _P]),
+    "fkv_measure_fp64_rate": (_I, [_P, _P]),
     "fkv_record_len": (_I, [_P]),
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
@@ -122,6 +126,15 @@ def packing_ratio(N: int) -> float:
 
 def max_span_len(r: float) -> int:
     return lib().fkv_max_span_len(float(r))
+
+
+def measure_fp64_rate(stream=None) -> float:
+    """Binary64 add/mul instructions per second of the current device."""
+    v = ctypes.c_double()
+    rc = lib().fkv_measure_fp64_rate(ctypes.byref(v), _stream(stream))
+    if rc != OK:
+        raise FkvError(rc, "fkv_measure_fp64_rate failed")
+    return v.value
 
 
 def cache_view(t: torch.Tensor, host: bool = False) -> _Cache:
@@ -244,6 +257,50 @@ class Context:
         self._sym(out)
         self._check(lib().fkv_read(self._h, _ptr(pts), pts.shape[0], n, _rows(pts, 2), _ptr(req), req.shape[0],
                                    _ptr(out), _stream(stream)))
+        return out
+
+    # -- ragged batches (streams of different lengths in one call)
+    def ragged_offsets(self, lengths, device="cuda"):
+        """Packed offsets for streams of the given lengths: (sym_off, pt_off),
+        int64 [n_streams + 1] device tensors (points packed with no slack)."""
+        ln = np.asarray(lengths, np.int64).ravel()
+        so = np.concatenate([[0], np.cumsum(ln)]).astype(np.int64)
+        po = np.concatenate([[0], np.cumsum((ln + self.L - 1) // self.L)]).astype(np.int64)
+        return torch.from_numpy(so).to(device), torch.from_numpy(po).to(device)
+
+    def span_encode_ragged(self, sym: torch.Tensor, sym_off: torch.Tensor, pt_off: torch.Tensor,
+                           pts: torch.Tensor = None, n_slots: int = None, stream=None) -> torch.Tensor:
+        """sym: flat symbols (sym_dtype) of all streams; sym_off, pt_off: int64
+        [n_streams + 1] device offsets -> pts float64 [slots, 2] (n_slots, or
+        pt_off's last entry read back, a synchronisation, when pts is None)."""
+        self._sym(sym)
+        ns = sym_off.numel() - 1
+        if pts is None:
+            slots = int(pt_off[-1].item()) if n_slots is None else int(n_slots)
+            pts = torch.empty((max(slots, 1), 2), dtype=torch.float64, device=sym.device)
+        self._check(lib().fkv_span_encode_ragged(self._h, _ptr(sym), _ptr(sym_off), ns, _ptr(pts), _ptr(pt_off),
+                                                 _stream(stream)))
+        return pts
+
+    def span_decode_ragged(self, pts: torch.Tensor, pt_off: torch.Tensor, sym_off: torch.Tensor,
+                           sym: torch.Tensor = None, n_sym: int = None, stream=None) -> torch.Tensor:
+        ns = sym_off.numel() - 1
+        if sym is None:
+            n = int(sym_off[-1].item()) if n_sym is None else int(n_sym)
+            sym = torch.empty(max(n, 1), dtype=self.sym_dtype, device=pts.device)
+        self._sym(sym)
+        self._check(lib().fkv_span_decode_ragged(self._h, _ptr(pts), _ptr(pt_off), ns, _ptr(sym), _ptr(sym_off),
+                                                 _stream(stream)))
+        return sym
+
+    def read_ragged(self, pts: torch.Tensor, pt_off: torch.Tensor, sym_off: torch.Tensor, req: torch.Tensor,
+                    out: torch.Tensor = None, stream=None) -> torch.Tensor:
+        """req int64 [n_req, 2] = (stream, position within it) -> symbols [n_req]."""
+        if out is None:
+            out = torch.empty(req.shape[0], dtype=self.sym_dtype, device=pts.device)
+        self._sym(out)
+        self._check(lib().fkv_read_ragged(self._h, _ptr(pts), _ptr(pt_off), _ptr(sym_off), sym_off.numel() - 1,
+                                          _ptr(req), req.shape[0], _ptr(out), _stream(stream)))
         return out
 
     def suffix_search(self, pts: torch.Tensor, n: int, query, cap: int = 1 << 16, match: torch.Tensor = None,

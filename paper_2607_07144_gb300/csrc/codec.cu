@@ -409,7 +409,7 @@ k_read(const double2 *__restrict__ pts, int64_t n_streams, int64_t n, int64_t pt
         const int64_t st = req[2 * q], pos = req[2 * q + 1];
         if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
             out[q] = static_cast<Sym>(~0u);
-            atomicOr(status, FKV_ST_CORRUPT);
+            atomicOr(status, FKV_ST_RANGE);
             continue;
         }
         const int64_t u = pos / L;
@@ -456,6 +456,145 @@ k_append(double2 *__restrict__ pts, int64_t n_streams, int64_t pt_stride, int64_
     if (isnan(p.x))
         atomicOr(status, FKV_ST_CORRUPT);
     pts[stream * pt_stride + u] = p;
+}
+
+// ------------------------------------------------------------ ragged batches
+// Streams of different lengths in one call (the sequences of a serving batch
+// rarely share a length): stream i holds len_i = so[i + 1] - so[i] symbols at
+// sym + so[i] and owns point slots [po[i], po[i + 1]) of pts, at least
+// ceil(len_i / L) of them.  so and po are device arrays of n_streams + 1
+// offsets.  The kernels walk the point slots [po[0], po[n_streams])
+// grid-stride, one span per thread, and find a slot's stream by binary search
+// over po.  A stream whose offsets are inconsistent (a negative length, fewer
+// point slots than spans) is left alone and reported by the range status bit;
+// the check runs once per stream, so a stream with no slots is reported too.
+
+// The stream owning point slot g: the largest i < n_streams with po[i] <= g
+// (po nondecreasing; every index read stays in [0, n_streams]).
+__device__ __forceinline__ int64_t ragged_stream(const int64_t *__restrict__ po, int64_t n_streams, int64_t g)
+{
+    int64_t lo = 0, hi = n_streams;
+    while (hi - lo > 1) {
+        const int64_t mid = (lo + hi) >> 1;
+        if (__ldg(&po[mid]) <= g)
+            lo = mid;
+        else
+            hi = mid;
+    }
+    return lo;
+}
+
+// Length of stream i and whether its offsets hold together.
+__device__ __forceinline__ bool ragged_ok(const int64_t *__restrict__ so, const int64_t *__restrict__ po, int64_t i,
+                                          int L, int64_t *len)
+{
+    const int64_t n = __ldg(&so[i + 1]) - __ldg(&so[i]);
+    const int64_t slots = __ldg(&po[i + 1]) - __ldg(&po[i]);
+    *len = n;
+    return n >= 0 && slots >= 0 && slots >= (n + L - 1) / L;
+}
+
+// Every thread of the grid takes part in checking the streams' offsets.
+__device__ __forceinline__ void ragged_check(const int64_t *__restrict__ so, const int64_t *__restrict__ po,
+                                             int64_t n_streams, int L, unsigned *status)
+{
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n_streams; i += stride) {
+        int64_t n;
+        if (!ragged_ok(so, po, i, L, &n))
+            atomicOr(status, FKV_ST_RANGE);
+    }
+}
+
+template <typename Sym>
+__global__ void __launch_bounds__(kThreads)
+k_span_encode_ragged(const Sym *__restrict__ sym, const int64_t *__restrict__ so, int64_t n_streams,
+                     double2 *__restrict__ pts, const int64_t *__restrict__ po, const double2 *__restrict__ V,
+                     int N, double r, int L, unsigned *status)
+{
+    __shared__ double2 sV[vtab_len<Sym>()];
+    for (int i = threadIdx.x; i < N; i += kThreads)
+        sV[i] = V[i];
+    __syncthreads();
+    ragged_check(so, po, n_streams, L, status);
+    const int64_t g0 = __ldg(&po[0]), g1 = __ldg(&po[n_streams]);
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * kThreads;
+    for (int64_t g = g0 + static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; g < g1; g += stride) {
+        const int64_t i = ragged_stream(po, n_streams, g);
+        int64_t n;
+        if (!ragged_ok(so, po, i, L, &n))
+            continue;
+        const int64_t s = g - __ldg(&po[i]);
+        if (s < 0 || s * L >= n)
+            continue;                       // a slot past the stream's last span
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+        const double2 p = encode_span(sym + __ldg(&so[i]) + s * L, m, sV, N, r, 0.0, 0.0);
+        if (isnan(p.x))
+            atomicOr(status, FKV_ST_CORRUPT);
+        pts[g] = p;
+    }
+}
+
+template <typename Sym>
+__global__ void __launch_bounds__(dec_threads<Sym>())
+k_span_decode_ragged(const double2 *__restrict__ pts, const int64_t *__restrict__ po, int64_t n_streams,
+                     Sym *__restrict__ sym, const int64_t *__restrict__ so, const fkv_decconst *__restrict__ dc,
+                     const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    __syncthreads();
+    ragged_check(so, po, n_streams, L, status);
+    const int64_t g0 = __ldg(&po[0]), g1 = __ldg(&po[n_streams]);
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t g = g0 + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < g1; g += stride) {
+        const int64_t i = ragged_stream(po, n_streams, g);
+        int64_t n;
+        if (!ragged_ok(so, po, i, L, &n))
+            continue;
+        const int64_t s = g - __ldg(&po[i]);
+        if (s < 0 || s * L >= n)
+            continue;
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - s * L));
+        const double2 p = pts[g];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        Sym *dst = sym + __ldg(&so[i]) + s * L;
+        fkvdec::walk(t, X, Y, m, [&](int j, int c) { dst[m - 1 - j] = static_cast<Sym>(c); });
+        const long long lim = __ldg(&dc->alim[m]);
+        if (X > lim || X < -lim || Y > lim || Y < -lim)
+            atomicOr(status, FKV_ST_CORRUPT);
+    }
+}
+
+// Random access into a ragged batch: request q = (stream, position), the
+// position checked against that stream's own length.
+template <typename Sym>
+__global__ void __launch_bounds__(dec_threads<Sym>())
+k_read_ragged(const double2 *__restrict__ pts, const int64_t *__restrict__ po, const int64_t *__restrict__ so,
+              int64_t n_streams, const int64_t *__restrict__ req, int64_t n_req, Sym *__restrict__ out,
+              const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L, unsigned *status)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
+    __syncthreads();
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < n_req; q += stride) {
+        const int64_t st = req[2 * q], pos = req[2 * q + 1];
+        int64_t n = 0;
+        if (st < 0 || st >= n_streams || !ragged_ok(so, po, st, L, &n) || pos < 0 || pos >= n) {
+            out[q] = static_cast<Sym>(~0u);
+            atomicOr(status, FKV_ST_RANGE);
+            continue;
+        }
+        const int64_t u = pos / L;
+        const int o = static_cast<int>(pos - u * L);
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+        const double2 p = pts[__ldg(&po[st]) + u];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        int c = 0;
+        fkvdec::walk(t, X, Y, m - o, [&](int, int cc) { c = cc; });
+        out[q] = static_cast<Sym>(c);
+    }
 }
 
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -673,7 +812,7 @@ k_lossy_read(const LossyArgs a, int64_t n_streams, int64_t n, const int64_t *__r
         const int64_t st = req[2 * q], pos = req[2 * q + 1];
         if (st < 0 || st >= n_streams || pos < 0 || pos >= n) {
             out[q] = static_cast<Sym>(~0u);
-            atomicOr(status, FKV_ST_CORRUPT);
+            atomicOr(status, FKV_ST_RANGE);
             continue;
         }
         const int64_t u = pos / L;
@@ -1036,3 +1175,158 @@ cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t c
     return lossy_read_t(c, a, n_streams, n, req, n_req, static_cast<uint8_t *>(out), st);
 }
 
+
+// ------------------------------------------------------------ ragged launches
+namespace {
+
+// Persistent grid for the ragged kernels: the slot count lives on the device,
+// so the grid is sized to fill the GPU and the kernels stride over the slots.
+template <typename Sym>
+cudaError_t ragged_decoder_grid(const fkv_ctx *c, const void *kern, int smem, unsigned *grid)
+{
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess)
+        return e;
+    return decode_grid(c, kern, smem, 1ll << 40, grid, dec_threads<Sym>());
+}
+
+template <typename Sym>
+cudaError_t encode_ragged_t(const fkv_ctx *c, const Sym *sym, const int64_t *so, int64_t n_streams, double *pts,
+                            const int64_t *po, cudaStream_t st)
+{
+    unsigned grid = 0;
+    cudaError_t e = decode_grid(c, reinterpret_cast<const void *>(k_span_encode_ragged<Sym>), 0, 1ll << 40, &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_span_encode_ragged<Sym><<<grid, kThreads, 0, st>>>(sym, so, n_streams, reinterpret_cast<double2 *>(pts), po,
+                                                         c->d_V, c->N, c->r, c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+template <typename Sym>
+cudaError_t decode_ragged_t(const fkv_ctx *c, const double *pts, const int64_t *po, int64_t n_streams, Sym *sym,
+                            const int64_t *so, cudaStream_t st)
+{
+    const int smem = tables_bytes(c->N, c->L);
+    unsigned grid = 0;
+    cudaError_t e = ragged_decoder_grid<Sym>(c, reinterpret_cast<const void *>(k_span_decode_ragged<Sym>), smem,
+                                             &grid);
+    if (e != cudaSuccess)
+        return e;
+    k_span_decode_ragged<Sym><<<grid, dec_threads<Sym>(), smem, st>>>(reinterpret_cast<const double2 *>(pts), po,
+                                                                      n_streams, sym, so, c->d_dec, c->d_T, c->N,
+                                                                      c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+template <typename Sym>
+cudaError_t read_ragged_t(const fkv_ctx *c, const double *pts, const int64_t *po, const int64_t *so,
+                          int64_t n_streams, const int64_t *req, int64_t n_req, Sym *out, cudaStream_t st)
+{
+    const int smem = tables_bytes(c->N, c->L);
+    unsigned grid = 0;
+    cudaError_t e = ragged_decoder_grid<Sym>(c, reinterpret_cast<const void *>(k_read_ragged<Sym>), smem, &grid);
+    if (e != cudaSuccess)
+        return e;
+    const int64_t need = cdiv(n_req, dec_threads<Sym>());
+    if (static_cast<int64_t>(grid) > need)
+        grid = static_cast<unsigned>(need);
+    k_read_ragged<Sym><<<grid, dec_threads<Sym>(), smem, st>>>(reinterpret_cast<const double2 *>(pts), po, so,
+                                                               n_streams, req, n_req, out, c->d_dec, c->d_T, c->N,
+                                                               c->L, c->d_status);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_span_encode_ragged(const fkv_ctx *c, const void *sym, const int64_t *so, int64_t n_streams,
+                                      double *pts, const int64_t *po, cudaStream_t st)
+{
+    if (wide(c))
+        return encode_ragged_t(c, static_cast<const uint16_t *>(sym), so, n_streams, pts, po, st);
+    return encode_ragged_t(c, static_cast<const uint8_t *>(sym), so, n_streams, pts, po, st);
+}
+
+cudaError_t launch_span_decode_ragged(const fkv_ctx *c, const double *pts, const int64_t *po, int64_t n_streams,
+                                      void *sym, const int64_t *so, cudaStream_t st)
+{
+    if (wide(c))
+        return decode_ragged_t(c, pts, po, n_streams, static_cast<uint16_t *>(sym), so, st);
+    return decode_ragged_t(c, pts, po, n_streams, static_cast<uint8_t *>(sym), so, st);
+}
+
+cudaError_t launch_read_ragged(const fkv_ctx *c, const double *pts, const int64_t *po, const int64_t *so,
+                               int64_t n_streams, const int64_t *req, int64_t n_req, void *out, cudaStream_t st)
+{
+    if (wide(c))
+        return read_ragged_t(c, pts, po, so, n_streams, req, n_req, static_cast<uint16_t *>(out), st);
+    return read_ragged_t(c, pts, po, so, n_streams, req, n_req, static_cast<uint8_t *>(out), st);
+}
+
+// ------------------------------------------------------------ FP64 probe
+// Binary64 add/mul throughput with independent chains: every thread runs
+// kChains chains of x <- x * a, x <- x + b (round to nearest, no FMA: the
+// encoder's operation mix), whose fixed point b / (1 - a) keeps the values
+// bounded.  The chains' sum is written only when it equals an impossible
+// value, so the work stays live without a store per thread.
+namespace {
+constexpr int kFp64Chains = 8;
+__device__ double g_fp64_sink;
+
+__global__ void __launch_bounds__(256) k_fp64_rate(int iters, double a, double b)
+{
+    double x[kFp64Chains];
+#pragma unroll
+    for (int i = 0; i < kFp64Chains; ++i)
+        x[i] = 1.0 + 1e-3 * i + 1e-7 * threadIdx.x;
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int i = 0; i < kFp64Chains; ++i) {
+            x[i] = __dmul_rn(x[i], a);
+            x[i] = __dadd_rn(x[i], b);
+        }
+    }
+    double s = 0.0;
+#pragma unroll
+    for (int i = 0; i < kFp64Chains; ++i)
+        s += x[i];
+    if (s == -1.0)
+        g_fp64_sink = s;
+}
+}  // namespace
+
+cudaError_t measure_fp64_rate(int device, cudaStream_t st, double *ops_per_s)
+{
+    int sms = 0;
+    cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess)
+        return e;
+    const int blocks = sms * 4, iters = 4096;
+    cudaEvent_t t0, t1;
+    if ((e = cudaEventCreate(&t0)) != cudaSuccess)
+        return e;
+    if ((e = cudaEventCreate(&t1)) != cudaSuccess) {
+        cudaEventDestroy(t0);
+        return e;
+    }
+    float best = 0.0f;
+    for (int rep = 0; rep < 4 && e == cudaSuccess; ++rep) {   // the first launch warms up
+        cudaEventRecord(t0, st);
+        k_fp64_rate<<<blocks, 256, 0, st>>>(iters, 0.99999999, 1e-8);
+        cudaEventRecord(t1, st);
+        e = cudaGetLastError();
+        if (e == cudaSuccess)
+            e = cudaEventSynchronize(t1);
+        float ms = 0.0f;
+        if (e == cudaSuccess)
+            e = cudaEventElapsedTime(&ms, t0, t1);
+        if (e == cudaSuccess && rep > 0 && (best == 0.0f || ms < best))
+            best = ms;
+    }
+    cudaEventDestroy(t0);
+    cudaEventDestroy(t1);
+    if (e != cudaSuccess)
+        return e;
+    *ops_per_s = 2.0 * kFp64Chains * static_cast<double>(iters) * blocks * 256 / (best * 1e-3);
+    return cudaSuccess;
+}

@@ -13,55 +13,43 @@
 //
 // The array lives for the life of the process on every GPU that loads this
 // library and holds kStaticScratchBytes (16 MiB) of decoded symbols: at most
-// batch * n_layers * n_rec * R bytes per call (R = fkv_record_len).  Every
+// batch * n_layers * n_rec * R bytes per call (R = fkv_record_len).  It is
+// taken from device memory when fkv_create first looks up its address on a
+// device (static_scratch_resolve below), not by this entry point.  Every
 // call shares it, so calls whose kernels overlap on the GPU (different
 // streams without ordering) race on it and must be serialised by the caller.
 // It keeps whatever the previous call left; nothing here needs it zeroed,
 // because the decode kernel overwrites every byte the gather then reads.
-#include <mutex>
-
 #include "fkv_internal.h"
 
 namespace {
 
 constexpr size_t kStaticScratchBytes = 16u << 20;
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) uint8_t g_static_scratch[kStaticScratchBytes];
 
-std::mutex g_lock;
-void *g_scratch_addr[kMaxDevices] = {};
+}  // namespace
 
-// Device address of g_static_scratch on the current device (looked up once
-// per device with that device current).  In host code the symbol itself is a
-// host-side stand-in and must never be handed to a kernel.
-int scratch_address(fkv_ctx *ctx, uint8_t **out)
+// Called by fkv_create with the context's device current.  In host code the
+// symbol g_static_scratch is a host-side stand-in and must never be handed to
+// a kernel; its device address comes from cudaGetSymbolAddress.  Under lazy
+// module loading that first lookup is what loads this file's module and
+// takes the 16 MiB array from device memory, so it happens here, inside the
+// (synchronous, allocating) context creation, and never inside
+// fkv_decode_kv_static.  The address is kept in the context, whose lifetime
+// ends before any reset of the device could invalidate it.
+int static_scratch_resolve(fkv_ctx *ctx)
 {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) {
-        ctx->err = std::string("static scratch: cudaGetDevice: ") + cudaGetErrorString(e);
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess || !p) {
+        ctx->err = std::string("static scratch: cudaGetSymbolAddress: ") + cudaGetErrorString(e);
         return FKV_ECUDA;
     }
-    if (dev < 0 || dev >= kMaxDevices) {
-        ctx->err = "static scratch: device index out of range";
-        return FKV_EINVAL;
-    }
-    std::lock_guard<std::mutex> g(g_lock);
-    if (!g_scratch_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_scratch);
-        if (e != cudaSuccess || !p) {
-            ctx->err = std::string("static scratch: cudaGetSymbolAddress: ") + cudaGetErrorString(e);
-            return FKV_ECUDA;
-        }
-        g_scratch_addr[dev] = p;
-    }
-    *out = static_cast<uint8_t *>(g_scratch_addr[dev]);
+    ctx->static_scratch = static_cast<uint8_t *>(p);
+    ctx->static_scratch_bytes = kStaticScratchBytes;
     return FKV_OK;
 }
-
-}  // namespace
 
 extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t n_rec, int64_t pt_stride,
                                     fkv_cache *k_out, fkv_cache *v_out, int64_t t0, void *stream)
@@ -86,7 +74,7 @@ extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t
     const int64_t R = fkv_record_len(ctx);
     const int64_t n_streams = ref->batch * ctx->Ly;
     const int64_t n = n_rec * R;
-    if (n_streams <= 0 || n > static_cast<int64_t>(kStaticScratchBytes) / fkv_symbol_bytes(ctx) / n_streams) {
+    if (n_streams <= 0 || n > static_cast<int64_t>(ctx->static_scratch_bytes) / fkv_symbol_bytes(ctx) / n_streams) {
         ctx->err = "fkv_decode_kv_static: batch * n_layers * n_rec * record_len symbols exceed the 16 MiB static "
                    "scratch; decode fewer sequences per call";
         return FKV_EINVAL;
@@ -104,10 +92,11 @@ extern "C" int fkv_decode_kv_static(fkv_ctx *ctx, const double *pts_dev, int64_t
         ctx->err = "bad output cache view";
         return FKV_EINVAL;
     }
-    uint8_t *scratch = nullptr;
-    int rc = scratch_address(ctx, &scratch);
-    if (rc != FKV_OK)
-        return rc;
+    uint8_t *scratch = ctx->static_scratch;
+    if (!scratch) {
+        ctx->err = "fkv_decode_kv_static: the context has no static scratch address";
+        return FKV_ECUDA;
+    }
     // the same planar decode and gathers as fkv_decode_kv, through the static scratch
     return decode_archive(ctx, pts_dev, n_streams, n_rec, pt_stride, scratch, k_out, v_out, t0,
                           static_cast<cudaStream_t>(stream));

@@ -369,6 +369,11 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
     CK(cudaMemset(ctx->d_status, 0, sizeof(unsigned)), "status init");
 
     if (cb) {
+        // the allocation-free archive read's fixed scratch: its address is
+        // looked up here, so that call itself never loads a module
+        const int src = static_scratch_resolve(ctx);
+        if (src != FKV_OK)
+            return bail(src);
         const int K = cb->codewords == 0 ? 256 : cb->codewords;
         const int smax = K == 256 ? 8 : 2;
         if (N != K || (K != 256 && K != 1024) || (cb->pooled != 0 && cb->pooled != 1) || cb->n_layers < 1 ||
@@ -454,6 +459,8 @@ int fkv_sync_status(fkv_ctx *ctx, void *stream)
         return fail(ctx, FKV_ETIMEOUT, "a device wait timed out");
     if (st & FKV_ST_CORRUPT)
         return fail(ctx, FKV_ECORRUPT, "corrupt point or symbol (anchor check failed)");
+    if (st & FKV_ST_RANGE)
+        return fail(ctx, FKV_ERANGE, "a request named a position or stream outside the archive");
     return FKV_OK;
 }
 
@@ -513,6 +520,75 @@ int fkv_read(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n, 
         return fail(ctx, FKV_EINVAL, "misaligned buffer");
     CK(launch_read(ctx, pts_dev, n_streams, n, pt_stride, req_dev, n_req, out_dev, as_stream(stream)),
        "read launch");
+    return FKV_OK;
+}
+
+namespace {
+
+// Host checks shared by the ragged calls (the offsets themselves live on the
+// device and are checked there).
+const char *check_ragged(const fkv_ctx *ctx, const void *sym, const int64_t *so, int64_t n_streams,
+                         const double *pts, const int64_t *po)
+{
+    if (n_streams < 0)
+        return "negative stream count";
+    if (!so || !po || (n_streams > 0 && (!sym || !pts)))
+        return "null pointer";
+    if (reinterpret_cast<uintptr_t>(so) % 8 || reinterpret_cast<uintptr_t>(po) % 8)
+        return "offset arrays must be 8-byte aligned";
+    if (reinterpret_cast<uintptr_t>(pts) % 16)
+        return "points must be 16-byte aligned";
+    if (reinterpret_cast<uintptr_t>(sym) % sym_size(ctx))
+        return "uint16 symbols must be 2-byte aligned";
+    return nullptr;
+}
+
+}  // namespace
+
+int fkv_span_encode_ragged(fkv_ctx *ctx, const void *sym_dev, const int64_t *sym_off_dev, int64_t n_streams,
+                           double *pts_dev, const int64_t *pt_off_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (const char *why = check_ragged(ctx, sym_dev, sym_off_dev, n_streams, pts_dev, pt_off_dev))
+        return fail(ctx, FKV_EINVAL, why);
+    if (n_streams == 0)
+        return FKV_OK;
+    CK(launch_span_encode_ragged(ctx, sym_dev, sym_off_dev, n_streams, pts_dev, pt_off_dev, as_stream(stream)),
+       "ragged span encode launch");
+    return FKV_OK;
+}
+
+int fkv_span_decode_ragged(fkv_ctx *ctx, const double *pts_dev, const int64_t *pt_off_dev, int64_t n_streams,
+                           void *sym_dev, const int64_t *sym_off_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (const char *why = check_ragged(ctx, sym_dev, sym_off_dev, n_streams, pts_dev, pt_off_dev))
+        return fail(ctx, FKV_EINVAL, why);
+    if (n_streams == 0)
+        return FKV_OK;
+    CK(launch_span_decode_ragged(ctx, pts_dev, pt_off_dev, n_streams, sym_dev, sym_off_dev, as_stream(stream)),
+       "ragged span decode launch");
+    return FKV_OK;
+}
+
+int fkv_read_ragged(fkv_ctx *ctx, const double *pts_dev, const int64_t *pt_off_dev, const int64_t *sym_off_dev,
+                    int64_t n_streams, const int64_t *req_dev, int64_t n_req, void *out_dev, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (n_req < 0)
+        return fail(ctx, FKV_EINVAL, "negative size");
+    if (n_req == 0)
+        return FKV_OK;
+    if (const char *why = check_ragged(ctx, out_dev, sym_off_dev, n_streams, pts_dev, pt_off_dev))
+        return fail(ctx, FKV_EINVAL, why);
+    if (!req_dev || !out_dev || reinterpret_cast<uintptr_t>(req_dev) % 8)
+        return fail(ctx, FKV_EINVAL, "bad request buffer");
+    CK(launch_read_ragged(ctx, pts_dev, pt_off_dev, sym_off_dev, n_streams, req_dev, n_req, out_dev,
+                          as_stream(stream)),
+       "ragged read launch");
     return FKV_OK;
 }
 
@@ -652,6 +728,17 @@ int fkv_ac_decode(fkv_ctx *ctx, const uint32_t *words_dev, int64_t word_stride, 
                         as_stream(stream)),
        "arithmetic decode launch");
     return FKV_OK;
+}
+
+int fkv_measure_fp64_rate(double *ops_per_s, void *stream)
+{
+    if (!ops_per_s)
+        return FKV_EINVAL;
+    *ops_per_s = 0.0;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return FKV_ECUDA;
+    return measure_fp64_rate(dev, as_stream(stream), ops_per_s) == cudaSuccess ? FKV_OK : FKV_ECUDA;
 }
 
 int fkv_record_len(const fkv_ctx *ctx)
@@ -885,11 +972,17 @@ int fkv_append(fkv_ctx *ctx, fkv_streams *s, const void *sym_dev, int64_t m, int
         double *np = nullptr;
         CK(cudaMalloc(&np, static_cast<size_t>(s->n_streams) * cap * 16), "stream grow");
         const int64_t used = (s->length + ctx->L - 1) / ctx->L;
+        cudaError_t e = cudaSuccess;
         if (used > 0)
-            CK(cudaMemcpy2DAsync(np, cap * 16, s->d_pts, s->cap_spans * 16, used * 16, s->n_streams,
-                                 cudaMemcpyDeviceToDevice, as_stream(stream)),
-               "stream grow copy");
-        CK(cudaStreamSynchronize(as_stream(stream)), "stream grow sync");
+            e = cudaMemcpy2DAsync(np, cap * 16, s->d_pts, s->cap_spans * 16, used * 16, s->n_streams,
+                                  cudaMemcpyDeviceToDevice, as_stream(stream));
+        if (e == cudaSuccess)
+            e = cudaStreamSynchronize(as_stream(stream));
+        if (e != cudaSuccess) {
+            // the set keeps its old buffer; the new one is given back
+            cudaFree(np);
+            return cuda_fail(ctx, e, "stream grow copy");
+        }
         cudaFree(s->d_pts);
         s->d_pts = np;
         s->cap_spans = cap;

@@ -14,6 +14,7 @@
 // Device status bits (ctx->d_status); mapped to FKV_E* by fkv_sync_status.
 #define FKV_ST_CORRUPT 1u
 #define FKV_ST_TIMEOUT 2u
+#define FKV_ST_RANGE 4u      // a request named a position or stream outside the archive
 
 // Codebook-side constants of one K-or-V half of the archive.  G codebook
 // groups (G = Ly * H per-head, Ly pooled), K = ctx->KC codewords per stage.
@@ -56,6 +57,10 @@ struct fkv_ctx {
     fkv_cbset cb[2];
     uint8_t *d_scratch = nullptr;
     size_t scratch_bytes = 0;
+    // device address and size of the library's fixed scratch array on this
+    // context's device (decode_static.cu), looked up once by fkv_create
+    uint8_t *static_scratch = nullptr;
+    size_t static_scratch_bytes = 0;
     std::string err;
 };
 
@@ -82,6 +87,14 @@ cudaError_t launch_span_decode(const fkv_ctx *c, const double *pts, int64_t n_st
 cudaError_t launch_read(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
                         int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
                         cudaStream_t st);
+// Ragged batches: stream i's symbols at sym + so[i], len_i = so[i+1] - so[i];
+// its points in slots [po[i], po[i+1]) of pts (device offset arrays).
+cudaError_t launch_span_encode_ragged(const fkv_ctx *c, const void *sym, const int64_t *so, int64_t n_streams,
+                                      double *pts, const int64_t *po, cudaStream_t st);
+cudaError_t launch_span_decode_ragged(const fkv_ctx *c, const double *pts, const int64_t *po, int64_t n_streams,
+                                      void *sym, const int64_t *so, cudaStream_t st);
+cudaError_t launch_read_ragged(const fkv_ctx *c, const double *pts, const int64_t *po, const int64_t *so,
+                               int64_t n_streams, const int64_t *req, int64_t n_req, void *out, cudaStream_t st);
 cudaError_t launch_suffix_search(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n,
                                  int64_t pt_stride, const uint16_t *query, int qlen, int64_t *out, int64_t cap,
                                  int64_t *counts, cudaStream_t st);
@@ -99,6 +112,9 @@ cudaError_t launch_lossy_decode(const fkv_ctx *c, const uint32_t *codes, int64_t
 cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t code_stride, const double *tail,
                               int64_t tail_stride, int64_t n_streams, int64_t n, int bits, int64_t keep_exact,
                               const int64_t *req, int64_t n_req, void *out, cudaStream_t st);
+// Binary64 add/mul instructions per second of the current device, measured
+// by independent chains (the span encoder's roofline denominator).
+cudaError_t measure_fp64_rate(int device, cudaStream_t st, double *ops_per_s);
 // ac.cu (Sec. 6 probability-weighted maps): words that always hold the code
 // of n symbols, and the warp-per-stream coder
 int64_t ac_capacity_words(int N, int64_t n);
@@ -122,6 +138,9 @@ cudaError_t launch_span_decode_planar(const fkv_ctx *c, const double *pts, int64
 bool check_outputs(const fkv_ctx *ctx, const fkv_cache *k_out, const fkv_cache *v_out, int64_t n_rec, int64_t t0);
 int decode_archive(fkv_ctx *ctx, const double *pts, int64_t n_streams, int64_t n_rec, int64_t pt_stride,
                    void *scratch, const fkv_cache *k_out, const fkv_cache *v_out, int64_t t0, cudaStream_t st);
+// decode_static.cu: look up the fixed scratch array's device address for the
+// current device (context creation only)
+int static_scratch_resolve(fkv_ctx *ctx);
 // gather.cu
 cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st);

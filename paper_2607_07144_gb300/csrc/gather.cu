@@ -318,7 +318,7 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
         for (int64_t i = lane; i < out_vec / 2; i += 32)
             store2(a.out, a.dtype, q * out_vec + 2 * i, 0.0f, 0.0f);
         if (lane == 0)
-            atomicOr(a.status, FKV_ST_CORRUPT);
+            atomicOr(a.status, FKV_ST_RANGE);
         return;
     }
     const int64_t n = a.n_rec * R;

@@ -6,6 +6,7 @@ import pytest
 import torch
 
 import synth
+from oracle import parity
 
 pytestmark = pytest.mark.gpu
 TORCH_DT = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}
@@ -57,10 +58,11 @@ def test_archive_round_trip(fkv, oracle_mod, base, cid):
     for (b, l) in [(0, 0), (cfg.batch - 1, cfg.n_layers - 1)]:
         ik, iv = oracle_mod.indices_from_records(sh[b, l], cfg.n_heads, cfg.stages_k, cfg.stages_v)
         for h in range(cfg.n_heads):
-            yk = oracle_mod.round_to(oracle_mod.rvq_decode(ik[h], cbk[l, h]), cfg.dtype)
-            got = Kr[l, b, h, cfg.t0:cfg.t1].float().cpu().numpy().astype(np.float64)
-            assert np.mean(got == yk) > 0.999
-            assert np.max(np.abs(got - yk)) <= np.max(np.abs(yk)) * 2 ** -7
+            for out, idx, cb in ((Kr, ik, cbk), (Vr, iv, cbv)):
+                got = out[l, b, h, cfg.t0:cfg.t1].float().cpu().numpy().astype(np.float64)
+                hard, _, _ = parity.rounded_mismatches(got, oracle_mod.rvq_decode(idx[h], cb[l, h]), cfg.dtype,
+                                                       oracle_mod.rvq_decode(idx[h], np.abs(cb[l, h])))
+                assert hard == 0
     # random record reads equal the full decode
     n_req = 3000
     rng = np.random.default_rng(cid)

@@ -164,7 +164,7 @@ def test_random_read_equals_full_decode(fkv, oracle_mod, N):
     assert np.array_equal(got[sel], oracle_mod.read(pts[2].cpu().numpy(), n, req[sel, 1], N, ctx.r, ctx.L))
     bad = torch.tensor([[0, n], [ns, 0], [-1, 0]], dtype=torch.int64, device="cuda")
     out = ctx.read(pts, n, bad).cpu().numpy()
-    assert np.all(out.view(np.uint16) == 0xFFFF) and ctx.sync_status() == -5
+    assert np.all(out.view(np.uint16) == 0xFFFF) and ctx.sync_status() == -2   # FKV_ERANGE
 
 
 @pytest.mark.parametrize("N", [257, 1024])

@@ -110,7 +110,7 @@ def test_strided_buffers_and_reads(fkv, oracle_mod):
     assert torch.equal(got, full[torch.from_numpy(req[:, 0]).cuda(), torch.from_numpy(req[:, 1]).cuda()])
     bad = torch.tensor([[0, n], [ns, 0], [-1, 3]], dtype=torch.int64, device="cuda")
     out = ctx.lossy_read(codes[:, :words + 5], tail[:, :ts + 1], n, bits, keep, bad).cpu().numpy()
-    assert np.all(out == 0xFF) and ctx.sync_status() == -5
+    assert np.all(out == 0xFF) and ctx.sync_status() == -2     # FKV_ERANGE
 
 
 def test_bad_arguments_are_rejected(fkv):

@@ -28,17 +28,8 @@ def fkv():
 
 def compare_rvq(gpu, ora, gap):
     """-> (hard mismatches, near-tie mismatches, compared entries)."""
-    n, S = ora.shape
-    prefix = np.ones(n, bool)
-    hard = near = seen = 0
-    for s in range(S):
-        diff = (gpu[:, s] != ora[:, s]) & prefix
-        h = diff & (gap[:, s] > GAP)
-        hard += int(h.sum())
-        near += int((diff & ~h).sum())
-        seen += int(prefix.sum())
-        prefix &= ~diff
-    return hard, near, seen
+    from oracle import parity
+    return parity.compare_rvq(gpu, ora, gap, GAP)
 
 
 def host_cache(cfg, kv):
@@ -120,20 +111,10 @@ def _check_rounded(got, ref64, dtype, absum):
     float64 sum rounded to nearest-even, except where the float32 summation
     error bound (4 * 2^-24 * sum |c_s|, plus 1e-6 relative) straddles a
     rounding boundary.  Returns the number of such borderline differences."""
-    want = synth_round(ref64, dtype)
-    ok = got == want
-    if ok.all():
-        return 0
-    eps = 4 * 2.0 ** -24 * absum + 1e-6 * np.abs(ref64)
-    borderline = synth_round(ref64 - eps, dtype) != synth_round(ref64 + eps, dtype)
-    bad = ~(ok | borderline)
-    assert not bad.any(), (int(bad.sum()), got[bad][:5], ref64[bad][:5])
-    return int((~ok).sum())
-
-
-def synth_round(y, dtype):
-    import oracle
-    return oracle.round_to(y, dtype)
+    from oracle import parity
+    hard, border, _ = parity.rounded_mismatches(got, ref64, dtype, absum)
+    assert hard == 0, hard
+    return border
 
 
 def test_small_gpt2_fp16_full(fkv, oracle_mod):
@@ -160,12 +141,16 @@ def test_small_llama_bf16_d128(fkv, oracle_mod):
     ctx, sym, gi, K64, V64, cbk, cbv = check_config_full(fkv, oracle_mod, cfg)
     P = cfg.n_archived
     Kr = torch.zeros(cfg.cache_shape(), dtype=torch.bfloat16, device="cuda")
-    ctx.rvq_decode(sym, P, Kr, None, t0=cfg.t0)
+    Vr = torch.zeros(cfg.cache_shape(), dtype=torch.bfloat16, device="cuda")
+    ctx.rvq_decode(sym, P, Kr, Vr, t0=cfg.t0)
     Kr = Kr.float().cpu().numpy().astype(np.float64)
+    Vr = Vr.float().cpu().numpy().astype(np.float64)
     for (b, l), (ik, iv) in gi.items():
         for h in range(cfg.n_heads):
             _check_rounded(Kr[l, b, h, cfg.t0:cfg.t1], oracle_mod.rvq_decode(ik[h], cbk[l, h]), "bf16",
                            oracle_mod.rvq_decode(ik[h], np.abs(cbk[l, h])))
+            _check_rounded(Vr[l, b, h, cfg.t0:cfg.t1], oracle_mod.rvq_decode(iv[h], cbv[l, h]), "bf16",
+                           oracle_mod.rvq_decode(iv[h], np.abs(cbv[l, h])))
 
 
 def _one_group_cfg(dim, dtype, seq):

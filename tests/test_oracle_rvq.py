@@ -143,3 +143,59 @@ def test_round_to_nearest_even(oracle_mod):
     assert np.array_equal(oracle_mod.round_to(x64, "f16"),
                           torch.from_numpy(x64).to(torch.float16).to(torch.float64).numpy())
     assert oracle_mod.round_to(np.array([1 + 2.0 ** -11]), "f16")[0] == 1.0
+
+
+def _bruteforce_gap(x, cb):
+    """Per stage: (second-best - best squared distance) / ||stage residual||^2,
+    from a numpy float64 search that keeps its own residual."""
+    res = np.asarray(x, np.float64).copy()
+    gaps = []
+    for C in np.asarray(cb, np.float64):
+        d = ((res[:, None, :] - C[None, :, :]) ** 2).sum(-1)
+        part = np.partition(d, 1, axis=1)
+        rn = (res * res).sum(1)
+        gaps.append((part[:, 1] - part[:, 0]) / rn)
+        res -= C[d.argmin(axis=1)]
+    return np.stack(gaps, axis=1)
+
+
+@pytest.mark.parametrize("D,S,K", [(8, 1, 256), (16, 3, 256), (64, 4, 256), (128, 2, 256), (64, 1, 1024),
+                                   (64, 2, 1024)])
+def test_gap_matches_bruteforce(oracle_mod, D, S, K):
+    # the quantity the GPU parity criterion excuses mismatches on: the top-2
+    # distance gap of each stage over that stage's residual norm
+    rng = np.random.default_rng(10 + D + S + K)
+    x = rng.normal(size=(150, D))
+    cb = (rng.normal(size=(S, K, D)) * 0.8 ** np.arange(S)[:, None, None]).astype(np.float32)
+    idx, gap = oracle_mod.rvq_encode(x, cb)
+    want = _bruteforce_gap(x, cb)
+    assert np.all(np.isfinite(gap))
+    np.testing.assert_allclose(gap, want, rtol=1e-9, atol=1e-12)
+
+
+def test_gap_is_normalised_by_the_stage_residual(oracle_mod):
+    # stage 2 residuals are ~1e-3 of the input, so a gap divided by ||x||^2
+    # (instead of the stage residual's norm) would be ~1e-6 of the right value
+    rng = np.random.default_rng(11)
+    c0 = (10.0 * rng.normal(size=(256, 32))).astype(np.float32)
+    c1 = (0.01 * rng.normal(size=(256, 32))).astype(np.float32)
+    a = rng.integers(0, 256, size=120)
+    x = c0[a].astype(np.float64) + 0.01 * rng.normal(size=(120, 32))
+    cb = np.stack([c0, c1])
+    idx, gap = oracle_mod.rvq_encode(x, cb)
+    want = _bruteforce_gap(x, cb)
+    assert np.all(idx[:, 0] == a)
+    np.testing.assert_allclose(gap, want, rtol=1e-9, atol=1e-12)
+    assert np.median(gap[:, 1]) > 1e-2          # O(1) gaps at the small second stage
+
+
+def test_gap_when_the_best_codeword_comes_first(oracle_mod):
+    # the winner at index 0 leaves the second-best to the later candidates
+    # only (the branch that tracks a runner-up below the current best)
+    rng = np.random.default_rng(12)
+    cb = rng.normal(size=(1, 256, 24)).astype(np.float32)
+    x = cb[0, 0].astype(np.float64)[None, :] + 1e-3 * rng.normal(size=(40, 24))
+    idx, gap = oracle_mod.rvq_encode(x, cb)
+    assert np.all(idx[:, 0] == 0)
+    np.testing.assert_allclose(gap, _bruteforce_gap(x, cb), rtol=1e-9, atol=1e-12)
+    assert np.all(np.isfinite(gap)) and np.all(gap > 0)

@@ -58,6 +58,27 @@ def test_static_scratch_decode_matches_allocating_decode(fkv):
         assert torch.all(Kb[:, :, :, :cfg.t0] == 7.0) and torch.all(Vb[:, :, :, cfg.t1:] == 7.0)
 
 
+def test_first_call_takes_no_device_memory(fkv):
+    # the fixed array's address is looked up when the context is created, so
+    # the first allocation-free decode on a context loads no module and takes
+    # no device memory (its kernels are the allocating decode's, loaded by
+    # that call first, together with its own scratch)
+    cfg = synth.small_config(synth.CFG1, 504, n_layers=2, batch=2, seq=36 + 100)
+    ctx = fkv.Context(256, codebooks=(synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)))
+    K, V, pts = _archive(fkv, ctx, cfg)
+    Ka, Va = torch.zeros_like(K), torch.zeros_like(V)
+    ctx.decode_kv(pts, cfg.n_archived, Ka, Va, t0=cfg.t0)
+    Kb, Vb = torch.zeros_like(K), torch.zeros_like(V)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    ctx.decode_kv_static(pts, cfg.n_archived, Kb, Vb, t0=cfg.t0)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert ctx.sync_status() == 0
+    assert free1 == free0
+    assert torch.equal(Kb, Ka) and torch.equal(Vb, Va)
+
+
 def test_static_scratch_rejects_oversized_archives(fkv):
     cfg = synth.small_config(synth.CFG1, 503, n_layers=12, batch=8, seq=1024)
     ctx = fkv.Context(256, codebooks=(synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)))
@@ -70,5 +91,21 @@ def test_static_scratch_rejects_oversized_archives(fkv):
         ctx.decode_kv_static(pts, n_rec, out, None, t0=0)
     assert ei.value.code == -1 and "16 MiB" in str(ei.value)
     assert torch.count_nonzero(out) == 0                               # nothing was launched
-    ctx.decode_kv_static(pts, n_rec - 1, out, None, t0=0)            # at the limit: accepted
-    torch.cuda.synchronize()
+
+
+def test_static_scratch_at_its_limit_matches_allocating_decode(fkv):
+    # a real archive exactly as large as the fixed array allows
+    base = synth.small_config(synth.CFG1, 505, n_layers=2, batch=2, seq=36, n_heads=4)
+    R = base.n_heads * (base.stages_k + base.stages_v)
+    n_rec = (16 << 20) // (base.batch * base.n_layers * R)
+    cfg = synth.small_config(synth.CFG1, 505, n_layers=2, batch=2, seq=36 + n_rec, n_heads=4)
+    assert cfg.n_archived == n_rec and cfg.batch * cfg.n_layers * n_rec * R <= 16 << 20
+    ctx = fkv.Context(256, codebooks=(synth.codebooks(cfg, 0), synth.codebooks(cfg, 1)))
+    K, V, pts = _archive(fkv, ctx, cfg)
+    Ka, Va = torch.zeros_like(K), torch.zeros_like(V)
+    ctx.decode_kv(pts, n_rec, Ka, Va, t0=cfg.t0)
+    Kb, Vb = torch.zeros_like(K), torch.zeros_like(V)
+    ctx.decode_kv_static(pts, n_rec, Kb, Vb, t0=cfg.t0)
+    assert ctx.sync_status() == 0
+    assert torch.equal(Kb, Ka) and torch.equal(Vb, Va)
+    assert torch.count_nonzero(Kb[:, :, :, cfg.t0:cfg.t1]) > 0
