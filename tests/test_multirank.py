@@ -50,7 +50,7 @@ def test_two_gloo_ranks_replicas_and_max_timing():
         p.join(timeout=60)
         assert p.exitcode == 0
     import synth
-    assert out[0][0] == synth.CFG1.cfg_id and out[1][0] == synth.CFG1.cfg_id + 1000
+    assert out[0][0] == synth.CFG3.cfg_id and out[1][0] == synth.CFG3.cfg_id + 1000
     assert out[0][1] != out[1][1]                          # each rank archives its own data
     for r in range(world):
         assert out[r][2] == [2.0, 10.0]                    # the job's time is the slowest rank's
