@@ -13,13 +13,25 @@
 // of T[j][c] = round((1-r) r^j V(c) 2^62), j = m - k, and two subtractions.
 //
 // Classification takes an fp32 fast path with a certified margin and falls
-// back to exact 64x64->128-bit dot products in the rare near-boundary case:
+// back to integer dot products in the rare near-boundary case: the high words
+// of the 64x64->128-bit products, each dropping less than 2^-60, so a
+// difference of two such dot products is off by less than 2^-59 (and by
+// 2^-61 more from the vertices' Q1.62 rounding).  The decision it makes is
+// the sign of Q . (V(a) - V(b)) for neighbouring vertices a, b, whose
+// magnitude for a point of the true cell is at least
+//     r^(m-1) (1 - cos(2 pi / N)) (1 - 2 r)
+// (the point after the span's first symbol, (1 - r) V(c), is the closest
+// case; a later point's own offset costs at most the factor 1 - 2 r).  With
+// span lengths up to 44 / log2(1/r), r^(m-1) >= 2^-44 / r, and r_N ~ pi / N,
+// that is at least about 2^-44 * 2 pi / N >= 2^-51.3 for every N <= 1024,
+// 2^7 above the error (at N = 1024, L = 5 the bound is 2^-49.1, and that
+// value is reached by alternating-neighbour spans):
 //   * N = 4: the vertices are the axis directions, exact integer compares;
 //   * N <= 8: fp32 scores q . V(c); exact scores when the best two are closer
 //     than a bound far above the fp32 error;
 //   * N > 8: Voronoi regions of the vertices are angular sectors, so the fp32
 //     angle picks the sector; within 1e-3 sector widths of a boundary the two
-//     neighbouring sectors are decided by the exact sign of Q . (V(a) - V(b)).
+//     neighbouring sectors are decided by the sign of Q . (V(a) - V(b)).
 #pragma once
 
 #include <climits>
@@ -60,6 +72,8 @@ __device__ inline Tables load(const fkv_decconst *__restrict__ g, const longlong
     return Tables{T, vx, vy, vf, N};
 }
 
+// Q . V(c) in units of 2^-60: the high words of the two 128-bit products
+// (the error bound is in the header comment).
 __device__ __forceinline__ long long exact_dot(const Tables &t, long long X, long long Y, int c)
 {
     return __mul64hi(X, t.vx[c]) + __mul64hi(Y, t.vy[c]);

@@ -70,8 +70,6 @@ void destroy_cbset(fkv_cbset &s)
     cudaFree(s.escale);
     cudaFree(s.escale_h);
     cudaFree(s.cbaug);
-    cudaFree(s.cbound);
-    cudaFree(s.cnorm);
     s = fkv_cbset();
 }
 
@@ -129,8 +127,6 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
     std::vector<int> es(static_cast<size_t>(G) * stages);
     std::vector<__half> c16(ncode * 2 * D);
     std::vector<__half> caug(ncode * 16, __float2half(0.0f));
-    std::vector<float4> cbound(static_cast<size_t>(G) * stages);
-    std::vector<float> cnorm(ncode);
     for (int gs = 0; gs < G * stages; ++gs) {
         const float *cb = host + static_cast<size_t>(gs) * K * D;
         float m = 0.0f;
@@ -154,24 +150,17 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         }
         es[gs] = e;
         const float mul = -2.0f;
-        double bmax = 0.0, blmax = 0.0, nmax = 0.0;
         for (int j = 0; j < K; ++j) {
-            double ns = 0.0, bh = 0.0, bl = 0.0;
+            double ns = 0.0;
             for (int d = 0; d < D; ++d) {
                 const double vs = ldexp(static_cast<double>(cb[j * D + d]), -e);
                 ns += vs * vs;
                 const float sv = mul * ldexpf(cb[j * D + d], -e);
                 const __half hi = __float2half_rn(sv);
                 const __half lo = __float2half_rn(sv - __half2float(hi));
-                bh += static_cast<double>(__half2float(hi)) * __half2float(hi);
-                bl += static_cast<double>(__half2float(lo)) * __half2float(lo);
                 c16[((static_cast<size_t>(gs) * 2 + 0) * K + j) * D + d] = hi;
                 c16[((static_cast<size_t>(gs) * 2 + 1) * K + j) * D + d] = lo;
             }
-            cnorm[static_cast<size_t>(gs) * K + j] = static_cast<float>(ns);
-            bmax = fmax(bmax, sqrt(bh));
-            blmax = fmax(blmax, sqrt(bl));
-            nmax = fmax(nmax, ns);
             // K rows in the core-matrix layout: 256-row blocks of 8 KB, back to back
             __half *blk = caug.data() + static_cast<size_t>(gs) * K * 16;
             __half parts[3];
@@ -181,10 +170,6 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
                 blk[core16_offset(j, k) / 2] = val;
             }
         }
-        // rounded up: the kernels' error bounds take these as upper bounds
-        const double up = 1.0 + 1e-6;
-        cbound[gs] = make_float4(static_cast<float>(bmax * up), static_cast<float>(blmax * up),
-                                 static_cast<float>(nmax * up), 0.0f);
     }
     CK(cudaMalloc(&s.cb32, ncode * D * sizeof(float)), "codebook alloc");
     CK(cudaMalloc(&s.cb16, ncode * 2 * D * sizeof(__half)), "codebook alloc");
@@ -202,10 +187,6 @@ int upload_cbset(fkv_ctx *ctx, int kv, const float *host, int stages)
         CK(cudaMalloc(&s.escale_h, eh.size() * sizeof(int)), "codebook alloc");
         CK(cudaMemcpy(s.escale_h, eh.data(), eh.size() * sizeof(int), cudaMemcpyHostToDevice), "codebook copy");
     }
-    CK(cudaMalloc(&s.cbound, cbound.size() * sizeof(float4)), "codebook alloc");
-    CK(cudaMemcpy(s.cbound, cbound.data(), cbound.size() * sizeof(float4), cudaMemcpyHostToDevice), "codebook copy");
-    CK(cudaMalloc(&s.cnorm, cnorm.size() * sizeof(float)), "codebook alloc");
-    CK(cudaMemcpy(s.cnorm, cnorm.data(), cnorm.size() * sizeof(float), cudaMemcpyHostToDevice), "codebook copy");
     CK(cudaMalloc(&s.cbaug, caug.size() * sizeof(__half)), "codebook alloc");
     CK(cudaMemcpy(s.cbaug, caug.data(), caug.size() * sizeof(__half), cudaMemcpyHostToDevice), "codebook copy");
     EncodeTiledFn enc = encode_tiled();

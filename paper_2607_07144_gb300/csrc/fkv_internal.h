@@ -28,11 +28,6 @@ struct fkv_cbset {
     // 64-dimensional heads only (rvq.cu k_rvq64): cb16 holds the hi/lo split of
     // -2 c 2^-e with max |c 2^-e| in [2^3, 2^9), and cbaug the norm operand.
     __half *cbaug = nullptr;  // [G][S] blocks of K x 16 fp16 in core-matrix layout (32 B per codeword)
-    // Single-pass certification (rvq.cu k_rvq128): per (group, stage) the
-    // largest norms of the hi and lo fp16 operands b = fp16(-2 c'),
-    // b_lo = fp16(-2 c' - b) and of ||c'||^2, and the exact squared norms.
-    float4 *cbound = nullptr; // [G][S] (max ||b_j||, max ||b_lo_j||, max ||c'_j||^2, 0), rounded up
-    float *cnorm = nullptr;   // [G][S][K] ||c'_j||^2
 };
 
 // Largest alphabet: symbols are uint8 up to N = 256 and uint16 above.
