@@ -83,9 +83,24 @@ def load_peaks():
 
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per RVQ launch of
-# the headline workload from an ncu capture of the current k_rvq128, or None
-# until the kernel as it stands has been captured.
-RVQ_DRAM_BYTES_PER_LAUNCH = None
+# the headline workload, from one ncu capture of the current k_rvq128 on the
+# same cache cut to 4096 archived positions (the full cache is too large for a
+# multi-metric capture): 1,257,913,600 B for the key launch and 1,176,856,576 B
+# for the value launch.  The hi/lo fp16 codebook operands (4 x 256 x 128 x 2 x
+# 2 B per key head, half that per value head) are read once whatever the
+# length; the rest grows with the positions.  The figure is the mean of the key
+# and value launches at the headline length.  Set it to None when k_rvq128
+# changes until it is captured again.
+def _rvq_traffic_full(slice_pos=4096, slice_bytes=((1257913600, 4), (1176856576, 2))):
+    groups = HEADLINE.n_layers * HEADLINE.n_heads
+    full = []
+    for total, stages in slice_bytes:
+        cb = groups * stages * 256 * HEADLINE.dim * 2 * 2
+        full.append((total - cb) * HEADLINE.n_archived / slice_pos + cb)
+    return sum(full) / len(full)
+
+
+RVQ_DRAM_BYTES_PER_LAUNCH = _rvq_traffic_full()
 
 # Nominal FP64 add/mul rate: GB300's 1.25 TFLOP/s of FP64 FMA is 625 G add or
 # mul instructions per second at the 2070 MHz boost clock (1.99 per clock per
@@ -965,7 +980,8 @@ def main():
     sm_mhz = res["clocks"].get("sm_mhz") or 2070.0
     rates = archive_rates(cfg, res["phase"], res["R"], res["P"], res["n_rec"], res["spans"], res["ns"], peaks,
                           res["fp64"])
-    dominant = roofline(rates, peaks, RVQ_DRAM_BYTES_PER_LAUNCH, "k_rvq128 (RVQ assignment, 128-dim heads)")
+    traffic = RVQ_DRAM_BYTES_PER_LAUNCH if args.seq == HEADLINE.seq else None
+    dominant = roofline(rates, peaks, traffic, "k_rvq128 (RVQ assignment, 128-dim heads)")
     kernels = {"rvq (tcgen05, k_rvq128)": rates["rvq"], "span_encode": rates["span_encode"],
                "decode_kv (decode + gather)": rates["decode_kv"]}
     kernels.update(secondary_report(res, peaks, res["fp64"], sm_mhz))

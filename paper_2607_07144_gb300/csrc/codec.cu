@@ -133,6 +133,56 @@ __host__ __device__ inline int tables_bytes(int N, int L)
     return (fkvdec::smem_bytes(N, L) + 15) & ~15;
 }
 
+// A persistent block's chunk (stream, span block), chunk = stream * bps +
+// block, stepped gridDim.x chunks at a time without a division per step: the
+// whole streams and remaining blocks of one step are worked out once.
+struct ChunkWalk {
+    int64_t stream, sb;
+    unsigned dq, dr, bps;
+    __device__ explicit ChunkWalk(int bps_) : bps(static_cast<unsigned>(bps_))
+    {
+        stream = blockIdx.x / bps;
+        sb = blockIdx.x - static_cast<unsigned>(stream) * bps;
+        dq = gridDim.x / bps;
+        dr = gridDim.x - dq * bps;
+    }
+    __device__ void next()
+    {
+        sb += dr;
+        stream += dq;
+        if (sb >= bps) {
+            sb -= bps;
+            ++stream;
+        }
+    }
+};
+
+// Unsigned 32-bit division by an invariant d >= 1 as a multiply-high, a
+// subtract, an add and two shifts (Granlund and Montgomery, "Division by
+// invariant integers using multiplication", PLDI 1994, Sec. 4): with l =
+// ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1, t = mulhi(m, q) and
+// q / d = (t + ((q - t) >> min(l, 1))) >> max(l - 1, 0) for every 32-bit q.
+struct FastDiv {
+    unsigned m;
+    int sh1, sh2;
+    __host__ static FastDiv make(unsigned d)
+    {
+        int l = 0;
+        while ((1ull << l) < d)
+            ++l;
+        FastDiv f;
+        f.m = static_cast<unsigned>((((1ull << l) - d) << 32) / d + 1);
+        f.sh1 = l < 1 ? l : 1;
+        f.sh2 = l - 1 > 0 ? l - 1 : 0;
+        return f;
+    }
+    __device__ __forceinline__ unsigned div(unsigned q) const
+    {
+        const unsigned t = __umulhi(m, q);
+        return (t + ((q - t) >> sh1)) >> sh2;
+    }
+};
+
 // Decode span s of `stream` (one per thread): the walk's symbols go through
 // `put(j, c)`, j = 0 .. m-1 from the span's last symbol back to its first,
 // straight from registers to their place; a point whose walk does not end at
@@ -166,14 +216,14 @@ k_span_decode(const double2 *__restrict__ pts, int64_t n, int64_t pt_stride, int
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
     __syncthreads();
     constexpr int TPB = dec_threads<Sym>();
-    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
-        const int64_t stream = ck / bps;
-        const int64_t s = (ck - stream * bps) * TPB + threadIdx.x;
+    ChunkWalk w(bps);
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x, w.next()) {
+        const int64_t s = w.sb * TPB + threadIdx.x;
         if (s >= spans)
             continue;
-        Sym *dst = sym + stream * sym_stride + s * L;
+        Sym *dst = sym + w.stream * sym_stride + s * L;
         int m = 0;
-        decode_span(t, pts, n, pt_stride, stream, s, dc, L, status,
+        decode_span(t, pts, n, pt_stride, w.stream, s, dc, L, status,
                     [&](int j, int c) { dst[m - 1 - j] = static_cast<Sym>(c); }, m);
     }
 }
@@ -215,9 +265,10 @@ k_span_decode_staged(const double2 *__restrict__ pts, int64_t n, int64_t pt_stri
     uint8_t *sbuf = dsm + tables_bytes(N, L);
     __syncthreads();
     constexpr int TPB = dec_threads<Sym>();
-    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
-        const int64_t stream = ck / bps;
-        const int64_t s0 = (ck - stream * bps) * TPB;
+    ChunkWalk w(bps);
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x, w.next()) {
+        const int64_t stream = w.stream;
+        const int64_t s0 = w.sb * TPB;
         const int64_t b = s0 * L;
         const int64_t e = min(n, (s0 + TPB) * L);
         uint8_t *dst = reinterpret_cast<uint8_t *>(sym + stream * sym_stride + b);
@@ -232,63 +283,61 @@ k_span_decode_staged(const double2 *__restrict__ pts, int64_t n, int64_t pt_stri
 // The same decode for a whole archive of token records, written out in the
 // planar layout the archive gather reads: per stream, the H key planes
 // (n_rec x S_K indices each, one plane per head) and then the H value planes
-// (n_rec x S_V).  A thread places each symbol of its span as the walk yields
-// it, last to first, stepping a (record, K or V, head, stage) position back
-// by one per symbol from the one of the span's last symbol (one division per
-// span).
+// (n_rec x S_V).  A block first tabulates, for each of the R symbols of a
+// record, its offset inside its record's first plane row; a thread then places
+// each symbol of its span as the walk yields it, last to first, at that
+// offset plus record x stages, stepping back one symbol of the record (and a
+// record at its start) per symbol.  Positions inside a stream are 32-bit (the
+// launcher keeps a stream below 2^31 symbols) and the span's last record comes
+// from a multiply-high division.
 template <typename Sym>
 __global__ void __launch_bounds__(dec_threads<Sym>())
-k_span_decode_planar(const double2 *__restrict__ pts, int64_t n_rec, int64_t pt_stride, int64_t spans, int bps,
-                     int64_t n_chunks, Sym *__restrict__ out, int H, int SK, int SV,
+k_span_decode_planar(const double2 *__restrict__ pts, unsigned n_rec, int64_t pt_stride, unsigned spans, int bps,
+                     unsigned n_chunks, Sym *__restrict__ out, int H, int SK, int SV, FastDiv div_r,
                      const fkv_decconst *__restrict__ dc, const longlong2 *__restrict__ T, int N, int L,
                      unsigned *status)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(dc, T, N, L, dsm);
-    __syncthreads();
     const int R = H * (SK + SV);
     const int nk = H * SK;
-    const int64_t n = n_rec * R;
-    const int64_t vplanes = static_cast<int64_t>(nk) * n_rec;     // offset of the value planes
+    const unsigned n = n_rec * static_cast<unsigned>(R);
     constexpr int TPB = dec_threads<Sym>();
-    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
-        const int64_t stream = ck / bps;
-        const int64_t s = (ck - stream * bps) * TPB + threadIdx.x;
+    // symbol o of a record: plane offset (K planes, then V planes) + stage
+    unsigned *poff = reinterpret_cast<unsigned *>(dsm + tables_bytes(N, L));
+    for (int o = threadIdx.x; o < R; o += TPB) {
+        const bool v = o >= nk;
+        const int S = v ? SV : SK, oo = v ? o - nk : o;
+        const int h = oo / S;
+        poff[o] = (v ? static_cast<unsigned>(nk) * n_rec : 0u) + static_cast<unsigned>(h) * n_rec * S + (oo - h * S);
+    }
+    __syncthreads();
+    const long long lim_full = __ldg(&dc->alim[L]);
+    ChunkWalk w(bps);
+    for (unsigned ck = blockIdx.x; ck < n_chunks; ck += gridDim.x, w.next()) {
+        const unsigned s = static_cast<unsigned>(w.sb) * TPB + threadIdx.x;
         if (s >= spans)
             continue;
-        Sym *base = out + stream * n;
-        // position of the span's last symbol
-        const int64_t q = min(s * L + L, n) - 1;
-        int64_t rec = q / R;
-        int o = static_cast<int>(q - rec * R);
-        int seg = o < nk ? 0 : 1;
-        if (seg)
-            o -= nk;
-        const int S0 = seg ? SV : SK;
-        int h = o / S0, st = o - h * S0;
-        int m = 0;
-        decode_span(t, pts, n, pt_stride, stream, s, dc, L, status,
-                    [&](int, int c) {
-                        const int Sg = seg ? SV : SK;
-                        base[(seg ? vplanes : 0) + static_cast<int64_t>(h) * n_rec * Sg + rec * Sg + st] =
-                            static_cast<Sym>(c);
-                        if (st > 0) {
-                            --st;
-                        } else if (h > 0) {
-                            --h;
-                            st = Sg - 1;
-                        } else if (seg) {
-                            seg = 0;
-                            h = H - 1;
-                            st = SK - 1;
-                        } else {
-                            seg = 1;
-                            h = H - 1;
-                            st = SV - 1;
-                            --rec;
-                        }
-                    },
-                    m);
+        const unsigned first = s * static_cast<unsigned>(L);
+        const int m = n - first < static_cast<unsigned>(L) ? static_cast<int>(n - first) : L;
+        const unsigned q = first + m - 1;             // the span's last symbol
+        unsigned rec = div_r.div(q);
+        int o = static_cast<int>(q - rec * static_cast<unsigned>(R));
+        Sym *base = out + w.stream * static_cast<int64_t>(n);
+        const double2 p = pts[w.stream * pt_stride + s];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        fkvdec::walk(t, X, Y, m, [&](int, int c) {
+            const unsigned S = o < nk ? SK : SV;
+            base[poff[o] + rec * S] = static_cast<Sym>(c);
+            if (o == 0) {
+                o = R;
+                --rec;
+            }
+            --o;
+        });
+        const long long lim = m == L ? lim_full : __ldg(&dc->alim[m]);
+        if (X > lim || X < -lim || Y > lim || Y < -lim)
+            atomicOr(status, FKV_ST_CORRUPT);
     }
 }
 
@@ -775,9 +824,10 @@ k_lossy_decode(const LossyArgs a, int64_t n, int64_t spans, int bps, int64_t n_c
     for (int i = threadIdx.x; i < N; i += kThreads)
         sV[i] = V[i];
     __syncthreads();
-    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x) {
-        const int64_t stream = ck / bps;
-        const int64_t s0 = (ck - stream * bps) * kThreads;
+    ChunkWalk cw(bps);
+    for (int64_t ck = blockIdx.x; ck < n_chunks; ck += gridDim.x, cw.next()) {
+        const int64_t stream = cw.stream;
+        const int64_t s0 = cw.sb * kThreads;
         const int64_t b = s0 * L;
         const int64_t e = min(n, (s0 + kThreads) * L);
         uint8_t *dst = reinterpret_cast<uint8_t *>(sym + stream * sym_stride + b);
@@ -927,16 +977,18 @@ cudaError_t span_decode_planar_t(const fkv_ctx *c, const double *pts, int64_t n_
                                  int64_t pt_stride, Sym *out, cudaStream_t st)
 {
     const int SK = c->cb[0].stages, SV = c->cb[1].stages;
-    const int64_t n = n_rec * c->H * (SK + SV);
+    const int R = c->H * (SK + SV);
+    const int64_t n = n_rec * R;
     constexpr int TPB = dec_threads<Sym>();
     const int64_t spans = cdiv(n, c->L);
     const int64_t bps = cdiv(spans, TPB);
     const int64_t n_chunks = n_streams * bps;
     if (n_chunks == 0)
         return cudaSuccess;
-    if (bps > 0x7FFFFFFF)
+    // 32-bit positions inside a stream, and chunk numbers
+    if (n > 0x7FFFFFFF || n_chunks > 0x7FFFFFFF)
         return cudaErrorInvalidConfiguration;
-    const int smem = tables_bytes(c->N, c->L);
+    const int smem = tables_bytes(c->N, c->L) + R * static_cast<int>(sizeof(unsigned));
     cudaError_t e = cudaFuncSetAttribute(k_span_decode_planar<Sym>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          smem);
     if (e != cudaSuccess)
@@ -945,10 +997,10 @@ cudaError_t span_decode_planar_t(const fkv_ctx *c, const double *pts, int64_t n_
     e = decode_grid(c, reinterpret_cast<const void *>(k_span_decode_planar<Sym>), smem, n_chunks, &grid, TPB);
     if (e != cudaSuccess)
         return e;
-    k_span_decode_planar<Sym><<<grid, TPB, smem, st>>>(reinterpret_cast<const double2 *>(pts), n_rec,
-                                                            pt_stride, spans, static_cast<int>(bps), n_chunks,
-                                                            out, c->H, SK, SV, c->d_dec, c->d_T, c->N, c->L,
-                                                            c->d_status);
+    k_span_decode_planar<Sym><<<grid, TPB, smem, st>>>(
+        reinterpret_cast<const double2 *>(pts), static_cast<unsigned>(n_rec), pt_stride,
+        static_cast<unsigned>(spans), static_cast<int>(bps), static_cast<unsigned>(n_chunks), out, c->H, SK, SV,
+        FastDiv::make(static_cast<unsigned>(R)), c->d_dec, c->d_T, c->N, c->L, c->d_status);
     return cudaGetLastError();
 }
 

@@ -46,6 +46,19 @@ def test_rvq_flops_match_the_llama_workload():
     assert "of measured" in dom["kernel"]
 
 
+def test_rvq_traffic_scaling():
+    """The scaled per-launch DRAM traffic: unchanged at the captured length,
+    and close to the algorithmic bytes (input + codebook operands + indices)
+    of a full-length launch."""
+    c = synth.CFG3
+    same = bench._rvq_traffic_full(slice_pos=c.n_archived)
+    assert same == (1257913600 + 1176856576) / 2
+    nvec = c.n_layers * c.batch * c.n_heads * c.n_archived
+    groups = c.n_layers * c.n_heads
+    alg = [nvec * c.dim * 2 + groups * s * 256 * c.dim * 4 + nvec * s for s in (4, 2)]
+    assert abs(bench.RVQ_DRAM_BYTES_PER_LAUNCH / (sum(alg) / 2) - 1) < 0.05
+
+
 def test_decode_bytes_and_fp64_fractions():
     cfg = synth.CFG1
     rates, (P, R, ns, n_rec, spans) = _rates(cfg, 0.445, 0.237, 0.088, 0.160)
