@@ -30,8 +30,11 @@
 //   * N <= 8: fp32 scores q . V(c); exact scores when the best two are closer
 //     than a bound far above the fp32 error;
 //   * N > 8: Voronoi regions of the vertices are angular sectors, so the fp32
-//     angle picks the sector; within 1e-3 sector widths of a boundary the two
-//     neighbouring sectors are decided by the sign of Q . (V(a) - V(b)).
+//     angle picks the sector; within twice the angle's error bound of a
+//     boundary (the bound: 1.2e-5 rad for the arctangent polynomial plus
+//     1.5e-6 rad for the fp32 direction, division and reflections, plus
+//     N 2^-24 sector widths for the scaling) the two neighbouring sectors are
+//     decided by the sign of Q . (V(a) - V(b)).
 #pragma once
 
 #include <climits>
@@ -40,12 +43,18 @@
 
 namespace fkvdec {
 
+// atan u ~ u (a1 + a3 u^2 + a5 u^4 + a7 u^6 + a9 u^8) on [0, 1], from
+// fit_atan.py: float32 Horner evaluation within 1.18e-5 rad of atan
+__device__ constexpr float kAtan[5] = {9.998637438e-01f, -3.302824795e-01f, 1.800999194e-01f, -8.509350568e-02f,
+                                       2.082198113e-02f};
+
 struct Tables {
     const longlong2 *T;   // [L][N] (x, y), shared memory
     const long long *vx;  // [N] V(c) in Q1.62, shared memory
     const long long *vy;
     const float2 *vf;     // [N] V(c) as float, shared memory
     int N;
+    float sect_thr;       // sector test: |fraction| below this is decided in fp32
 };
 
 // Shared-memory footprint of the tables for (N, L).
@@ -69,7 +78,7 @@ __device__ inline Tables load(const fkv_decconst *__restrict__ g, const longlong
         vy[i] = g->vy[i];
         vf[i] = make_float2(g->vfx[i], g->vfy[i]);
     }
-    return Tables{T, vx, vy, vf, N};
+    return Tables{T, vx, vy, vf, N, g->sect_thr};
 }
 
 // Q . V(c) in units of 2^-60: the high words of the two 128-bit products
@@ -138,7 +147,21 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
             return bi;
         return classify_exact_all(t, X, Y);
     }
-    const float a = atan2f(qy, qx) * (static_cast<float>(N) * 0.15915494309189535f);
+    // the angle of (qx, qy): octant reduction to u in [0, 1], atan u from
+    // the odd polynomial of fit_atan.py (error below 1.2e-5 rad), then the
+    // octant's reflections, giving an angle in [-pi, pi]
+    const float ax = fabsf(qx), ay = fabsf(qy);
+    const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
+    const float u = mx > 0.0f ? __fdividef(mn, mx) : 0.0f;
+    const float u2 = u * u;
+    float ph = u * fmaf(fmaf(fmaf(fmaf(kAtan[4], u2, kAtan[3]), u2, kAtan[2]), u2, kAtan[1]), u2, kAtan[0]);
+    if (ay > ax)
+        ph = 1.57079637f - ph;
+    if (qx < 0.0f)
+        ph = 3.14159274f - ph;
+    if (qy < 0.0f)
+        ph = -ph;
+    const float a = ph * (static_cast<float>(N) * 0.159154937f);
     const float ar = rintf(a);
     const float f = a - ar;                        // in [-0.5, 0.5]
     int c0 = static_cast<int>(ar);
@@ -146,7 +169,8 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
         c0 += N;
     if (c0 >= N)
         c0 -= N;
-    if (fabsf(f) < 0.499f)
+    // away from a sector boundary by more than twice the angle's error bound
+    if (fabsf(f) < t.sect_thr)
         return c0;
     int c1 = f > 0.0f ? c0 + 1 : c0 - 1;           // the neighbour across the near boundary
     if (c1 < 0)

@@ -359,6 +359,12 @@ int fkv_create(int N, double r, int span_len, const fkv_codebooks *cb, fkv_ctx *
         dec.alim[m] = q_round(0.0625L * rj, 62);
         rj *= static_cast<long double>(r);
     }
+    // the fp32 sector angle's error, in sector widths: 1.2e-5 rad (arctangent
+    // polynomial) + 1.5e-6 rad (direction, division, reflections), times
+    // N / (2 pi), + N 2^-24 (scaling); fractions within twice that of a
+    // boundary take the exact test
+    const double sect_err = N * (1.2e-5 + 1.5e-6) / (2.0 * 3.14159265358979) + N * 0x1p-24;
+    dec.sect_thr = static_cast<float>(0.5 - 2.0 * sect_err);
     CK(cudaMalloc(&ctx->d_V, N * sizeof(double2)), "vertex alloc");
     CK(cudaMemcpy(ctx->d_V, V.data(), N * sizeof(double2), cudaMemcpyHostToDevice), "vertex copy");
     CK(cudaMalloc(&ctx->d_dec, sizeof(fkv_decconst)), "decoder alloc");

@@ -38,6 +38,7 @@ struct fkv_decconst {
     long long vx[FKV_MAX_N], vy[FKV_MAX_N];    // V(c)
     float vfx[FKV_MAX_N], vfy[FKV_MAX_N];      // V(c) rounded to float
     long long alim[48];            // anchor limit 2^-4 r^m in Q1.62, per span length m
+    float sect_thr;                // sector test threshold, N > 8 (decode_core.cuh classify)
 };
 
 struct fkv_ctx {
