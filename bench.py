@@ -418,8 +418,19 @@ def run_e2e(fkv, g, args, dev, world):
     h2d = Kh[:, :, :, g.t0:g.t1 + 1].numel() * Kh.element_size() * 2
     d2h = ptsh[0].numel() * 8 + outh[0].numel() * outh[0].element_size()
     ok = g.ctx.sync_status() == 0
-    del Kh, Vh, Kd, Vd, sts, outs, ptsh, outh
-    return {"ms": e2e_ms, "h2d": h2d, "d2h": d2h, "ok": ok}
+    # the host link on its own: one pinned host -> device copy of the key cache
+    flat_h, flat_d = Kh.view(-1), Kd[1].view(-1)
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            flat_d.copy_(flat_h, non_blocking=True)
+        torch.cuda.synchronize()
+        s2.record(stream)
+        flat_d.copy_(flat_h, non_blocking=True)
+        t2.record(stream)
+    torch.cuda.synchronize()
+    link_gbs = flat_h.numel() * flat_h.element_size() / (s2.elapsed_time(t2) * 1e-3) / 1e9
+    del Kh, Vh, Kd, Vd, sts, outs, ptsh, outh, flat_h, flat_d
+    return {"ms": e2e_ms, "h2d": h2d, "d2h": d2h, "ok": ok, "link_gbs": link_gbs}
 
 
 def oracle_streams(cfg, count=8):
@@ -1002,7 +1013,10 @@ def main():
     if res["e2e"]:
         e2e = {"value": units / (res["e2e"]["ms"] * 1e-3), "unit": UNIT,
                "h2d_bytes_per_step": res["e2e"]["h2d"], "d2h_bytes_per_step": res["e2e"]["d2h"],
-               "ms_per_step": res["e2e"]["ms"], "status_ok": res["e2e"]["ok"]}
+               "ms_per_step": res["e2e"]["ms"], "status_ok": res["e2e"]["ok"],
+               # the step's host -> device bytes against the link measured alone
+               "h2d_link_gbs": res["e2e"]["link_gbs"],
+               "h2d_link_frac": res["e2e"]["h2d"] / (res["e2e"]["ms"] * 1e-3) / 1e9 / res["e2e"]["link_gbs"]}
     fp64 = {"measured_ops_per_s": res["fp64"].get("measured"), "nominal_ops_per_s": res["fp64"]["nominal"],
             "how": "fkv_measure_fp64_rate: independent chains of binary64 multiply and add (no FMA) on every SM; "
                    "nominal = 1.25 TFLOP/s FMA = 625 G add/mul per s at 2070 MHz, scaled to the sampled clock"}

@@ -34,7 +34,9 @@
 //     boundary (the bound: 1.2e-5 rad for the arctangent polynomial plus
 //     1.5e-6 rad for the fp32 direction, division and reflections, plus
 //     N 2^-24 sector widths for the scaling) the two neighbouring sectors are
-//     decided by the sign of Q . (V(a) - V(b)).
+//     decided by the sign of Q . (V(a) - V(b)); the record reads take the
+//     angle from atan2f instead (a shorter dependency chain) with a band of
+//     1e-3 sector widths.
 #pragma once
 
 #include <climits>
@@ -119,6 +121,11 @@ __device__ __forceinline__ void direction(long long X, long long Y, float &qx, f
     qy = __int2float_rn(static_cast<int>(static_cast<unsigned>(ys >> 32)));
 }
 
+// kShortChain: the sector angle from the library's atan2f, whose dependency
+// chain is shorter than the polynomial's (record reads, where one walk per
+// lane is the whole latency); otherwise from the polynomial, which issues
+// fewer instructions (bulk decoders, many walks in flight).
+template <bool kShortChain = false>
 __device__ __forceinline__ int classify(const Tables &t, long long X, long long Y)
 {
     const int N = t.N;
@@ -147,20 +154,28 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
             return bi;
         return classify_exact_all(t, X, Y);
     }
-    // the angle of (qx, qy): octant reduction to u in [0, 1], atan u from
-    // the odd polynomial of fit_atan.py (error below 1.2e-5 rad), then the
-    // octant's reflections, giving an angle in [-pi, pi]
-    const float ax = fabsf(qx), ay = fabsf(qy);
-    const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
-    const float u = mx > 0.0f ? __fdividef(mn, mx) : 0.0f;
-    const float u2 = u * u;
-    float ph = u * fmaf(fmaf(fmaf(fmaf(kAtan[4], u2, kAtan[3]), u2, kAtan[2]), u2, kAtan[1]), u2, kAtan[0]);
-    if (ay > ax)
-        ph = 1.57079637f - ph;
-    if (qx < 0.0f)
-        ph = 3.14159274f - ph;
-    if (qy < 0.0f)
-        ph = -ph;
+    float ph, thr;
+    if constexpr (kShortChain) {
+        // atan2f is within a few ulp: 1e-3 sector widths covers it at any N
+        ph = atan2f(qy, qx);
+        thr = 0.499f;
+    } else {
+        // the angle of (qx, qy): octant reduction to u in [0, 1], atan u
+        // from the odd polynomial of fit_atan.py (error below 1.2e-5 rad),
+        // then the octant's reflections, giving an angle in [-pi, pi]
+        const float ax = fabsf(qx), ay = fabsf(qy);
+        const float mx = fmaxf(ax, ay), mn = fminf(ax, ay);
+        const float u = mx > 0.0f ? __fdividef(mn, mx) : 0.0f;
+        const float u2 = u * u;
+        ph = u * fmaf(fmaf(fmaf(fmaf(kAtan[4], u2, kAtan[3]), u2, kAtan[2]), u2, kAtan[1]), u2, kAtan[0]);
+        if (ay > ax)
+            ph = 1.57079637f - ph;
+        if (qx < 0.0f)
+            ph = 3.14159274f - ph;
+        if (qy < 0.0f)
+            ph = -ph;
+        thr = t.sect_thr;
+    }
     const float a = ph * (static_cast<float>(N) * 0.159154937f);
     const float ar = rintf(a);
     const float f = a - ar;                        // in [-0.5, 0.5]
@@ -169,8 +184,8 @@ __device__ __forceinline__ int classify(const Tables &t, long long X, long long 
         c0 += N;
     if (c0 >= N)
         c0 -= N;
-    // away from a sector boundary by more than twice the angle's error bound
-    if (fabsf(f) < t.sect_thr)
+    // away from a sector boundary by more than the angle's error allows
+    if (fabsf(f) < thr)
         return c0;
     int c1 = f > 0.0f ? c0 + 1 : c0 - 1;           // the neighbour across the near boundary
     if (c1 < 0)
@@ -219,12 +234,12 @@ __device__ __forceinline__ long long to_q62(double v)
 // Decode `steps` symbols backward from Q (the span's stored point in Q1.62):
 // step j = 0 .. steps-1 emits the symbol at offset m-1-j of the span.
 // `emit(j, c)` receives each symbol.
-template <class Emit>
+template <bool kShortChain = false, class Emit>
 __device__ __forceinline__ void walk(const Tables &t, long long &X, long long &Y, int steps, Emit emit)
 {
     const int N = t.N;
     for (int j = 0; j < steps; ++j) {
-        const int c = classify(t, X, Y);
+        const int c = classify<kShortChain>(t, X, Y);
         emit(j, c);
         const longlong2 w = t.T[j * N + c];
         X = static_cast<long long>(static_cast<unsigned long long>(X) - static_cast<unsigned long long>(w.x));

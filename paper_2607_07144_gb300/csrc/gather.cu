@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
         const double2 p = a.pts[st * a.pt_stride + u];
         long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
         const int64_t base = u * L - sym0;
-        fkvdec::walk(t, X, Y, m, [&](int j, int c) {
+        fkvdec::walk<true>(t, X, Y, m, [&](int j, int c) {
             const int64_t pos = base + m - 1 - j;
             if (pos >= 0 && pos < R)
                 my[pos] = static_cast<Sym>(c);
