@@ -299,69 +299,96 @@ __host__ __device__ inline int read_tables_bytes(int N, int L)
 }
 
 // One warp per request: its lanes decode the spans covering the record into
-// shared memory, then gather the record's 2 * H head vectors.
+// shared memory, then rebuild the record's 2 * H head vectors, eight
+// consecutive dimensions per lane and item (two 16-byte codeword loads per
+// stage, four stages' loads issued before their sums).  Persistent: a block
+// loads the decoder tables once and its warps take requests blockIdx.x *
+// warps + warp, + gridDim.x * warps, ...  Three blocks per SM (80 registers,
+// a few spilled to L1) beat two without spills: 1.12 against 1.20 ms for
+// 262,144 Llama-shaped records.
 template <typename Sym>
-__global__ void __launch_bounds__(kReadWarps * 32) k_read_kv(const ReadArgs a)
+__global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a)
 {
     extern __shared__ __align__(16) uint8_t dsm[];
     const fkvdec::Tables t = fkvdec::load(a.dec, a.T, a.N, a.L, dsm);
     Sym *srec = reinterpret_cast<Sym *>(dsm + read_tables_bytes(a.N, a.L));
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t q = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp;
-    if (q >= a.n_req)
-        return;
-    const int64_t st = a.req[2 * q], rec = a.req[2 * q + 1];
     const int H = a.n_heads, D = a.D, R = a.R, L = a.L;
     const int64_t out_vec = static_cast<int64_t>(2) * H * D;
-    if (st < 0 || st >= a.n_streams || rec < 0 || rec >= a.n_rec) {
-        for (int64_t i = lane; i < out_vec / 2; i += 32)
-            store2(a.out, a.dtype, q * out_vec + 2 * i, 0.0f, 0.0f);
-        if (lane == 0)
-            atomicOr(a.status, FKV_ST_RANGE);
-        return;
-    }
-    const int64_t n = a.n_rec * R;
-    const int64_t sym0 = rec * R;
-    const int64_t u0 = sym0 / L, u1 = (sym0 + R - 1) / L;
+    const int gsh = D == 128 ? 4 : 3;             // log2 of the 8-dimension groups per head
+    const int items = 2 * H << gsh;
     Sym *my = srec + warp * kMaxRecord;
-    bool bad = false;
-    for (int64_t u = u0 + lane; u <= u1; u += 32) {
-        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
-        const double2 p = a.pts[st * a.pt_stride + u];
-        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
-        const int64_t base = u * L - sym0;
-        fkvdec::walk<true>(t, X, Y, m, [&](int j, int c) {
-            const int64_t pos = base + m - 1 - j;
-            if (pos >= 0 && pos < R)
-                my[pos] = static_cast<Sym>(c);
-        });
-        const long long lim = __ldg(&a.dec->alim[m]);
-        bad |= X > lim || X < -lim || Y > lim || Y < -lim;
-    }
-    if (bad)
-        atomicOr(a.status, FKV_ST_CORRUPT);
-    __syncwarp();
-    const int l = static_cast<int>(st % a.n_layers);
-    for (int kv = 0; kv < 2; ++kv) {
-        const int S = kv == 0 ? a.SK : a.SV;
-        const float *cb = kv == 0 ? a.cbk : a.cbv;
-        const int off = kv == 0 ? 0 : H * a.SK;
-        for (int hh = 0; hh < H; ++hh) {
-            const int64_t cg = a.pooled ? l : static_cast<int64_t>(l) * H + hh;
-            const float *gcb = cb + cg * S * a.KC * D;
-            const int64_t obase = q * out_vec + (static_cast<int64_t>(kv) * H + hh) * D;
-            for (int d = lane * 2; d < D; d += 64) {
-                float x = 0.0f, y = 0.0f;
-                for (int s = 0; s < S; ++s) {
-                    const float2 c = __ldg(reinterpret_cast<const float2 *>(
-                        gcb + (static_cast<int64_t>(s) * a.KC + my[off + hh * S + s]) * D + d));
-                    x += c.x;
-                    y += c.y;
-                }
-                store2(a.out, a.dtype, obase + d, x, y);
-            }
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp; q < a.n_req;
+         q += static_cast<int64_t>(gridDim.x) * kReadWarps) {
+        const int64_t st = a.req[2 * q], rec = a.req[2 * q + 1];
+        if (st < 0 || st >= a.n_streams || rec < 0 || rec >= a.n_rec) {
+            for (int64_t i = lane; i < out_vec / 2; i += 32)
+                store2(a.out, a.dtype, q * out_vec + 2 * i, 0.0f, 0.0f);
+            if (lane == 0)
+                atomicOr(a.status, FKV_ST_RANGE);
+            continue;
         }
+        const int64_t n = a.n_rec * R;
+        const int64_t sym0 = rec * R;
+        const int64_t u0 = sym0 / L, u1 = (sym0 + R - 1) / L;
+        bool bad = false;
+        for (int64_t u = u0 + lane; u <= u1; u += 32) {
+            const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+            const double2 p = a.pts[st * a.pt_stride + u];
+            long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+            const int64_t base = u * L - sym0;
+            fkvdec::walk<true>(t, X, Y, m, [&](int j, int c) {
+                const int64_t pos = base + m - 1 - j;
+                if (pos >= 0 && pos < R)
+                    my[pos] = static_cast<Sym>(c);
+            });
+            const long long lim = __ldg(&a.dec->alim[m]);
+            bad |= X > lim || X < -lim || Y > lim || Y < -lim;
+        }
+        if (bad)
+            atomicOr(a.status, FKV_ST_CORRUPT);
+        __syncwarp();
+        const int l = static_cast<int>(st % a.n_layers);
+#pragma unroll 2
+        for (int g = lane; g < items; g += 32) {
+            const int kv = g >= (H << gsh) ? 1 : 0;
+            const int gi = kv ? g - (H << gsh) : g;
+            const int hh = gi >> gsh, d0 = (gi - (hh << gsh)) * 8;
+            const int S = kv ? a.SV : a.SK;
+            const float *cb = kv ? a.cbv : a.cbk;
+            const int off = kv ? H * a.SK : 0;
+            const int64_t cg = a.pooled ? l : static_cast<int64_t>(l) * H + hh;
+            const float *gcb = cb + cg * S * a.KC * D + d0;
+            float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f), y = x;
+            for (int s0 = 0; s0 < S; s0 += 4) {
+                float4 c[8];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    if (s0 + k < S) {
+                        const float4 *row = reinterpret_cast<const float4 *>(
+                            gcb + (static_cast<int64_t>(s0 + k) * a.KC + my[off + hh * S + s0 + k]) * D);
+                        c[2 * k] = __ldg(row);
+                        c[2 * k + 1] = __ldg(row + 1);
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    if (s0 + k < S) {
+                        x.x += c[2 * k].x;
+                        x.y += c[2 * k].y;
+                        x.z += c[2 * k].z;
+                        x.w += c[2 * k].w;
+                        y.x += c[2 * k + 1].x;
+                        y.y += c[2 * k + 1].y;
+                        y.z += c[2 * k + 1].z;
+                        y.w += c[2 * k + 1].w;
+                    }
+                }
+            }
+            store8(a.out, a.dtype, q * out_vec + (static_cast<int64_t>(kv) * H + hh) * D + d0, x, y);
+        }
+        __syncwarp();                             // the next request reuses `my`
     }
 }
 
@@ -466,9 +493,6 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     a.status = c->d_status;
     if (n_req <= 0)
         return cudaSuccess;
-    const int64_t blocks = (n_req + kReadWarps - 1) / kReadWarps;
-    if (blocks > 0x7FFFFFFF)
-        return cudaErrorInvalidConfiguration;
     const int esz = c->KC == 256 ? 1 : 2;
     const int smem = read_tables_bytes(a.N, a.L) + kReadWarps * kMaxRecord * esz;
     const void *kern = esz == 1 ? reinterpret_cast<const void *>(k_read_kv<uint8_t>)
@@ -476,6 +500,18 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess)
         return e;
+    // persistent: as many blocks as fit at once, or one per eight requests
+    int sms = 0, per_sm = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
+    if (e != cudaSuccess)
+        return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kReadWarps * 32, smem);
+    if (e != cudaSuccess)
+        return e;
+    int64_t blocks = (n_req + kReadWarps - 1) / kReadWarps;
+    const int64_t resident = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
+    if (blocks > resident)
+        blocks = resident;
     void *args[] = {&a};
     e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kReadWarps * 32), args, smem, st);
     if (e != cudaSuccess)
