@@ -384,7 +384,11 @@ int fkv_cache_upload(fkv_ctx *ctx, const fkv_cache *src_host, const fkv_cache *d
  * decode only the spans of that record and write its K and V head vectors to
  * out_dev, laid out [n_req][2 (K, V)][n_heads][dim] in `dtype`.  Streams hold
  * n_rec records each, points as in fkv_decode_kv.  Out-of-range requests
- * write zeros and set FKV_ERANGE. */
+ * write zeros and set FKV_ERANGE.  The requests are taken grouped by layer
+ * (a counting sort of their indices on the device, so that one layer's
+ * codebooks serve the requests in flight); the context keeps the index
+ * buffer, allocating it on first use and whenever n_req outgrows it (after a
+ * synchronisation of `stream`). */
 int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec,
                 int64_t pt_stride, const int64_t *req_dev, int64_t n_req, void *out_dev,
                 int dtype, void *stream);

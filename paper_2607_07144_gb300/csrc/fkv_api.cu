@@ -415,6 +415,7 @@ int fkv_destroy(fkv_ctx *ctx)
     cudaFree(ctx->d_T);
     cudaFree(ctx->d_status);
     cudaFree(ctx->d_scratch);
+    cudaFree(ctx->d_read_order);
     destroy_cbset(ctx->cb[0]);
     destroy_cbset(ctx->cb[1]);
     delete ctx;
@@ -900,8 +901,17 @@ int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t 
         return fail(ctx, FKV_EINVAL, "point stride too small");
     if (reinterpret_cast<uintptr_t>(out_dev) % 16 || reinterpret_cast<uintptr_t>(pts_dev) % 16)
         return fail(ctx, FKV_EINVAL, "misaligned buffer");
+    const size_t need = static_cast<size_t>(read_order_ints(ctx, n_req)) * sizeof(int);
+    if (need > ctx->read_order_bytes) {
+        CK(cudaStreamSynchronize(as_stream(stream)), "read order sync");
+        cudaFree(ctx->d_read_order);
+        ctx->d_read_order = nullptr;
+        ctx->read_order_bytes = 0;
+        CK(cudaMalloc(&ctx->d_read_order, need), "read order alloc");
+        ctx->read_order_bytes = need;
+    }
     CK(launch_read_kv(ctx, pts_dev, n_streams, n_rec, pt_stride, req_dev, n_req, out_dev, dtype,
-                      as_stream(stream)),
+                      need ? ctx->d_read_order : nullptr, as_stream(stream)),
        "read_kv launch");
     return FKV_OK;
 }

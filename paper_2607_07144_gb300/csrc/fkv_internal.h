@@ -58,6 +58,10 @@ struct fkv_ctx {
     fkv_cbset cb[2];
     uint8_t *d_scratch = nullptr;
     size_t scratch_bytes = 0;
+    // record reads: request indices grouped by layer and the layer counters
+    // (gather.cu launch_read_kv), grown on demand
+    int *d_read_order = nullptr;
+    size_t read_order_bytes = 0;
     // device address and size of the library's fixed scratch array on this
     // context's device (decode_static.cu), looked up once by fkv_create
     uint8_t *static_scratch = nullptr;
@@ -145,9 +149,14 @@ int static_scratch_resolve(fkv_ctx *ctx);
 // gather.cu
 cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st);
+// order: null, or room for read_order_ints(c, n_req) ints, 16-byte aligned
+// (requests then taken grouped by layer)
 cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
                            int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
-                           int dtype, cudaStream_t st);
+                           int dtype, int *order, cudaStream_t st);
+// ints of the record reads' order buffer for n_req requests, or 0 when the
+// requests are taken in their given order (too many requests or layers)
+int64_t read_order_ints(const fkv_ctx *c, int64_t n_req);
 
 // ------------------------------------------------------- device helpers
 #ifdef __CUDACC__

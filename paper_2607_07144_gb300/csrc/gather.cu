@@ -282,6 +282,7 @@ struct ReadArgs {
     const double2 *pts;
     int64_t n_streams, n_rec, pt_stride;
     const int64_t *req;
+    const int4 *order;             // (request, stream or -1, record, 0) grouped by layer, or null
     int64_t n_req;
     void *out;
     int dtype;
@@ -319,9 +320,18 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
     const int gsh = D == 128 ? 4 : 3;             // log2 of the 8-dimension groups per head
     const int items = 2 * H << gsh;
     Sym *my = srec + warp * kMaxRecord;
-    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp; q < a.n_req;
-         q += static_cast<int64_t>(gridDim.x) * kReadWarps) {
-        const int64_t st = a.req[2 * q], rec = a.req[2 * q + 1];
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * kReadWarps + warp; i < a.n_req;
+         i += static_cast<int64_t>(gridDim.x) * kReadWarps) {
+        int64_t q = i, st, rec;
+        if (a.order) {
+            const int4 e = a.order[i];
+            q = e.x;
+            st = e.y;
+            rec = e.z;
+        } else {
+            st = a.req[2 * q];
+            rec = a.req[2 * q + 1];
+        }
         if (st < 0 || st >= a.n_streams || rec < 0 || rec >= a.n_rec) {
             for (int64_t i = lane; i < out_vec / 2; i += 32)
                 store2(a.out, a.dtype, q * out_vec + 2 * i, 0.0f, 0.0f);
@@ -392,7 +402,85 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
     }
 }
 
+// The layer of request q, or n_layers for an out-of-range request (taken last).
+__device__ __forceinline__ int req_layer(const int64_t *req, int64_t q, int64_t n_streams, int64_t n_rec,
+                                         int n_layers)
+{
+    const int64_t st = req[2 * q], rec = req[2 * q + 1];
+    return st < 0 || st >= n_streams || rec < 0 || rec >= n_rec ? n_layers : static_cast<int>(st % n_layers);
+}
+
+// Counting sort of the requests by layer, step 1: per-layer counts (a
+// shared-memory histogram per block, then one global add per layer).
+__global__ void __launch_bounds__(256) k_order_count(const int64_t *__restrict__ req, int64_t n_req, int64_t n_streams,
+                                                     int64_t n_rec, int n_layers, int *__restrict__ cnt)
+{
+    extern __shared__ int hist[];
+    for (int i = threadIdx.x; i <= n_layers; i += blockDim.x)
+        hist[i] = 0;
+    __syncthreads();
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < n_req;
+         q += static_cast<int64_t>(gridDim.x) * blockDim.x)
+        atomicAdd(&hist[req_layer(req, q, n_streams, n_rec, n_layers)], 1);
+    __syncthreads();
+    for (int i = threadIdx.x; i <= n_layers; i += blockDim.x)
+        if (hist[i])
+            atomicAdd(&cnt[i], hist[i]);
+}
+
+// Step 2: counts -> first slot of each layer (exclusive prefix sum, one thread).
+__global__ void k_order_scan(int *cnt, int n_layers)
+{
+    int sum = 0;
+    for (int i = 0; i <= n_layers; ++i) {
+        const int c = cnt[i];
+        cnt[i] = sum;
+        sum += c;
+    }
+}
+
+// Step 3: each block counts its contiguous share of the requests per layer,
+// reserves a run of slots per layer with one global add, and places its
+// requests in those runs as (request, stream, record, 0), stream -1 for an
+// out-of-range request.  The order inside a layer is arbitrary: every output
+// goes to its own request's place.
+__global__ void __launch_bounds__(256) k_order_scatter(const int64_t *__restrict__ req, int64_t n_req,
+                                                       int64_t n_streams, int64_t n_rec, int n_layers,
+                                                       int *__restrict__ slot, int4 *__restrict__ order)
+{
+    extern __shared__ int sh[];                  // [n_layers + 1] counts, then run starts
+    int *cntl = sh, *base = sh + n_layers + 1;
+    const int64_t q0 = n_req * blockIdx.x / gridDim.x, q1 = n_req * (blockIdx.x + 1) / gridDim.x;
+    for (int i = threadIdx.x; i <= n_layers; i += blockDim.x)
+        cntl[i] = 0;
+    __syncthreads();
+    for (int64_t q = q0 + threadIdx.x; q < q1; q += blockDim.x)
+        atomicAdd(&cntl[req_layer(req, q, n_streams, n_rec, n_layers)], 1);
+    __syncthreads();
+    for (int i = threadIdx.x; i <= n_layers; i += blockDim.x) {
+        base[i] = cntl[i] ? atomicAdd(&slot[i], cntl[i]) : 0;
+        cntl[i] = 0;
+    }
+    __syncthreads();
+    for (int64_t q = q0 + threadIdx.x; q < q1; q += blockDim.x) {
+        const int ly = req_layer(req, q, n_streams, n_rec, n_layers);
+        const int pos = base[ly] + atomicAdd(&cntl[ly], 1);
+        order[pos] = ly < n_layers ? make_int4(static_cast<int>(q), static_cast<int>(req[2 * q]),
+                                               static_cast<int>(req[2 * q + 1]), 0)
+                                   : make_int4(static_cast<int>(q), -1, 0, 0);
+    }
+}
+
 }  // namespace
+
+int64_t read_order_ints(const fkv_ctx *c, int64_t n_req)
+{
+    // 32-bit request, stream and record numbers in the entries; the
+    // per-block counts and run starts in 48 KB of shared memory
+    if (n_req <= 0 || n_req > 0x7FFFFFFF || 2 * (c->Ly + 1) > 12 * 1024)
+        return 0;
+    return 4 * n_req + c->Ly + 1;
+}
 
 cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
                               int64_t n_rec, const fkv_cache *out, int64_t t0, cudaStream_t st)
@@ -465,7 +553,7 @@ cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int lay
 
 cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_streams, int64_t n_rec,
                            int64_t pt_stride, const int64_t *req, int64_t n_req, void *out,
-                           int dtype, cudaStream_t st)
+                           int dtype, int *order, cudaStream_t st)
 {
     ReadArgs a;
     a.pts = reinterpret_cast<const double2 *>(pts);
@@ -473,6 +561,7 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     a.n_rec = n_rec;
     a.pt_stride = pt_stride;
     a.req = req;
+    a.order = nullptr;
     a.n_req = n_req;
     a.out = out;
     a.dtype = dtype;
@@ -505,6 +594,24 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device);
     if (e != cudaSuccess)
         return e;
+    if (order && n_streams <= 0x7FFFFFFF && n_rec <= 0x7FFFFFFF) {
+        // requests grouped by layer: n_req int4 entries, the layer counters after them
+        int4 *ent = reinterpret_cast<int4 *>(order);
+        int *cnt = order + 4 * n_req;
+        e = cudaMemsetAsync(cnt, 0, (c->Ly + 1) * sizeof(int), st);
+        if (e != cudaSuccess)
+            return e;
+        const int64_t need = (n_req + 255) / 256;
+        const unsigned g = static_cast<unsigned>(need < 4 * sms ? need : 4 * sms);
+        const size_t hsm = (c->Ly + 1) * sizeof(int);
+        k_order_count<<<g, 256, hsm, st>>>(req, n_req, n_streams, n_rec, c->Ly, cnt);
+        k_order_scan<<<1, 1, 0, st>>>(cnt, c->Ly);
+        k_order_scatter<<<g, 256, 2 * hsm, st>>>(req, n_req, n_streams, n_rec, c->Ly, cnt, ent);
+        e = cudaGetLastError();
+        if (e != cudaSuccess)
+            return e;
+        a.order = ent;
+    }
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kReadWarps * 32, smem);
     if (e != cudaSuccess)
         return e;

@@ -148,3 +148,32 @@ def test_decode_time_streaming(fkv, oracle_mod):
     ctx.rvq_encode(0, K, 4, 4 + prefill + 24, whole)
     ctx.rvq_encode(1, V, 4, 4 + prefill + 24, whole)
     assert np.array_equal(whole.cpu().numpy(), full)
+
+
+def test_record_reads_in_any_order(fkv):
+    """Record reads (Sec. 2) taken grouped by layer inside the library: every
+    output lands at its own request's place whatever the order, across calls
+    whose request count grows (the order buffer is reallocated), with
+    out-of-range requests mixed in (zeros and FKV_ERANGE)."""
+    cfg = synth.small_config(synth.CFG3, 313, n_layers=5, batch=3, seq=36 + 77)
+    K = synth.gpu_kv_cache(cfg, 0)
+    V = synth.gpu_kv_cache(cfg, 1)
+    ctx, sym, pts = write_archive(fkv, cfg, K, V)
+    P = cfg.n_archived
+    Kr, Vr = torch.zeros_like(K), torch.zeros_like(V)
+    ctx.decode_kv(pts, P, Kr, Vr, t0=cfg.t0)
+    ns = cfg.batch * cfg.n_layers
+    ti = lambda a: torch.from_numpy(a).cuda()
+    for n_req, seed in ((100, 1), (5000, 2), (40000, 3), (7, 4)):
+        rng = np.random.default_rng(seed)
+        req = np.stack([rng.integers(0, ns, n_req), rng.integers(0, P, n_req)], axis=1)
+        bad = rng.random(n_req) < 0.05
+        req[bad, 0] = rng.choice([-1, ns, ns + 7], bad.sum())
+        out = torch.full((n_req, 2, cfg.n_heads, cfg.dim), 9.0, dtype=K.dtype, device="cuda")
+        ctx.read_kv(pts, P, ti(req), out)
+        assert ctx.sync_status() == (-2 if bad.any() else 0)
+        ok = ~bad
+        b, l, t = req[ok, 0] // cfg.n_layers, req[ok, 0] % cfg.n_layers, req[ok, 1] + cfg.t0
+        assert torch.equal(out[ti(np.flatnonzero(ok)), 0], Kr[ti(l), ti(b), :, ti(t)])
+        assert torch.equal(out[ti(np.flatnonzero(ok)), 1], Vr[ti(l), ti(b), :, ti(t)])
+        assert torch.count_nonzero(out[ti(np.flatnonzero(bad))]) == 0
