@@ -299,6 +299,37 @@ __device__ __forceinline__ void add_codeword(uint4 hv, uint4 lv, float f, float 
     }
 }
 
+// Chunk c of this row's operand plus f times 8 float32 codeword elements:
+// v = (hi + lo) + c f, the hi + lo sum exact in fp32 (lo lies at least 11 bits
+// below hi) by one conversion and one mixed-precision multiply-add, then one
+// rounding in the final multiply-add.
+__device__ __forceinline__ void load_add_chunk(const uint8_t *ahi, const uint8_t *alo, int row, int c, float4 c0,
+                                               float4 c1, float f, float *v)
+{
+    const uint32_t off = swz(row, c);
+    const uint4 hv = *reinterpret_cast<const uint4 *>(ahi + off);
+    const uint4 lv = *reinterpret_cast<const uint4 *>(alo + off);
+    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
+    const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
+    const float cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float s0, s1;
+        asm("{\n\t.reg .b16 h0, h1, l0, l1, one;\n\t"
+            "mov.b32 {h0, h1}, %2;\n\t"
+            "mov.b32 {l0, l1}, %3;\n\t"
+            "mov.b16 one, 0x3C00;\n\t"
+            "cvt.f32.f16 %0, l0;\n\t"
+            "cvt.f32.f16 %1, l1;\n\t"
+            "fma.rn.f32.f16 %0, h0, one, %0;\n\t"
+            "fma.rn.f32.f16 %1, h1, one, %1;\n\t}"
+            : "=f"(s0), "=f"(s1)
+            : "r"(hw[i]), "r"(lw[i]));
+        v[2 * i] = fmaf(cw[2 * i], f, s0);
+        v[2 * i + 1] = fmaf(cw[2 * i + 1], f, s1);
+    }
+}
+
 // Eight consecutive input elements (chunk c of the row) as floats.
 template <int ESZ>
 __device__ __forceinline__ void unpack8(const uint4 *xr, int dtype, int c, float *v)
@@ -1022,18 +1053,17 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                 tc_fence_before();
                 idx[s] = static_cast<uint8_t>(bidx);
                 if (s + 1 < S) {
-                    // t <- t + (hi + lo) 2^(-1-er) from the codeword's global hi/lo rows
-                    const float f = pow2f(-1 - er);
-                    const uint4 *gh = reinterpret_cast<const uint4 *>(
-                        a.cb16 + ((static_cast<int64_t>(cgroup(g) * S + s) * 2) * kCodes + bidx) * D);
-                    constexpr int LO = kCodes * D / 8;   // uint4 from a hi row to its lo row
+                    // t <- t - c 2^(-e-er) (t is the row in units of 2^-(e+er)),
+                    // c the chosen codeword's float32 row
+                    const float f = -pow2f(-e - er);
+                    const float4 *gc = reinterpret_cast<const float4 *>(
+                        a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D);
                     if (e_next == e) {
 #pragma unroll 4
                         for (int c = 0; c < 16; ++c) {
                             float t[8];
                             uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
-                            load_chunk(hp, lp, row, c & 7, t);
-                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+                            load_add_chunk(hp, lp, row, c & 7, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
                             store_chunk(hp, lp, row, c & 7, t);
                         }
                     } else {
@@ -1041,8 +1071,8 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
 #pragma unroll 1
                         for (int c = 0; c < 16; ++c) {
                             float t[8];
-                            load_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7, t);
-                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+                            load_add_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7,
+                                           __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; i += 2)
                                 mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
@@ -1057,8 +1087,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         for (int c = 0; c < 16; ++c) {
                             float t[8];
                             uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
-                            load_chunk(hp, lp, row, c & 7, t);
-                            add_codeword(__ldg(gh + c), __ldg(gh + LO + c), f, t);
+                            load_add_chunk(hp, lp, row, c & 7, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; ++i)
                                 t[i] *= gsc;
