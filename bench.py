@@ -83,20 +83,21 @@ def load_peaks():
 
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per RVQ launch of
-# the headline workload, from one ncu capture of the current k_rvq128 on the
-# same cache cut to 4096 archived positions (the full cache is too large for a
-# multi-metric capture): 1,257,913,600 B for the key launch and 1,176,856,576 B
-# for the value launch.  The hi/lo fp16 codebook operands (4 x 256 x 128 x 2 x
-# 2 B per key head, half that per value head) are read once whatever the
-# length; the rest grows with the positions.  The figure is the mean of the key
-# and value launches at the headline length.  Set it to None when k_rvq128
-# changes until it is captured again.
-def _rvq_traffic_full(slice_pos=4096, slice_bytes=((1257913600, 4), (1176856576, 2))):
-    groups = HEADLINE.n_layers * HEADLINE.n_heads
-    full = []
-    for total, stages in slice_bytes:
-        cb = groups * stages * 256 * HEADLINE.dim * 2 * 2
-        full.append((total - cb) * HEADLINE.n_archived / slice_pos + cb)
+# the headline workload, from ncu captures of the current k_rvq128 on the same
+# cache cut to 4096 and to 8192 archived positions (the full cache is too large
+# for a multi-metric capture): key launch 1,340,393,728 and 2,456,583,168 B,
+# value launch 1,209,182,976 and 2,317,623,040 B.  Traffic is a fixed part (the
+# codebooks) plus a part that grows with the positions, so the two lengths fix
+# a line, extrapolated to the headline length; the figure is the mean of the
+# key and value launches.  Set it to None when k_rvq128 changes until it is
+# captured again.
+RVQ_TRAFFIC_CAPTURES = ((4096, 8192), ((1340393728, 2456583168), (1209182976, 2317623040)))
+
+
+def _rvq_traffic_full(positions=None, captures=RVQ_TRAFFIC_CAPTURES):
+    (p1, p2), launches = captures
+    p = HEADLINE.n_archived if positions is None else positions
+    full = [b1 + (b2 - b1) * (p - p1) / (p2 - p1) for b1, b2 in launches]
     return sum(full) / len(full)
 
 

@@ -47,12 +47,14 @@ def test_rvq_flops_match_the_llama_workload():
 
 
 def test_rvq_traffic_scaling():
-    """The scaled per-launch DRAM traffic: unchanged at the captured length,
-    and close to the algorithmic bytes (input + codebook operands + indices)
-    of a full-length launch."""
+    """The per-launch DRAM traffic line through the two captured lengths: it
+    returns the captures at their own lengths and, at the headline length,
+    stays close to the algorithmic bytes (input + codebook operands +
+    indices) of a full-length launch."""
+    (p1, p2), launches = bench.RVQ_TRAFFIC_CAPTURES
+    assert bench._rvq_traffic_full(p1) == sum(b[0] for b in launches) / 2
+    assert bench._rvq_traffic_full(p2) == sum(b[1] for b in launches) / 2
     c = synth.CFG3
-    same = bench._rvq_traffic_full(slice_pos=c.n_archived)
-    assert same == (1257913600 + 1176856576) / 2
     nvec = c.n_layers * c.batch * c.n_heads * c.n_archived
     groups = c.n_layers * c.n_heads
     alg = [nvec * c.dim * 2 + groups * s * 256 * c.dim * 4 + nvec * s for s in (4, 2)]
