@@ -266,22 +266,32 @@ __device__ __forceinline__ uint32_t store_chunk(uint8_t *ahi, uint8_t *alo, int 
     return nz;
 }
 
-// Chunk c of this row's operand as 8 floats hi + lo (exact: lo lies at least
-// 11 bits below hi).
+// hi + lo of 16-bit halves as float32, exact (lo lies at least 11 bits below
+// hi): one conversion and one mixed-precision multiply-add per element.
+__device__ __forceinline__ void join_half2(uint32_t hw, uint32_t lw, float &v0, float &v1)
+{
+    asm("{\n\t.reg .b16 h0, h1, l0, l1, one;\n\t"
+        "mov.b32 {h0, h1}, %2;\n\t"
+        "mov.b32 {l0, l1}, %3;\n\t"
+        "mov.b16 one, 0x3C00;\n\t"
+        "cvt.f32.f16 %0, l0;\n\t"
+        "cvt.f32.f16 %1, l1;\n\t"
+        "fma.rn.f32.f16 %0, h0, one, %0;\n\t"
+        "fma.rn.f32.f16 %1, h1, one, %1;\n\t}"
+        : "=f"(v0), "=f"(v1)
+        : "r"(hw), "r"(lw));
+}
+
+// Chunk c of this row's operand as 8 floats hi + lo (exact).
 __device__ __forceinline__ void load_chunk(const uint8_t *ahi, const uint8_t *alo, int row, int c, float *v)
 {
     const uint32_t off = swz(row, c);
     const uint4 hv = *reinterpret_cast<const uint4 *>(ahi + off);
     const uint4 lv = *reinterpret_cast<const uint4 *>(alo + off);
-    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
-    const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float2 h = __half22float2(*reinterpret_cast<const __half2 *>(&hw[i]));
-        const float2 l = __half22float2(*reinterpret_cast<const __half2 *>(&lw[i]));
-        v[2 * i] = h.x + l.x;
-        v[2 * i + 1] = h.y + l.y;
-    }
+    join_half2(hv.x, lv.x, v[0], v[1]);
+    join_half2(hv.y, lv.y, v[2], v[3]);
+    join_half2(hv.z, lv.z, v[4], v[5]);
+    join_half2(hv.w, lv.w, v[6], v[7]);
 }
 
 // v += (hi + lo) f for the 8 codeword halves of chunk hv/lv (hi + lo exact in
@@ -292,42 +302,24 @@ __device__ __forceinline__ void add_codeword(uint4 hv, uint4 lv, float f, float 
     const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const float2 h = __half22float2(*reinterpret_cast<const __half2 *>(&hw[i]));
-        const float2 l = __half22float2(*reinterpret_cast<const __half2 *>(&lw[i]));
-        v[2 * i] = fmaf(h.x + l.x, f, v[2 * i]);
-        v[2 * i + 1] = fmaf(h.y + l.y, f, v[2 * i + 1]);
+        float c0, c1;
+        join_half2(hw[i], lw[i], c0, c1);
+        v[2 * i] = fmaf(c0, f, v[2 * i]);
+        v[2 * i + 1] = fmaf(c1, f, v[2 * i + 1]);
     }
 }
 
 // Chunk c of this row's operand plus f times 8 float32 codeword elements:
-// v = (hi + lo) + c f, the hi + lo sum exact in fp32 (lo lies at least 11 bits
-// below hi) by one conversion and one mixed-precision multiply-add, then one
-// rounding in the final multiply-add.
+// v = (hi + lo) + c f, the hi + lo sum exact, then one rounding in the final
+// multiply-add.
 __device__ __forceinline__ void load_add_chunk(const uint8_t *ahi, const uint8_t *alo, int row, int c, float4 c0,
                                                float4 c1, float f, float *v)
 {
-    const uint32_t off = swz(row, c);
-    const uint4 hv = *reinterpret_cast<const uint4 *>(ahi + off);
-    const uint4 lv = *reinterpret_cast<const uint4 *>(alo + off);
-    const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w};
-    const uint32_t lw[4] = {lv.x, lv.y, lv.z, lv.w};
+    load_chunk(ahi, alo, row, c, v);
     const float cw[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        float s0, s1;
-        asm("{\n\t.reg .b16 h0, h1, l0, l1, one;\n\t"
-            "mov.b32 {h0, h1}, %2;\n\t"
-            "mov.b32 {l0, l1}, %3;\n\t"
-            "mov.b16 one, 0x3C00;\n\t"
-            "cvt.f32.f16 %0, l0;\n\t"
-            "cvt.f32.f16 %1, l1;\n\t"
-            "fma.rn.f32.f16 %0, h0, one, %0;\n\t"
-            "fma.rn.f32.f16 %1, h1, one, %1;\n\t}"
-            : "=f"(s0), "=f"(s1)
-            : "r"(hw[i]), "r"(lw[i]));
-        v[2 * i] = fmaf(cw[2 * i], f, s0);
-        v[2 * i + 1] = fmaf(cw[2 * i + 1], f, s1);
-    }
+    for (int i = 0; i < 8; ++i)
+        v[i] = fmaf(cw[i], f, v[i]);
 }
 
 // Eight consecutive input elements (chunk c of the row) as floats.
