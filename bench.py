@@ -1040,8 +1040,9 @@ def main():
         "e2e": e2e,
         # per step: RVQ x4 (K and V archive, K and V of the appended position),
         # k_span_encode x2 (archive, tail append), k_span_decode_planar,
-        # k_gather x2, k_read_kv (as the ncu launch list shows)
-        "gpu_launches": 10 * args.steps,
+        # k_gather x2, the record reads' k_order_count, k_order_scan and
+        # k_order_scatter, and k_read_kv (as the ncu launch list shows)
+        "gpu_launches": 13 * args.steps,
         "clocks": res["clocks"],
         "status_ok": res["ok"],
     }
