@@ -781,18 +781,19 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
 // The k_rvq64 scheme (two tile slots, split-fp16 operands of -2 c', a per-row
 // shift, the residual in the operand tiles, exact ld.red argmin) with the
 // head dimension in two 64-wide K blocks.  A slot's hi and lo operand tiles
-// take 64 KB, so the stage codebook does not fit twice: it streams through
-// one buffer a K block at a time (hi and lo of 256 codewords x 64 dimensions,
-// 64 KB, with the 256 x 16 norm operand beside the first block).  Per stage
-// the MMA warp runs both blocks for slot 0 (the norm MMA plus 12 each),
-// committing its accumulator, then both blocks for slot 1, releasing the
-// buffer with a commit after each block; so the stage codebook streams in
-// twice, once per slot, and slot 1's MMAs run during slot 0's epilogue (and
-// slot 0's next stage during slot 1's), where running both slots block by
-// block kept the two in step and left the tensor pipe idle through every
-// epilogue (29.1 / 14.5 ms against 32.9 / 16.8 ms for the Llama-shaped key /
-// value launches).  The buffer is the MMAs' alone: the epilogue reads the
-// chosen codeword's row from the float32 codebook in global (L2) memory.
+// take 64 KB, so the stage codebook does not fit twice: it streams through a
+// ring of two 32 KB pieces, the hi and the lo half of each K block (256
+// codewords x 64 dimensions; the 256 x 16 norm operand rides with a stage's
+// first piece), so the next piece loads while the MMAs use the other.  Per
+// stage the MMA warp runs slot 0's four pieces (hi piece: hi*hi and lo*hi; lo
+// piece: hi*lo; the norm MMA first), committing its accumulator, then slot
+// 1's: the stage codebook streams in once per slot, and slot 1's MMAs run
+// during slot 0's epilogue (and slot 0's next stage during slot 1's).  Running
+// both slots block by block had kept the two in step and left the tensor pipe
+// idle through every epilogue (32.9 / 16.8 ms against 28.9 / 14.5 ms for the
+// Llama-shaped key / value launches; with the ring 27.95 / 13.99 ms).  The
+// buffers are the MMAs' alone: the epilogue reads the chosen codeword's row
+// from the float32 codebook in global (L2) memory.
 namespace v3 {
 constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups
 constexpr int kThreads = kWarps * 32;
@@ -801,14 +802,14 @@ constexpr int A_HALF = 2 * A_KB;             // hi (or lo): both K blocks
 constexpr int A_SLOT = 2 * A_HALF;           // 64 KB
 constexpr int A_AUG = kRows * 32;            // 4 KB per slot
 constexpr int B_TILE = kCodes * 128;         // 32 KB: 256 codewords x 64 fp16
-constexpr int B_BUF = 2 * B_TILE;            // hi + lo of one K block
+constexpr int B_BUF = 2 * B_TILE;            // the ring: two 32 KB codebook pieces
 constexpr int B_AUG = kCodes * 32;           // 8 KB
 constexpr int OFF_A = 0;
 constexpr int OFF_AAUG = 2 * A_SLOT;         // 128 KB
 constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 136 KB: 1024-aligned
 constexpr int OFF_BAUG = OFF_B + B_BUF;
-constexpr int OFF_BAR = OFF_BAUG + B_AUG;    // b_full, b_empty, a_ready[2], acc_full[2], drain
-constexpr int OFF_SLOT = OFF_BAR + 64;
+constexpr int OFF_BAR = OFF_BAUG + B_AUG;    // ring_full[2], ring_empty[2], a_ready[2], acc_full[2], drain
+constexpr int OFF_SLOT = OFF_BAR + 80;
 constexpr int OFF_LO = OFF_SLOT + 16;
 constexpr int OFF_ABORT = OFF_LO + 16;
 constexpr int END = OFF_ABORT + 16;
@@ -829,16 +830,18 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
     volatile int *abort_flag = reinterpret_cast<volatile int *>(base + OFF_ABORT);
     volatile int *lo_stamp = reinterpret_cast<volatile int *>(base + OFF_LO);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // barrier i: 0 b_full; 1 b_empty; 2,3 a_ready; 4,5 acc_full; 6 drain (MMA completion at exit)
+    // barrier i: 0,1 ring_full; 2,3 ring_empty; 4,5 a_ready; 6,7 acc_full; 8 drain (MMA completion at exit)
     auto bar = [&](int i) { return sbase + OFF_BAR + 8u * i; };
     if (tid == 0) {
         mbar_init(bar(0), 1);
         mbar_init(bar(1), 1);
-        mbar_init(bar(2), 128);
-        mbar_init(bar(3), 128);
-        mbar_init(bar(4), 1);
-        mbar_init(bar(5), 1);
+        mbar_init(bar(2), 1);
+        mbar_init(bar(3), 1);
+        mbar_init(bar(4), 128);
+        mbar_init(bar(5), 128);
         mbar_init(bar(6), 1);
+        mbar_init(bar(7), 1);
+        mbar_init(bar(8), 1);
         lo_stamp[0] = 0;
         lo_stamp[1] = 0;
         *abort_flag = 0;
@@ -859,87 +862,83 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
     if (warp == 0) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
-            int it = 0, last = -1;
+            // pieces of a slot's stage: q = 0 hi of K block 0 (with the norm
+            // operand for slot 0), 1 its lo, 2 hi of K block 1, 3 its lo;
+            // piece n goes to ring slot n & 1
+            int n = 0;
+            int last[2] = {-1, -1};
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
                 const int cg = cgroup(p / pairs_per_group);
                 for (int s = 0; s < S && ok; ++s) {
-                    for (int kb4 = 0; kb4 < 4; ++kb4, ++it) {
-                        const int kb = kb4 & 1;           // both K blocks for slot 0, then for slot 1
-                        if (!wait_or_abort(bar(1), (it & 1) ^ 1, a.status, abort_flag)) {
+                    for (int kq = 0; kq < 8; ++kq, ++n) {
+                        const int k = kq >> 2, q = kq & 3, r = n & 1;
+                        if (!wait_or_abort(bar(2 + r), ((n >> 1) & 1) ^ 1, a.status, abort_flag)) {
                             ok = false;
                             break;
                         }
-                        const int row0 = (cg * S + s) * 2 * kCodes;
-                        const uint32_t bb = sbase + OFF_B;
-                        mbar_arrive_expect_tx(bar(0), B_BUF + (kb == 0 ? B_AUG : 0));
-                        tma_load_2d(bb, &tmap, kb * 64, row0, bar(0));
-                        tma_load_2d(bb + B_TILE, &tmap, kb * 64, row0 + kCodes, bar(0));
-                        if (kb == 0)
+                        const int row0 = (cg * S + s) * 2 * kCodes + (q & 1) * kCodes;
+                        const bool aug = q == 0 && k == 0;
+                        mbar_arrive_expect_tx(bar(r), B_TILE + (aug ? B_AUG : 0));
+                        tma_load_2d(sbase + OFF_B + r * B_TILE, &tmap, (q >> 1) * 64, row0, bar(r));
+                        if (aug)   // free: the norm MMAs of the stage before precede the piece this ring slot held
                             bulk_load(sbase + OFF_BAUG, a.cbaug + static_cast<int64_t>(cg * S + s) * kCodes * 16,
-                                      B_AUG, bar(0));
-                        last = it;
+                                      B_AUG, bar(r));
+                        last[r] = n;
                     }
                 }
             }
             // no copy may still be landing in shared memory when the CTA exits
-            if (last >= 0)
-                mbar_wait(bar(0), last & 1, a.status);
+            for (int r = 0; r < 2; ++r)
+                if (last[r] >= 0)
+                    mbar_wait(bar(r), (last[r] >> 1) & 1, a.status);
         }
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
-            int it = 0;
+            int n = 0;
             uint32_t aph[2] = {0, 0};
             int pc = 0;
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
                 ++pc;
                 for (int s = 0; s < S && ok; ++s) {
-                    for (int kb4 = 0; kb4 < 4 && ok; ++kb4, ++it) {
-                        const int kb = kb4 & 1;
-                        ok = wait_or_abort(bar(0), it & 1, a.status, abort_flag);
+                    for (int kq = 0; kq < 8 && ok; ++kq, ++n) {
+                        const int k = kq >> 2, q = kq & 3, r = n & 1;
+                        ok = wait_or_abort(bar(r), (n >> 1) & 1, a.status, abort_flag);
                         if (!ok)
                             break;
-                        const uint32_t bb = sbase + OFF_B;
-                        {
-                            const int k = kb4 >> 1;       // slot k takes both K blocks in turn
-                            if (kb == 0) {
-                                ok = wait_or_abort(bar(2 + k), aph[k], a.status, abort_flag);
-                                if (!ok)
-                                    break;
-                                aph[k] ^= 1;
-                            }
-                            tc_fence_after();
-                            const bool lo = s > 0 || lo_stamp[k] == pc;
-                            const uint32_t ab = sbase + OFF_A + k * A_SLOT + kb * A_KB;
-                            const uint32_t acc = tmem + k * 256;
-                            if (kb == 0)   // codeword norms first (K = 16, no swizzle)
-                                umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(sbase + OFF_BAUG),
-                                         idesc, 0);
-#pragma unroll
-                            for (int kk = 0; kk < 4; ++kk) {
-                                const uint64_t dah = sdesc_sw128(ab + kk * 32);
-                                const uint64_t dal = sdesc_sw128(ab + A_HALF + kk * 32);
-                                const uint64_t dbh = sdesc_sw128(bb + kk * 32);
-                                const uint64_t dbl = sdesc_sw128(bb + B_TILE + kk * 32);
-                                umma_f16(acc, dah, dbh, idesc, 1);
-                                umma_f16(acc, dah, dbl, idesc, 1);
-                                if (lo)
-                                    umma_f16(acc, dal, dbh, idesc, 1);
-                            }
-                            if (kb == 1)
-                                umma_commit(bar(4 + k));
+                        if (q == 0) {
+                            ok = wait_or_abort(bar(4 + k), aph[k], a.status, abort_flag);
+                            if (!ok)
+                                break;
+                            aph[k] ^= 1;
                         }
-                        if (ok)
-                            umma_commit(bar(1));          // the buffer is free once these MMAs are done
+                        tc_fence_after();
+                        const bool lo = s > 0 || lo_stamp[k] == pc;
+                        const uint32_t bb = sbase + OFF_B + r * B_TILE;
+                        const uint32_t ab = sbase + OFF_A + k * A_SLOT + (q >> 1) * A_KB;
+                        const uint32_t acc = tmem + k * 256;
+                        if (q == 0)   // codeword norms first (K = 16, no swizzle)
+                            umma_f16(acc, sdesc_core16(sbase + OFF_AAUG + k * A_AUG), sdesc_core16(sbase + OFF_BAUG),
+                                     idesc, 0);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t db = sdesc_sw128(bb + kk * 32);
+                            umma_f16(acc, sdesc_sw128(ab + kk * 32), db, idesc, 1);     // hi*hi or hi*lo
+                            if ((q & 1) == 0 && lo)
+                                umma_f16(acc, sdesc_sw128(ab + A_HALF + kk * 32), db, idesc, 1);   // lo*hi
+                        }
+                        if (q == 3)
+                            umma_commit(bar(6 + k));
+                        umma_commit(bar(2 + r));          // the ring slot is free once these MMAs are done
                     }
                 }
             }
             // every MMA has completed before tensor memory is released
-            umma_commit(bar(6));
-            mbar_wait(bar(6), 0, a.status);
+            umma_commit(bar(8));
+            mbar_wait(bar(8), 0, a.status);
         }
     } else {
         // ---------------------------------------------------- epilogue groups
@@ -1018,7 +1017,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     lo_stamp[k] = pc;
             }
             fence_proxy_async_smem();
-            mbar_arrive(bar(2 + k));
+            mbar_arrive(bar(4 + k));
             if (p + static_cast<int>(gridDim.x) < n_pairs) {
                 // the next pair's input row into L2 while this pair runs
                 bool nin;
@@ -1031,7 +1030,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
             bool ok = true;
             for (int s = 0; s < S; ++s, ++it) {
                 const int e_next = s + 1 < S ? __ldg(&a.escale_h[g * S + s + 1]) : e;
-                ok = wait_or_abort(bar(4 + k), fph, a.status, abort_flag);
+                ok = wait_or_abort(bar(6 + k), fph, a.status, abort_flag);
                 // the tensor-memory loads below are warp-collective: the warp
                 // goes on, or leaves, as one
                 ok = __all_sync(0xFFFFFFFFu, ok);
@@ -1096,7 +1095,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     }
                     e = e_next;
                     fence_proxy_async_smem();
-                    mbar_arrive(bar(2 + k));
+                    mbar_arrive(bar(4 + k));
                 }
             }
             if (!ok)
