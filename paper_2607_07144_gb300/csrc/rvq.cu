@@ -793,9 +793,15 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
 // idle through every epilogue (32.9 / 16.8 ms against 28.9 / 14.5 ms for the
 // Llama-shaped key / value launches; with the ring 27.95 / 13.99 ms).  The
 // buffers are the MMAs' alone: the epilogue reads the chosen codeword's row
-// from the float32 codebook in global (L2) memory.
+// from the float32 codebook in global (L2) memory.  Four helper warps split the
+// residual update with the slot warps: after its argmin a slot warp leaves its
+// rows' chosen indices and shifts in shared memory and signals the quadrant's
+// helper, then updates the first K block while the helper updates the second;
+// a stage change of scale exchanges the two halves' row maxima through
+// mbarriers, and the MMA warp waits for the helpers' own barrier before a
+// slot's next stage (26.2 / 13.6 ms).
 namespace v3 {
-constexpr int kWarps = 10;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups
+constexpr int kWarps = 14;                   // 0 TMA, 1 MMA, 2..5 and 6..9 epilogue groups, 10..13 update helpers
 constexpr int kThreads = kWarps * 32;
 constexpr int A_KB = kRows * 128;            // 16 KB: 128 rows x 64 fp16 (128-byte swizzle)
 constexpr int A_HALF = 2 * A_KB;             // hi (or lo): both K blocks
@@ -808,8 +814,10 @@ constexpr int OFF_A = 0;
 constexpr int OFF_AAUG = 2 * A_SLOT;         // 128 KB
 constexpr int OFF_B = OFF_AAUG + 2 * A_AUG;  // 136 KB: 1024-aligned
 constexpr int OFF_BAUG = OFF_B + B_BUF;
-constexpr int OFF_BAR = OFF_BAUG + B_AUG;    // ring_full[2], ring_empty[2], a_ready[2], acc_full[2], drain
-constexpr int OFF_SLOT = OFF_BAR + 80;
+constexpr int OFF_BAR = OFF_BAUG + B_AUG;    // ring_full[2], ring_empty[2], a_ready[2], acc_full[2], drain,
+                                             // a_ready_h[2], hand[2][4], mx_e[2][4], mx_h[2][4]
+constexpr int OFF_HX = OFF_BAR + 8 * 40;     // per slot and row: chosen index, row shift, partial maxima
+constexpr int OFF_SLOT = OFF_HX + 2 * kRows * 16;
 constexpr int OFF_LO = OFF_SLOT + 16;
 constexpr int OFF_ABORT = OFF_LO + 16;
 constexpr int END = OFF_ABORT + 16;
@@ -830,7 +838,9 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
     volatile int *abort_flag = reinterpret_cast<volatile int *>(base + OFF_ABORT);
     volatile int *lo_stamp = reinterpret_cast<volatile int *>(base + OFF_LO);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // barrier i: 0,1 ring_full; 2,3 ring_empty; 4,5 a_ready; 6,7 acc_full; 8 drain (MMA completion at exit)
+    // barrier i: 0,1 ring_full; 2,3 ring_empty; 4,5 a_ready; 6,7 acc_full; 8 drain (MMA completion at exit);
+    // 9,10 a_ready_h (helpers); 11 + 4k + q hand (slot k, quadrant q: chosen indices ready); 19 + 4k + q
+    // mx_e and 27 + 4k + q mx_h (the two halves' row maxima when the next stage rescales)
     auto bar = [&](int i) { return sbase + OFF_BAR + 8u * i; };
     if (tid == 0) {
         mbar_init(bar(0), 1);
@@ -842,6 +852,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
         mbar_init(bar(6), 1);
         mbar_init(bar(7), 1);
         mbar_init(bar(8), 1);
+        mbar_init(bar(9), 128);                   // a_ready_h: the helpers' half of an update
+        mbar_init(bar(10), 128);
+        for (int i = 11; i < 35; ++i)             // hand, mx_e, mx_h: one warp each
+            mbar_init(bar(i), 32);
         lo_stamp[0] = 0;
         lo_stamp[1] = 0;
         *abort_flag = 0;
@@ -898,7 +912,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
         if (lane == 0) {
             const uint32_t idesc = idesc_f16_f32(kRows, kCodes);
             int n = 0;
-            uint32_t aph[2] = {0, 0};
+            uint32_t aph[2] = {0, 0}, hph[2] = {0, 0};
             int pc = 0;
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
@@ -911,6 +925,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                             break;
                         if (q == 0) {
                             ok = wait_or_abort(bar(4 + k), aph[k], a.status, abort_flag);
+                            if (ok && s > 0) {    // the helpers' half of the update
+                                ok = wait_or_abort(bar(9 + k), hph[k], a.status, abort_flag);
+                                hph[k] ^= 1;
+                            }
                             if (!ok)
                                 break;
                             aph[k] ^= 1;
@@ -940,6 +958,82 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
             umma_commit(bar(8));
             mbar_wait(bar(8), 0, a.status);
         }
+    } else if (warp >= 10) {
+        // ---------------------------------------------------- update helpers
+        // warp 10 + i serves quadrant (10 + i) & 3 of both slots: for every
+        // update, the second K block (dimensions 64..127) of its 32 rows
+        const int quad = warp & 3;
+        const int row = quad * 32 + lane;
+        uint8_t *hx0 = base + OFF_HX;
+        uint32_t hp_[2] = {0, 0}, xp_[2] = {0, 0};
+        bool ok = true;
+        for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
+            const int g = p / pairs_per_group;
+            int e = __ldg(&a.escale_h[g * S]);
+            for (int s = 0; s + 1 < S && ok; ++s) {
+                const int e_next = __ldg(&a.escale_h[g * S + s + 1]);
+                for (int k = 0; k < 2 && ok; ++k) {
+                    ok = wait_or_abort(bar(11 + 4 * k + quad), hp_[k], a.status, abort_flag);
+                    ok = __all_sync(0xFFFFFFFFu, ok);
+                    if (!ok)
+                        break;
+                    hp_[k] ^= 1;
+                    uint8_t *hx = hx0 + (k * kRows + row) * 16;
+                    const int bidx = hx[0];
+                    const int er = *reinterpret_cast<const int *>(hx + 4);
+                    uint8_t *ahi = base + OFF_A + k * A_SLOT + A_KB;
+                    uint8_t *alo = ahi + A_HALF;
+                    const float f = -pow2f(-e - er);
+                    const float4 *gc = reinterpret_cast<const float4 *>(
+                        a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D) + 16;
+                    if (e_next == e) {
+#pragma unroll 4
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            store_chunk(ahi, alo, row, c, t);
+                        }
+                    } else {
+                        float mx = 0.0f;
+#pragma unroll 1
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; i += 2)
+                                mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
+                        }
+                        // the row's maximum over both halves: exchange with the slot's warp
+                        *reinterpret_cast<float *>(hx + 12) = mx;
+                        mbar_arrive(bar(27 + 4 * k + quad));
+                        ok = wait_or_abort(bar(19 + 4 * k + quad), xp_[k], a.status, abort_flag);
+                        ok = __all_sync(0xFFFFFFFFu, ok);
+                        if (!ok)
+                            break;
+                        xp_[k] ^= 1;
+                        mx = fmaxf(mx, *reinterpret_cast<const float *>(hx + 8));
+                        int E = 0;
+                        if (mx > 0.0f)
+                            frexpf(mx, &E);
+                        const int tot = E + er + e - e_next;
+                        const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
+                        const float gsc = pow2f(er + e - e_next - er2);
+#pragma unroll 1
+                        for (int c = 0; c < 8; ++c) {
+                            float t[8];
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+#pragma unroll
+                            for (int i = 0; i < 8; ++i)
+                                t[i] *= gsc;
+                            store_chunk(ahi, alo, row, c, t);
+                        }
+                    }
+                    fence_proxy_async_smem();
+                    mbar_arrive(bar(9 + k));
+                }
+                e = e_next;
+            }
+        }
     } else {
         // ---------------------------------------------------- epilogue groups
         const int k = (warp - 2) >> 2;           // tile slot 0 or 1
@@ -963,7 +1057,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                                                    (l * a.s_layer + b * a.s_batch + h * a.s_head + t * a.s_pos) * ESZ);
         };
         int it = 0;
-        uint32_t fph = 0;
+        uint32_t fph = 0, xph = 0;
         int pc = 0;
         for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
             const int g = p / pairs_per_group, q = p - g * pairs_per_group;
@@ -1051,29 +1145,41 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                 idx[s] = static_cast<uint8_t>(bidx);
                 if (s + 1 < S) {
                     // t <- t - c 2^(-e-er) (t is the row in units of 2^-(e+er)),
-                    // c the chosen codeword's float32 row
+                    // c the chosen codeword's float32 row; this warp takes the first
+                    // K block, the quadrant's helper the second
+                    uint8_t *hx = base + OFF_HX + (k * kRows + row) * 16;
+                    hx[0] = static_cast<uint8_t>(bidx);
+                    *reinterpret_cast<int *>(hx + 4) = er;
+                    mbar_arrive(bar(11 + 4 * k + quad));
                     const float f = -pow2f(-e - er);
                     const float4 *gc = reinterpret_cast<const float4 *>(
                         a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D);
                     if (e_next == e) {
 #pragma unroll 4
-                        for (int c = 0; c < 16; ++c) {
+                        for (int c = 0; c < 8; ++c) {
                             float t[8];
-                            uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
-                            load_add_chunk(hp, lp, row, c & 7, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
-                            store_chunk(hp, lp, row, c & 7, t);
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            store_chunk(ahi, alo, row, c, t);
                         }
                     } else {
                         float mx = 0.0f;
 #pragma unroll 1
-                        for (int c = 0; c < 16; ++c) {
+                        for (int c = 0; c < 8; ++c) {
                             float t[8];
-                            load_add_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7,
-                                           __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; i += 2)
                                 mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
                         }
+                        // the row's maximum over both halves: exchange with the helper
+                        *reinterpret_cast<float *>(hx + 8) = mx;
+                        mbar_arrive(bar(19 + 4 * k + quad));
+                        ok = wait_or_abort(bar(27 + 4 * k + quad), xph, a.status, abort_flag);
+                        ok = __all_sync(0xFFFFFFFFu, ok);
+                        if (!ok)
+                            break;
+                        xph ^= 1;
+                        mx = fmaxf(mx, *reinterpret_cast<const float *>(hx + 12));
                         int E = 0;
                         if (mx > 0.0f)
                             frexpf(mx, &E);
@@ -1081,14 +1187,13 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
                         const float gsc = pow2f(er + e - e_next - er2);
 #pragma unroll 1
-                        for (int c = 0; c < 16; ++c) {
+                        for (int c = 0; c < 8; ++c) {
                             float t[8];
-                            uint8_t *hp = ahi + (c >> 3) * A_KB, *lp = alo + (c >> 3) * A_KB;
-                            load_add_chunk(hp, lp, row, c & 7, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; ++i)
                                 t[i] *= gsc;
-                            store_chunk(hp, lp, row, c & 7, t);
+                            store_chunk(ahi, alo, row, c, t);
                         }
                         er = er2;
                         write_aug_row(aaug, row, er);
