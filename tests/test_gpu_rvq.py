@@ -233,14 +233,15 @@ def test_small_batch(fkv, oracle_mod, dim, dtype, K, pooled):
         assert ik[0, 0, 0] == 17                        # the codeword-equal row
 
 
-@pytest.mark.parametrize("k1024", [False, True])
-def test_extreme_magnitudes_and_stage_scale_change(fkv, oracle_mod, k1024):
+@pytest.mark.parametrize("dim,k1024", [(64, False), (64, True), (128, False)])
+def test_extreme_magnitudes_and_stage_scale_change(fkv, oracle_mod, dim, k1024):
     """Rows far outside the codebook (1e20, 1e30), far inside it (1e-30,
     subnormal), and a second stage 1e4 times smaller than the first (its
     codebook takes another power-of-two scale, so every row is rescaled and its
-    shift chosen again between the stages), with 256 and 1024 codewords."""
-    dim, K = 64, (1024 if k1024 else 256)
-    rng = np.random.default_rng(11 + k1024)
+    shift chosen again between the stages, from the maximum over both halves
+    of a 128-dimensional row), with 256 and 1024 codewords."""
+    K = 1024 if k1024 else 256
+    rng = np.random.default_rng(11 + k1024 + dim)
     cbk = rng.normal(size=(1, 1, 2, K, dim)).astype(np.float32)
     cbk[0, 0, 1] *= 1e-4
     cbv = rng.normal(size=(1, 1, 1, K, dim)).astype(np.float32)
