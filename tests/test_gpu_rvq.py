@@ -188,7 +188,8 @@ def test_edge_vectors(fkv, oracle_mod, dim):
 
 
 @pytest.mark.parametrize("dim,dtype,K,pooled", [(64, "f16", 256, False), (64, "f32", 256, False),
-                                                (64, "bf16", 1024, True), (128, "bf16", 256, False)])
+                                                (64, "bf16", 1024, True), (128, "bf16", 256, False),
+                                                (128, "bf16", 256, True), (128, "f32", 256, False)])
 def test_small_batch(fkv, oracle_mod, dim, dtype, K, pooled):
     """At most 16 vectors per codebook group (a decode step's appended
     position: tiles with 1 to 16 live rows of 128): every index equals the
