@@ -103,6 +103,10 @@ def _rvq_traffic_full(positions=None, captures=RVQ_TRAFFIC_CAPTURES):
 
 RVQ_DRAM_BYTES_PER_LAUNCH = _rvq_traffic_full()
 
+# GB300's nominal HBM3e bandwidth (the measured copy bandwidth is the roofline's
+# denominator; this one is reported beside it).
+HBM_NOMINAL_GBS = 7900.0
+
 # Nominal FP64 add/mul rate: GB300's 1.25 TFLOP/s of FP64 FMA is 625 G add or
 # mul instructions per second at the 2070 MHz boost clock (1.99 per clock per
 # SM); the measured rate (fkv_measure_fp64_rate) is reported beside it.
@@ -277,7 +281,9 @@ def archive_rates(cfg, phase, R, P, n_rec, spans, ns, peaks, fp64_ops_per_s):
                         "frac_fp64_nominal": enc_fp64 / fp64_ops_per_s["nominal"]},
         "decode_kv": {"bound": "hbm", "ms": phase["decode_kv"], "bytes": dec_bytes,
                       "achieved_gbs": dec_bytes / (phase["decode_kv"] * 1e-3) / 1e9,
-                      "frac": dec_bytes / (phase["decode_kv"] * 1e-3) / 1e9 / peaks["hbm_gbs"]},
+                      "frac": dec_bytes / (phase["decode_kv"] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                      # against GB300's nominal 7.9 TB/s as well as the measured copy
+                      "frac_nominal": dec_bytes / (phase["decode_kv"] * 1e-3) / 1e9 / HBM_NOMINAL_GBS},
         "out_bytes": out_bytes,
     }
 

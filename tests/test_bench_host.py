@@ -71,6 +71,7 @@ def test_decode_bytes_and_fp64_fractions():
     assert d["bytes"] == ns * n_rec * R + ns * spans * 16 + out_bytes   # symbols + points in, K/V out
     assert abs(d["achieved_gbs"] - d["bytes"] / 0.160e-3 / 1e9) < 1e-6
     assert abs(d["frac"] - d["achieved_gbs"] / PEAKS["hbm_gbs"]) < 1e-12
+    assert abs(d["frac_nominal"] - d["achieved_gbs"] / 7900.0) < 1e-12
     e = rates["span_encode"]
     # six binary64 add/sub/mul per symbol against the measured and nominal rates
     assert abs(e["frac_fp64_measured"] - ns * P * R * 6 / 0.088e-3 / 600e9) < 1e-9
