@@ -987,7 +987,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     const float4 *gc = reinterpret_cast<const float4 *>(
                         a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D) + 16;
                     if (e_next == e) {
-#pragma unroll 4
+#pragma unroll
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
                             load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
@@ -1072,24 +1072,11 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
             int er;
             ++pc;
             {
+                // one pass when the row needs no shift (its magnitude below 2^12 in
+                // units of 2^-e, the usual case): the operand is stored as it is
+                // read; a row that turns out larger is stored again, shifted
                 const float se = pow2f(-e);
                 float mx = 0.0f;
-#pragma unroll 4
-                for (int c = 0; c < 16; ++c) {
-                    float f[8];
-                    uint4 xr[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-                    if (in) {
-                        xr[0] = __ldg(src + c * (ESZ / 2));
-                        if (ESZ == 4)
-                            xr[1] = __ldg(src + c * 2 + 1);
-                    }
-                    unpack8<ESZ>(xr, a.dtype, 0, f);
-#pragma unroll
-                    for (int i = 0; i < 8; i += 2)
-                        mx = max3f(mx, fabsf(f[i] * se), fabsf(f[i + 1] * se));
-                }
-                er = row_shift(mx);
-                const float sr = pow2f(-er);
                 uint32_t nz = 0;
 #pragma unroll 4
                 for (int c = 0; c < 16; ++c) {
@@ -1102,9 +1089,32 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     }
                     unpack8<ESZ>(xr, a.dtype, 0, f);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        f[i] = f[i] * se * sr;
+                    for (int i = 0; i < 8; ++i) {
+                        f[i] = f[i] * se;
+                        mx = fmaxf(mx, fabsf(f[i]));
+                    }
                     nz |= store_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7, f);
+                }
+                er = row_shift(mx);
+                if (__any_sync(0xFFFFFFFFu, er != 0)) {
+                    const float sr = pow2f(-er);
+#pragma unroll 4
+                    for (int c = 0; c < 16; ++c) {
+                        if (er == 0)
+                            continue;
+                        float f[8];
+                        uint4 xr[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+                        if (in) {
+                            xr[0] = __ldg(src + c * (ESZ / 2));
+                            if (ESZ == 4)
+                                xr[1] = __ldg(src + c * 2 + 1);
+                        }
+                        unpack8<ESZ>(xr, a.dtype, 0, f);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            f[i] = f[i] * se * sr;
+                        nz |= store_chunk(ahi + (c >> 3) * A_KB, alo + (c >> 3) * A_KB, row, c & 7, f);
+                    }
                 }
                 write_aug_row(aaug, row, er);
                 if (nz)
@@ -1155,7 +1165,7 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     const float4 *gc = reinterpret_cast<const float4 *>(
                         a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D);
                     if (e_next == e) {
-#pragma unroll 4
+#pragma unroll
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
                             load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
