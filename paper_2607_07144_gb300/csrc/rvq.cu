@@ -608,27 +608,34 @@ k_rvq64(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per
             int er;
             ++pc;
             {
+                // one pass when the row needs no shift (the usual case); a row that
+                // turns out larger is stored again, shifted
                 const float se = pow2f(-e);
                 float mx = 0.0f;
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    float f[8];
-                    unpack8<ESZ>(xr, a.dtype, c, f);
-#pragma unroll
-                    for (int i = 0; i < 8; i += 2)
-                        mx = max3f(mx, fabsf(f[i] * se), fabsf(f[i + 1] * se));
-                }
-                er = row_shift(mx);
-                const float sr = pow2f(-er);
                 uint32_t nz = 0;
 #pragma unroll
                 for (int c = 0; c < 8; ++c) {
                     float f[8];
                     unpack8<ESZ>(xr, a.dtype, c, f);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        f[i] = f[i] * se * sr;
+                    for (int i = 0; i < 8; ++i) {
+                        f[i] = f[i] * se;
+                        mx = fmaxf(mx, fabsf(f[i]));
+                    }
                     nz |= store_chunk(ahi, alo, row, c, f);
+                }
+                er = row_shift(mx);
+                if (__any_sync(0xFFFFFFFFu, er != 0) && er != 0) {
+                    const float sr = pow2f(-er);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        float f[8];
+                        unpack8<ESZ>(xr, a.dtype, c, f);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+                            f[i] = f[i] * se * sr;
+                        nz |= store_chunk(ahi, alo, row, c, f);
+                    }
                 }
                 write_aug_row(aaug, row, er);
                 if (nz)
