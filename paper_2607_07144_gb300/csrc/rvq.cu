@@ -1002,13 +1002,14 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         }
                     } else {
                         float mx = 0.0f;
-#pragma unroll 1
+#pragma unroll 4
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
                             load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; i += 2)
                                 mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
+                            store_chunk(ahi, alo, row, c, t);
                         }
                         // the row's maximum over both halves: exchange with the slot's warp
                         *reinterpret_cast<float *>(hx + 12) = mx;
@@ -1025,10 +1026,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         const int tot = E + er + e - e_next;
                         const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
                         const float gsc = pow2f(er + e - e_next - er2);
-#pragma unroll 1
+#pragma unroll
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
-                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            load_chunk(ahi, alo, row, c, t);
 #pragma unroll
                             for (int i = 0; i < 8; ++i)
                                 t[i] *= gsc;
@@ -1180,13 +1181,14 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         }
                     } else {
                         float mx = 0.0f;
-#pragma unroll 1
+#pragma unroll 4
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
                             load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
 #pragma unroll
                             for (int i = 0; i < 8; i += 2)
                                 mx = max3f(mx, fabsf(t[i]), fabsf(t[i + 1]));
+                            store_chunk(ahi, alo, row, c, t);
                         }
                         // the row's maximum over both halves: exchange with the helper
                         *reinterpret_cast<float *>(hx + 8) = mx;
@@ -1203,10 +1205,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                         const int tot = E + er + e - e_next;
                         const int er2 = tot > v2::kRowLog ? tot - v2::kRowLog : 0;
                         const float gsc = pow2f(er + e - e_next - er2);
-#pragma unroll 1
+#pragma unroll
                         for (int c = 0; c < 8; ++c) {
                             float t[8];
-                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
+                            load_chunk(ahi, alo, row, c, t);
 #pragma unroll
                             for (int i = 0; i < 8; ++i)
                                 t[i] *= gsc;
