@@ -291,6 +291,20 @@ int fkv_ac_decode(fkv_ctx *ctx, const uint32_t *words_dev, int64_t word_stride, 
  * on `stream` and waits for it; writes the rate to *ops_per_s (host). */
 int fkv_measure_fp64_rate(double *ops_per_s, void *stream);
 
+/* Failure-path check (no counterpart in the paper): runs, in one CTA on
+ * `stream`, the bounded device waits of the RVQ kernels against mbarriers
+ * that nothing completes, with their teardown (TMEM held and released as the
+ * MMA warp does).  The first waiter gives up after limit_ns (1e5..1e9 ns,
+ * else FKV_EINVAL) and raises the kernel's abort flag; a second waiter on
+ * the same barrier, under the library's full 2 s limit, must leave on that
+ * flag.  Waits for the kernel and writes to result[0..5] (host):
+ * [0] the first waiter's result (0 = gave up), [1] the second's, [2] 1 if
+ * the second left within 2 x limit_ns, [3] a bounded wait on a completed
+ * phase (1), [4] one on an open phase (0), [5] 1 once the teardown ran.
+ * The timeouts set FKV_ETIMEOUT in ctx's status word: fkv_sync_status()
+ * reports and clears it, and the context stays usable. */
+int fkv_check_bounded_wait(fkv_ctx *ctx, int64_t limit_ns, int32_t *result, void *stream);
+
 /* -------------------------------------------------- K/V archive path ---- */
 
 /* A K or V cache tensor on the device: head vectors of `dim` contiguous

@@ -69,6 +69,7 @@ SIGNATURES = {
     "fkv_ac_encode": (_I, [_P, _P, _I64, _I64, _I64, _I, _P, _I64, _P, _P]),
     "fkv_ac_decode": (_I, [_P, _P, _I64, _P, _I64, _I64, _I, _P, _I64, _P]),
     "fkv_measure_fp64_rate": (_I, [_P, _P]),
+    "fkv_check_bounded_wait": (_I, [_P, _I64, _P, _P]),
     "fkv_record_len": (_I, [_P]),
     "fkv_rvq_encode": (_I, [_P, _I, _P, _I64, _I64, _P, _I64, _I64, _P]),
     "fkv_rvq_decode": (_I, [_P, _P, _I64, _I64, _P, _P, _I64, _P]),
@@ -228,6 +229,12 @@ class Context:
 
     def sync_status(self, stream=None) -> int:
         return lib().fkv_sync_status(self._h, _stream(stream))
+
+    def check_bounded_wait(self, limit_ns: int, stream=None) -> list:
+        """fkv_check_bounded_wait: the six results, as ints."""
+        res = (ctypes.c_int32 * 6)()
+        self._check(lib().fkv_check_bounded_wait(self._h, int(limit_ns), res, _stream(stream)))
+        return list(res)
 
     def n_spans(self, n: int) -> int:
         return (int(n) + self.L - 1) // self.L

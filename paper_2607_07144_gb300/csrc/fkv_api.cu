@@ -748,6 +748,30 @@ int fkv_measure_fp64_rate(double *ops_per_s, void *stream)
     return measure_fp64_rate(dev, as_stream(stream), ops_per_s) == cudaSuccess ? FKV_OK : FKV_ECUDA;
 }
 
+int fkv_check_bounded_wait(fkv_ctx *ctx, int64_t limit_ns, int32_t *result, void *stream)
+{
+    if (!ctx)
+        return FKV_EINVAL;
+    if (!result)
+        return fail(ctx, FKV_EINVAL, "null result");
+    if (limit_ns < 100000 || limit_ns > 1000000000)
+        return fail(ctx, FKV_EINVAL, "limit_ns outside [1e5, 1e9]");
+    cudaStream_t st = as_stream(stream);
+    int *d = nullptr;
+    CK(cudaMalloc(&d, 6 * sizeof(int)), "wait check: malloc");
+    cudaError_t e = cudaMemsetAsync(d, 0, 6 * sizeof(int), st);
+    if (e == cudaSuccess)
+        e = launch_wait_check(ctx->d_status, static_cast<uint64_t>(limit_ns), d, st);
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(result, d, 6 * sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+        e = cudaStreamSynchronize(st);
+    const cudaError_t ef = cudaFree(d);
+    CK(e, "wait check");
+    CK(ef, "wait check: free");
+    return FKV_OK;
+}
+
 int fkv_record_len(const fkv_ctx *ctx)
 {
     if (!ctx || !ctx->has_cb)

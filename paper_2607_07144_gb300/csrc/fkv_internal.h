@@ -120,6 +120,10 @@ cudaError_t launch_lossy_read(const fkv_ctx *c, const uint32_t *codes, int64_t c
 // Binary64 add/mul instructions per second of the current device, measured
 // by independent chains (the span encoder's roofline denominator).
 cudaError_t measure_fp64_rate(int device, cudaStream_t st, double *ops_per_s);
+// One CTA that runs the RVQ kernels' bounded waits against barriers that
+// never complete (limit_ns for the first waiter) and their teardown: results
+// to out_dev[0..5] (device ints), the timeout bit to *status.
+cudaError_t launch_wait_check(unsigned *status, uint64_t limit_ns, int *out_dev, cudaStream_t st);
 // ac.cu (Sec. 6 probability-weighted maps): words that always hold the code
 // of n symbols, and the warp-per-stream coder
 int64_t ac_capacity_words(int N, int64_t n);
@@ -208,7 +212,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
 }
 
 // Bounded wait on an mbarrier phase; false (and a status bit) on timeout.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned *status)
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigned *status,
+                                          uint64_t limit_ns = kWaitLimitNs)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -216,7 +221,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, unsigne
     while (true) {
         if (mbar_try_wait(bar, parity))
             return true;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             atomicOr(status, FKV_ST_TIMEOUT);
             return false;
         }

@@ -58,7 +58,7 @@ __device__ __forceinline__ float pow2f(int e)
 
 // Bounded wait that also gives up once another thread has flagged an abort.
 __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, unsigned *status,
-                                              volatile int *abort_flag)
+                                              volatile int *abort_flag, uint64_t limit_ns = kWaitLimitNs)
 {
     if (mbar_try_wait(bar, parity))
         return true;
@@ -68,7 +68,7 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uns
             return true;
         if (*abort_flag)
             return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             atomicOr(status, FKV_ST_TIMEOUT);
             *abort_flag = 1;
             return false;
@@ -1242,7 +1242,67 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
     }
 }
 
+// ===================================================================
+// The failure path of the kernels above, on barriers that never complete.
+// Warp 1 holds TMEM as the MMA warp does; warp 0's lane 0 waits on bar 0,
+// which nothing arrives on, gives up after limit_ns and raises the abort
+// flag; warp 1's lane 0 waits on the same barrier with the library's full
+// limit and must leave on the flag, well before its own timer.  Warp 2 checks
+// that a plain bounded wait passes a completed phase and times out on an
+// open one.  All warps then meet and TMEM is released, as in the kernels'
+// teardown.  out: [0] warp 0's wait result, [1] warp 1's, [2] 1 if warp 1
+// left within 2 x limit_ns (on the flag), [3] the completed phase's wait,
+// [4] the open phase's wait, [5] 1 after the teardown.
+__global__ void __launch_bounds__(96, 1) k_wait_check(unsigned *status, uint64_t limit_ns, int *out)
+{
+    __shared__ __align__(8) uint64_t bars[3];
+    __shared__ int abort_word;
+    __shared__ uint32_t tmem_slot;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int *abort_flag = &abort_word;
+    auto bar = [&](int i) { return smem_u32(&bars[i]); };
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 3; ++i)
+            mbar_init(bar(i), 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1)
+        tmem_alloc(smem_u32(&tmem_slot), 32);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(&tmem_slot);
+    if (lane == 0) {
+        if (warp == 0) {
+            out[0] = wait_or_abort(bar(0), 0, status, abort_flag, limit_ns) ? 1 : 0;
+        } else if (warp == 1) {
+            const uint64_t t0 = globaltimer_ns();
+            out[1] = wait_or_abort(bar(0), 0, status, abort_flag) ? 1 : 0;
+            out[2] = globaltimer_ns() - t0 < 2 * limit_ns ? 1 : 0;
+        } else {
+            mbar_arrive(bar(1));
+            out[3] = mbar_wait(bar(1), 0, status, limit_ns) ? 1 : 0;
+            out[4] = mbar_wait(bar(2), 0, status, limit_ns) ? 1 : 0;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tmem_dealloc(tmem, 32);
+    }
+    if (threadIdx.x == 0)
+        out[5] = 1;
+}
+
 }  // namespace
+
+cudaError_t launch_wait_check(unsigned *status, uint64_t limit_ns, int *out_dev, cudaStream_t st)
+{
+    k_wait_check<<<1, 96, 0, st>>>(status, limit_ns, out_dev);
+    return cudaGetLastError();
+}
 
 template <int ESZ, int NB>
 cudaError_t launch_rvq64(const CUtensorMap &tmap, const RvqArgs &a, int ppg, int n_pairs, unsigned grid,
