@@ -322,6 +322,52 @@ __device__ __forceinline__ void load_add_chunk(const uint8_t *ahi, const uint8_t
         v[i] = fmaf(cw[i], f, v[i]);
 }
 
+// t <- t + c f for the 32 rows of one TMEM lane quadrant and one K block,
+// the warp taking one row at a time: lane i holds dimensions 2i and 2i+1 of
+// the block, so a row's codeword half (256 bytes of float32) is one load of
+// two whole lines, and its operand words are one conflict-free 128-byte
+// access per half.  (Row per lane, each load would touch 32 lines for 16
+// bytes of each.)  bidx and f are this lane's own row's chosen codeword and
+// factor, broadcast row by row; cbk points at the K block's first element of
+// codeword 0 of the stage codebook.  Same arithmetic as load_add_chunk and
+// store_chunk: hi + lo exact, one rounding in the multiply-add.
+__device__ __forceinline__ void update_rows_t(uint8_t *ahi, uint8_t *alo, int quad, const float2 *cbk, int bidx,
+                                              float f)
+{
+    const int lane = threadIdx.x & 31;
+    const uint32_t lofs = static_cast<uint32_t>(((lane >> 2) << 4) | ((lane & 3) << 2));
+    const float2 *cl = cbk + lane;
+    uint8_t *qhi = ahi + quad * 32 * 128, *qlo = alo + quad * 32 * 128;
+#pragma unroll
+    for (int m0 = 0; m0 < 32; m0 += 8) {
+        float2 cv[8];
+        uint32_t hv[8], lv[8];
+        float fm[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int m = m0 + j;
+            const int bm = __shfl_sync(0xFFFFFFFFu, bidx, m);
+            fm[j] = __shfl_sync(0xFFFFFFFFu, f, m);
+            cv[j] = __ldg(cl + bm * 64);
+            const uint32_t off = m * 128 + (lofs ^ (j << 4));      // swz: row & 7 == j
+            hv[j] = *reinterpret_cast<const uint32_t *>(qhi + off);
+            lv[j] = *reinterpret_cast<const uint32_t *>(qlo + off);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            float v0, v1;
+            join_half2(hv[j], lv[j], v0, v1);
+            v0 = fmaf(cv[j].x, fm[j], v0);
+            v1 = fmaf(cv[j].y, fm[j], v1);
+            uint32_t h, l;
+            split_half2(v0, v1, h, l);
+            const uint32_t off = (m0 + j) * 128 + (lofs ^ (j << 4));
+            *reinterpret_cast<uint32_t *>(qhi + off) = h;
+            *reinterpret_cast<uint32_t *>(qlo + off) = l;
+        }
+    }
+}
+
 // Eight consecutive input elements (chunk c of the row) as floats.
 template <int ESZ>
 __device__ __forceinline__ void unpack8(const uint4 *xr, int dtype, int c, float *v)
@@ -991,15 +1037,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     uint8_t *ahi = base + OFF_A + k * A_SLOT + A_KB;
                     uint8_t *alo = ahi + A_HALF;
                     const float f = -pow2f(-e - er);
-                    const float4 *gc = reinterpret_cast<const float4 *>(
-                        a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D) + 16;
+                    const float *cbs = a.cb32 + static_cast<int64_t>(cgroup(g) * S + s) * kCodes * D;
+                    const float4 *gc = reinterpret_cast<const float4 *>(cbs + bidx * D) + 16;
                     if (e_next == e) {
-#pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            float t[8];
-                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
-                            store_chunk(ahi, alo, row, c, t);
-                        }
+                        update_rows_t(ahi, alo, quad, reinterpret_cast<const float2 *>(cbs + 64), bidx, f);
                     } else {
                         float mx = 0.0f;
 #pragma unroll 4
@@ -1170,15 +1211,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     *reinterpret_cast<int *>(hx + 4) = er;
                     mbar_arrive(bar(11 + 4 * k + quad));
                     const float f = -pow2f(-e - er);
-                    const float4 *gc = reinterpret_cast<const float4 *>(
-                        a.cb32 + (static_cast<int64_t>(cgroup(g) * S + s) * kCodes + bidx) * D);
+                    const float *cbs = a.cb32 + static_cast<int64_t>(cgroup(g) * S + s) * kCodes * D;
+                    const float4 *gc = reinterpret_cast<const float4 *>(cbs + bidx * D);
                     if (e_next == e) {
-#pragma unroll
-                        for (int c = 0; c < 8; ++c) {
-                            float t[8];
-                            load_add_chunk(ahi, alo, row, c, __ldg(gc + 2 * c), __ldg(gc + 2 * c + 1), f, t);
-                            store_chunk(ahi, alo, row, c, t);
-                        }
+                        update_rows_t(ahi, alo, quad, reinterpret_cast<const float2 *>(cbs), bidx, f);
                     } else {
                         float mx = 0.0f;
 #pragma unroll 4
