@@ -338,18 +338,30 @@ __device__ __forceinline__ void update_rows_t(uint8_t *ahi, uint8_t *alo, int qu
     const uint32_t lofs = static_cast<uint32_t>(((lane >> 2) << 4) | ((lane & 3) << 2));
     const float2 *cl = cbk + lane;
     uint8_t *qhi = ahi + quad * 32 * 128, *qlo = alo + quad * 32 * 128;
+    // software-pipelined over batches of 8 rows: the next batch's codeword
+    // loads are in flight while this batch is updated
+    float2 cv[2][8];
+    float fm[2][8];
 #pragma unroll
-    for (int m0 = 0; m0 < 32; m0 += 8) {
-        float2 cv[8];
+    for (int j = 0; j < 8; ++j) {
+        fm[0][j] = __shfl_sync(0xFFFFFFFFu, f, j);
+        cv[0][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, j) * 64);
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+        const int cur = b & 1, nxt = cur ^ 1;
+        if (b < 3) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int m = 8 * (b + 1) + j;
+                fm[nxt][j] = __shfl_sync(0xFFFFFFFFu, f, m);
+                cv[nxt][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, m) * 64);
+            }
+        }
         uint32_t hv[8], lv[8];
-        float fm[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-            const int m = m0 + j;
-            const int bm = __shfl_sync(0xFFFFFFFFu, bidx, m);
-            fm[j] = __shfl_sync(0xFFFFFFFFu, f, m);
-            cv[j] = __ldg(cl + bm * 64);
-            const uint32_t off = m * 128 + (lofs ^ (j << 4));      // swz: row & 7 == j
+            const uint32_t off = (8 * b + j) * 128 + (lofs ^ (j << 4));     // swz: row & 7 == j
             hv[j] = *reinterpret_cast<const uint32_t *>(qhi + off);
             lv[j] = *reinterpret_cast<const uint32_t *>(qlo + off);
         }
@@ -357,11 +369,11 @@ __device__ __forceinline__ void update_rows_t(uint8_t *ahi, uint8_t *alo, int qu
         for (int j = 0; j < 8; ++j) {
             float v0, v1;
             join_half2(hv[j], lv[j], v0, v1);
-            v0 = fmaf(cv[j].x, fm[j], v0);
-            v1 = fmaf(cv[j].y, fm[j], v1);
+            v0 = fmaf(cv[cur][j].x, fm[cur][j], v0);
+            v1 = fmaf(cv[cur][j].y, fm[cur][j], v1);
             uint32_t h, l;
             split_half2(v0, v1, h, l);
-            const uint32_t off = (m0 + j) * 128 + (lofs ^ (j << 4));
+            const uint32_t off = (8 * b + j) * 128 + (lofs ^ (j << 4));
             *reinterpret_cast<uint32_t *>(qhi + off) = h;
             *reinterpret_cast<uint32_t *>(qlo + off) = l;
         }
