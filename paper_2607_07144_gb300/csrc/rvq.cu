@@ -323,59 +323,68 @@ __device__ __forceinline__ void load_add_chunk(const uint8_t *ahi, const uint8_t
 }
 
 // t <- t + c f for the 32 rows of one TMEM lane quadrant and one K block,
-// the warp taking one row at a time: lane i holds dimensions 2i and 2i+1 of
-// the block, so a row's codeword half (256 bytes of float32) is one load of
-// two whole lines, and its operand words are one conflict-free 128-byte
-// access per half.  (Row per lane, each load would touch 32 lines for 16
-// bytes of each.)  bidx and f are this lane's own row's chosen codeword and
-// factor, broadcast row by row; cbk points at the K block's first element of
-// codeword 0 of the stage codebook.  Same arithmetic as load_add_chunk and
-// store_chunk: hi + lo exact, one rounding in the multiply-add.
-__device__ __forceinline__ void update_rows_t(uint8_t *ahi, uint8_t *alo, int quad, const float2 *cbk, int bidx,
+// the warp taking two rows at a time: half-warp h holds row 2p + h, its lane
+// i (0..15) dimensions 4i .. 4i+3 of the block, so a row's codeword half
+// (256 bytes of float32) is one 16-byte load per lane over two whole lines,
+// and its operand words one conflict-free 128-byte access per half.  (Row
+// per lane, each load would touch 32 lines for 16 bytes of each.)  bidx and
+// f are this lane's own row's chosen codeword and factor, broadcast row by
+// row (f is passed as uniform, UF, when every row's is the same); cbk points
+// at the K block's first element of codeword 0 of the stage codebook.  Same
+// arithmetic as load_add_chunk and store_chunk: hi + lo exact, one rounding
+// in the multiply-add.  Software-pipelined over batches of 8 rows: the next
+// batch's codeword loads are in flight while one batch is updated.
+template <bool UF>
+__device__ __forceinline__ void update_rows_t(uint8_t *ahi, uint8_t *alo, int quad, const float *cbk, int bidx,
                                               float f)
 {
     const int lane = threadIdx.x & 31;
-    const uint32_t lofs = static_cast<uint32_t>(((lane >> 2) << 4) | ((lane & 3) << 2));
-    const float2 *cl = cbk + lane;
+    const int hs = lane >> 4, li = lane & 15;
+    const uint32_t cw = static_cast<uint32_t>(li >> 1), wo = static_cast<uint32_t>((li & 1) << 3);
+    const float4 *cl = reinterpret_cast<const float4 *>(cbk) + li;
     uint8_t *qhi = ahi + quad * 32 * 128, *qlo = alo + quad * 32 * 128;
-    // software-pipelined over batches of 8 rows: the next batch's codeword
-    // loads are in flight while this batch is updated
-    float2 cv[2][8];
-    float fm[2][8];
+    float4 cv[2][4];
+    float fm[2][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        fm[0][j] = __shfl_sync(0xFFFFFFFFu, f, j);
-        cv[0][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, j) * 64);
+    for (int j = 0; j < 4; ++j) {
+        const int m = 2 * j + hs;
+        fm[0][j] = UF ? f : __shfl_sync(0xFFFFFFFFu, f, m);
+        cv[0][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, m) * 32);
     }
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
         const int cur = b & 1, nxt = cur ^ 1;
         if (b < 3) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int m = 8 * (b + 1) + j;
-                fm[nxt][j] = __shfl_sync(0xFFFFFFFFu, f, m);
-                cv[nxt][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, m) * 64);
+            for (int j = 0; j < 4; ++j) {
+                const int m = 8 * (b + 1) + 2 * j + hs;
+                fm[nxt][j] = UF ? f : __shfl_sync(0xFFFFFFFFu, f, m);
+                cv[nxt][j] = __ldg(cl + __shfl_sync(0xFFFFFFFFu, bidx, m) * 32);
             }
         }
-        uint32_t hv[8], lv[8];
+        uint2 hv[4], lv[4];
+        uint32_t off[4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const uint32_t off = (8 * b + j) * 128 + (lofs ^ (j << 4));     // swz: row & 7 == j
-            hv[j] = *reinterpret_cast<const uint32_t *>(qhi + off);
-            lv[j] = *reinterpret_cast<const uint32_t *>(qlo + off);
+        for (int j = 0; j < 4; ++j) {
+            const int r7 = 2 * j + hs;                                    // row & 7
+            off[j] = static_cast<uint32_t>((8 * b + r7) * 128) + ((cw ^ static_cast<uint32_t>(r7)) << 4) + wo;   // swz
+            hv[j] = *reinterpret_cast<const uint2 *>(qhi + off[j]);
+            lv[j] = *reinterpret_cast<const uint2 *>(qlo + off[j]);
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            float v0, v1;
-            join_half2(hv[j], lv[j], v0, v1);
+        for (int j = 0; j < 4; ++j) {
+            float v0, v1, v2, v3;
+            join_half2(hv[j].x, lv[j].x, v0, v1);
+            join_half2(hv[j].y, lv[j].y, v2, v3);
             v0 = fmaf(cv[cur][j].x, fm[cur][j], v0);
             v1 = fmaf(cv[cur][j].y, fm[cur][j], v1);
-            uint32_t h, l;
-            split_half2(v0, v1, h, l);
-            const uint32_t off = (8 * b + j) * 128 + (lofs ^ (j << 4));
-            *reinterpret_cast<uint32_t *>(qhi + off) = h;
-            *reinterpret_cast<uint32_t *>(qlo + off) = l;
+            v2 = fmaf(cv[cur][j].z, fm[cur][j], v2);
+            v3 = fmaf(cv[cur][j].w, fm[cur][j], v3);
+            uint2 h, l;
+            split_half2(v0, v1, h.x, l.x);
+            split_half2(v2, v3, h.y, l.y);
+            *reinterpret_cast<uint2 *>(qhi + off[j]) = h;
+            *reinterpret_cast<uint2 *>(qlo + off[j]) = l;
         }
     }
 }
@@ -1052,7 +1061,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     const float *cbs = a.cb32 + static_cast<int64_t>(cgroup(g) * S + s) * kCodes * D;
                     const float4 *gc = reinterpret_cast<const float4 *>(cbs + bidx * D) + 16;
                     if (e_next == e) {
-                        update_rows_t(ahi, alo, quad, reinterpret_cast<const float2 *>(cbs + 64), bidx, f);
+                        if (__all_sync(0xFFFFFFFFu, er == 0))
+                            update_rows_t<true>(ahi, alo, quad, cbs + 64, bidx, f);
+                        else
+                            update_rows_t<false>(ahi, alo, quad, cbs + 64, bidx, f);
                     } else {
                         float mx = 0.0f;
 #pragma unroll 4
@@ -1226,7 +1238,10 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     const float *cbs = a.cb32 + static_cast<int64_t>(cgroup(g) * S + s) * kCodes * D;
                     const float4 *gc = reinterpret_cast<const float4 *>(cbs + bidx * D);
                     if (e_next == e) {
-                        update_rows_t(ahi, alo, quad, reinterpret_cast<const float2 *>(cbs), bidx, f);
+                        if (__all_sync(0xFFFFFFFFu, er == 0))
+                            update_rows_t<true>(ahi, alo, quad, cbs, bidx, f);
+                        else
+                            update_rows_t<false>(ahi, alo, quad, cbs, bidx, f);
                     } else {
                         float mx = 0.0f;
 #pragma unroll 4
