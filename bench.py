@@ -85,13 +85,13 @@ def load_peaks():
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per RVQ launch of
 # the headline workload, from ncu captures of the current k_rvq128 on the same
 # cache cut to 4096 and to 8192 archived positions (the full cache is too large
-# for a multi-metric capture): key launch 1,339,402,752 and 2,522,289,408 B,
-# value launch 1,209,244,672 and 2,333,881,856 B.  Traffic is a fixed part (the
+# for a multi-metric capture): key launch 1,340,126,208 and 2,458,886,400 B,
+# value launch 1,209,800,960 and 2,317,281,024 B.  Traffic is a fixed part (the
 # codebooks) plus a part that grows with the positions, so the two lengths fix
 # a line, extrapolated to the headline length; the figure is the mean of the
 # key and value launches.  Set it to None when k_rvq128 changes until it is
 # captured again.
-RVQ_TRAFFIC_CAPTURES = ((4096, 8192), ((1339402752, 2522289408), (1209244672, 2333881856)))
+RVQ_TRAFFIC_CAPTURES = ((4096, 8192), ((1340126208, 2458886400), (1209800960, 2317281024)))
 
 
 def _rvq_traffic_full(positions=None, captures=RVQ_TRAFFIC_CAPTURES):
