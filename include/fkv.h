@@ -400,7 +400,11 @@ int fkv_cache_upload(fkv_ctx *ctx, const fkv_cache *src_host, const fkv_cache *d
  * n_rec records each, points as in fkv_decode_kv.  Out-of-range requests
  * write zeros and set FKV_ERANGE.  The requests are taken grouped by layer
  * (a counting sort of their indices on the device, so that one layer's
- * codebooks serve the requests in flight); the context keeps the index
+ * codebooks serve the requests in flight).  A batch of at least 512 requests
+ * per layer is staged: its records' symbols are decoded into a buffer first,
+ * then rebuilt from (codebook group, dimension slice) copies in shared memory
+ * as in fkv_decode_kv; smaller batches rebuild each record from codeword rows
+ * in L2.  Both give the same values.  The context keeps the index (and symbol)
  * buffer, allocating it on first use and whenever n_req outgrows it (after a
  * synchronisation of `stream`). */
 int fkv_read_kv(fkv_ctx *ctx, const double *pts_dev, int64_t n_streams, int64_t n_rec,

@@ -129,17 +129,80 @@ __host__ __device__ constexpr int gather_dp(int S, int KC)
     return KC == 256 ? (S <= 2 ? 64 : (S <= 4 ? 32 : 16)) : (S <= 1 ? 32 : 16);
 }
 
+// The stage sum of one vector's eight dimensions (granules ga, gb of its
+// slice row; q4 granules per row) from the codebook slice in shared memory:
+// float32, stage order.  ids holds the S indices, the first in the low bits.
+template <int S, int KC>
+__device__ __forceinline__ void sum_stages8(const float4 *row0, uint64_t ids, int ga, int gb, float4 &x, float4 &y)
+{
+    constexpr int kBits = KC == 256 ? 8 : 16;
+    constexpr uint64_t kMask = (1ull << kBits) - 1;
+    constexpr int q4 = gather_dp(S, KC) / 4;
+    x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    y = x;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        const int row = s * KC + static_cast<int>((ids >> (kBits * s)) & kMask);
+        const float4 c = row0[row * q4 + ga];
+        const float4 e = row0[row * q4 + gb];
+        add2(x.x, x.y, c.x, c.y);
+        add2(x.z, x.w, c.z, c.w);
+        add2(y.x, y.y, e.x, e.y);
+        add2(y.z, y.w, e.z, e.w);
+    }
+}
+
+// The same for four dimensions of a 16-float slice row (granule dq; rows
+// permute their granules by an XOR of the row).
+template <int S, int KC>
+__device__ __forceinline__ float4 sum_stages4(const float4 *row0, uint64_t ids, int dq)
+{
+    constexpr int kBits = KC == 256 ? 8 : 16;
+    constexpr uint64_t kMask = (1ull << kBits) - 1;
+    constexpr int Dp = gather_dp(S, KC);
+    constexpr int q4 = Dp / 4;
+    constexpr bool xor_rows = Dp < 32;
+    float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        const int row = s * KC + static_cast<int>((ids >> (kBits * s)) & kMask);
+        const int xq = xor_rows ? (row >> 1) & 3 : 0;
+        const float4 c = row0[row * q4 + (dq ^ xq)];
+        add2(x.x, x.y, c.x, c.y);
+        add2(x.z, x.w, c.z, c.w);
+    }
+    return x;
+}
+
+// A (codebook group, dimension slice) of float32 codebooks (all S stages, KC
+// codewords each, Dp floats of every row) into shared memory: every 16-byte
+// copy in flight, one wait.  The block meets at both ends.
+template <int S, int KC>
+__device__ __forceinline__ void load_slice(float *scb, const float *src, int D)
+{
+    constexpr int Dp = gather_dp(S, KC);
+    constexpr int q4 = Dp / 4;
+    constexpr bool xor_rows = Dp < 32;
+    __syncthreads();
+    for (int i = threadIdx.x; i < S * KC * q4; i += blockDim.x) {
+        const int row = i / q4, q = i - row * q4;
+        const int pq = xor_rows ? q ^ ((row >> 1) & 3) : q;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(fkvd::smem_u32(scb + 4 * (row * q4 + pq))),
+                     "l"(src + static_cast<int64_t>(row) * D + 4 * q)
+                     : "memory");
+    }
+    asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+    __syncthreads();
+}
+
 template <int S, bool WIDE, int KC>
 __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
 {
     using Sym = typename std::conditional<KC == 256, uint8_t, uint16_t>::type;
     constexpr int kBits = 8 * sizeof(Sym);
-    constexpr uint64_t kMask = (1ull << kBits) - 1;
     extern __shared__ __align__(128) float scb[];   // [S][KC][Dp] floats
     constexpr int Dp = gather_dp(S, KC);
     const int D = a.D, parts = a.parts;
-    constexpr int q4 = Dp / 4;               // 16-byte granules per slice row
-    constexpr bool xor_rows = Dp < 32;       // 16-float rows: XOR-permuted granules
     constexpr int kDT = Dp >= 32 ? 8 : 4;    // dimensions a thread rebuilds
     constexpr int tpv = Dp / kDT;            // threads per vector
     constexpr int vpi = kThreads / tpv;      // vectors per pass
@@ -174,18 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
         const int l = g / a.n_heads, h = g % a.n_heads;
         const int d0 = part * Dp;
         if (gp != cur) {
-            // codebook slice -> shared memory: every 16-byte copy in flight, one wait
-            __syncthreads();
-            const float *src = a.cb32 + static_cast<int64_t>(cgi) * S * KC * D + d0;
-            for (int i = threadIdx.x; i < S * KC * q4; i += kThreads) {
-                const int row = i / q4, q = i - row * q4;
-                const int pq = xor_rows ? q ^ ((row >> 1) & 3) : q;
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(fkvd::smem_u32(scb + 4 * (row * q4 + pq))),
-                             "l"(src + static_cast<int64_t>(row) * D + 4 * q)
-                             : "memory");
-            }
-            asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
-            __syncthreads();
+            load_slice<S, KC>(scb, a.cb32 + static_cast<int64_t>(cgi) * S * KC * D + d0, D);
             cur = gp;
         }
         const int64_t v = v0 + threadIdx.x / tpv;
@@ -228,30 +280,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_gather(const GatherArgs a)
                 if (u >= n_it)
                     break;
                 if constexpr (kDT == 8) {
-                    float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f), y = x;
-                    const int ga = 2 * dq + ph, gb = 2 * dq + 1 - ph;
-#pragma unroll
-                    for (int s = 0; s < S; ++s) {
-                        const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
-                        const float4 c = row0[row * q4 + ga];
-                        const float4 e = row0[row * q4 + gb];
-                        add2(x.x, x.y, c.x, c.y);
-                        add2(x.z, x.w, c.z, c.w);
-                        add2(y.x, y.y, e.x, e.y);
-                        add2(y.z, y.w, e.z, e.w);
-                    }
+                    float4 x, y;
+                    sum_stages8<S, KC>(row0, ids[u], 2 * dq + ph, 2 * dq + 1 - ph, x, y);
                     store8(a.out, a.dtype, off[u], ph ? y : x, ph ? x : y);
                 } else {
-                    float4 x = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll
-                    for (int s = 0; s < S; ++s) {
-                        const int row = s * KC + static_cast<int>((ids[u] >> (kBits * s)) & kMask);
-                        const int xq = xor_rows ? (row >> 1) & 3 : 0;
-                        const float4 c = row0[row * q4 + (dq ^ xq)];
-                        add2(x.x, x.y, c.x, c.y);
-                        add2(x.z, x.w, c.z, c.w);
-                    }
-                    store4(a.out, a.dtype, off[u], x);
+                    store4(a.out, a.dtype, off[u], sum_stages4<S, KC>(row0, ids[u], dq));
                 }
             }
         }
@@ -302,6 +335,7 @@ struct ReadArgs {
     const fkv_decconst *dec;
     const longlong2 *T;
     unsigned *status;
+    void *scr;                     // staged reads: entry i's record symbols to scr + i R, no gather here
 };
 
 __host__ __device__ inline int read_tables_bytes(int N, int L)
@@ -369,6 +403,14 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
         if (bad)
             atomicOr(a.status, FKV_ST_CORRUPT);
         __syncwarp();
+        if (a.scr) {
+            // staged: the record's symbols for the codebook-slice gather
+            Sym *dst = static_cast<Sym *>(a.scr) + i * R;
+            for (int j = lane; j < R; j += 32)
+                dst[j] = my[j];
+            __syncwarp();
+            continue;
+        }
         const int l = static_cast<int>(st % a.n_layers);
 #pragma unroll 2
         for (int g = lane; g < items; g += 32) {
@@ -409,6 +451,132 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
             store8(a.out, a.dtype, q * out_vec + (static_cast<int64_t>(kv) * H + hh) * D + d0, x, y);
         }
         __syncwarp();                             // the next request reuses `my`
+    }
+}
+
+// Staged record reads, second step: the K (kv 0) or V (kv 1) head vectors of
+// every in-range request rebuilt like the whole-archive gather, from a
+// (codebook group, dimension slice) held in shared memory.  Entries are the
+// layer-ordered requests: entry i's symbols at scr + i R (the first step
+// decoded them), its request at order[i].x, and layer l's entries end at
+// ends[l].  Work items are (layer, head and slice, entry) in that order
+// (slice-major over the heads when the layer's codebook is pooled, so the
+// slice stays for all of them); each block takes an equal share and loads a
+// slice when its group or slice changes.  With thousands of requests per
+// layer each slice serves many vectors from shared memory instead of every
+// vector reading its codeword rows from L2.
+struct ReadGatherArgs {
+    const void *scr;
+    const int4 *order;
+    const int *ends;
+    const float *cb32;     // [G][S][KC][D]
+    void *out;             // [n_req][2][H][D]
+    int dtype;
+    int n_layers, n_heads, D, R, off, kv, pooled, parts;
+};
+
+template <int S, bool WIDE, int KC>
+__global__ void __launch_bounds__(kThreads, 1) k_read_gather(const ReadGatherArgs a)
+{
+    using Sym = typename std::conditional<KC == 256, uint8_t, uint16_t>::type;
+    constexpr int kBits = 8 * sizeof(Sym);
+    extern __shared__ __align__(128) float scb[];   // [S][KC][Dp] floats
+    constexpr int Dp = gather_dp(S, KC);
+    constexpr int kDT = Dp >= 32 ? 8 : 4;
+    constexpr int tpv = Dp / kDT;
+    constexpr int vpi = kThreads / tpv;
+    constexpr int kU = 4;
+    const int D = a.D, H = a.n_heads, parts = a.parts, R = a.R;
+    const int GHP = H * parts;
+    const int dq = threadIdx.x % tpv;
+    const int ph = kDT == 8 ? (threadIdx.x >> 2) & 1 : 0;
+    const int64_t out_vec = static_cast<int64_t>(2) * H * D;
+    const int64_t total = static_cast<int64_t>(GHP) * __ldg(&a.ends[a.n_layers - 1]);
+    int64_t lo = total * blockIdx.x / gridDim.x;
+    const int64_t hi = total * (blockIdx.x + 1) / gridDim.x;
+    int64_t cur = -1;
+    int l = 0;
+    int64_t start = 0, end = __ldg(&a.ends[0]);
+    const Sym *scr = static_cast<const Sym *>(a.scr);
+    const float4 *row0 = reinterpret_cast<const float4 *>(scb);
+    while (lo < hi) {
+        // layer l's items are [GHP start_l, GHP end_l); empty layers are passed over
+        while (lo >= static_cast<int64_t>(GHP) * end) {
+            ++l;
+            start = end;
+            end = __ldg(&a.ends[l]);
+        }
+        const int64_t n_l = end - start;
+        const int64_t r = lo - static_cast<int64_t>(GHP) * start;
+        const int seg = static_cast<int>(r / n_l);
+        const int64_t j0 = r - seg * n_l;
+        const int64_t j1 = min(n_l, j0 + (hi - lo));
+        lo += j1 - j0;
+        int h, part;
+        if (a.pooled) {
+            part = seg / H;
+            h = seg - part * H;
+        } else {
+            h = seg / parts;
+            part = seg - h * parts;
+        }
+        const int64_t cg = a.pooled ? l : static_cast<int64_t>(l) * H + h;
+        if (cg * parts + part != cur) {
+            load_slice<S, KC>(scb, a.cb32 + cg * S * KC * D + part * Dp, D);
+            cur = cg * parts + part;
+        }
+        const int64_t ooff = static_cast<int64_t>(a.kv * H + h) * D + part * Dp + dq * kDT;
+        for (int64_t j = j0 + threadIdx.x / tpv; j < j1; j += kU * vpi) {
+            using Ids = typename std::conditional<S * kBits <= 32, uint32_t, uint64_t>::type;
+            Ids ids[kU];
+            int q[kU];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                const int64_t e = start + j + u * vpi;
+                if (j + u * vpi < j1) {
+                    ids[u] = static_cast<Ids>(load_ids<S, WIDE>(scr + e * R + a.off + h * S));
+                    q[u] = __ldg(&a.order[e].x);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kU; ++u) {
+                if (j + u * vpi >= j1)
+                    break;
+                const int64_t o = q[u] * out_vec + ooff;
+                if constexpr (kDT == 8) {
+                    float4 x, y;
+                    sum_stages8<S, KC>(row0, ids[u], 2 * dq + ph, 2 * dq + 1 - ph, x, y);
+                    store8(a.out, a.dtype, o, ph ? y : x, ph ? x : y);
+                } else {
+                    store4(a.out, a.dtype, o, sum_stages4<S, KC>(row0, ids[u], dq));
+                }
+            }
+        }
+    }
+}
+
+template <int S, int KC>
+void *read_gather_kernel(bool wide)
+{
+    constexpr int bytes = S * (KC == 256 ? 1 : 2);
+    if ((bytes == 2 || bytes == 4 || bytes == 8) && wide)
+        return reinterpret_cast<void *>(k_read_gather<S, true, KC>);
+    return reinterpret_cast<void *>(k_read_gather<S, false, KC>);
+}
+
+void *read_gather_kernel_for(int S, bool wide, int KC)
+{
+    if (KC == 1024)
+        return S == 1 ? read_gather_kernel<1, 1024>(wide) : read_gather_kernel<2, 1024>(wide);
+    switch (S) {
+    case 1: return read_gather_kernel<1, 256>(wide);
+    case 2: return read_gather_kernel<2, 256>(wide);
+    case 3: return read_gather_kernel<3, 256>(wide);
+    case 4: return read_gather_kernel<4, 256>(wide);
+    case 5: return read_gather_kernel<5, 256>(wide);
+    case 6: return read_gather_kernel<6, 256>(wide);
+    case 7: return read_gather_kernel<7, 256>(wide);
+    default: return read_gather_kernel<8, 256>(wide);
     }
 }
 
@@ -483,13 +651,35 @@ __global__ void __launch_bounds__(256) k_order_scatter(const int64_t *__restrict
 
 }  // namespace
 
+// Staged reads (decode into a symbol buffer, then the codebook-slice gather)
+// pay for loading every slice of the codebooks, so they serve batches of at
+// least this many requests per layer; smaller batches read codeword rows from
+// L2 one request per warp.
+constexpr int64_t kStagedPerLayer = 512;
+
+static bool read_staged(const fkv_ctx *c, int64_t n_req)
+{
+    return n_req >= kStagedPerLayer * c->Ly;
+}
+
+// Ints before the staged reads' symbol buffer: the entries and the layer
+// counters, rounded up to 16 bytes.
+static int64_t read_scr_ints(const fkv_ctx *c, int64_t n_req)
+{
+    return (4 * n_req + c->Ly + 1 + 3) & ~int64_t(3);
+}
+
 int64_t read_order_ints(const fkv_ctx *c, int64_t n_req)
 {
     // 32-bit request, stream and record numbers in the entries; the
     // per-block counts and run starts in 48 KB of shared memory
     if (n_req <= 0 || n_req > 0x7FFFFFFF || 2 * (c->Ly + 1) > 12 * 1024)
         return 0;
-    return 4 * n_req + c->Ly + 1;
+    if (!read_staged(c, n_req))
+        return 4 * n_req + c->Ly + 1;
+    const int64_t R = static_cast<int64_t>(c->H) * (c->cb[0].stages + c->cb[1].stages);
+    const int64_t esz = c->KC == 256 ? 1 : 2;
+    return read_scr_ints(c, n_req) + (n_req * R * esz + 3) / 4;
 }
 
 cudaError_t launch_rvq_decode(const fkv_ctx *c, int kv, const void *sym, int layout, int64_t stream_stride,
@@ -590,6 +780,7 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     a.dec = c->d_dec;
     a.T = c->d_T;
     a.status = c->d_status;
+    a.scr = nullptr;
     if (n_req <= 0)
         return cudaSuccess;
     const int esz = c->KC == 256 ? 1 : 2;
@@ -621,6 +812,8 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
         if (e != cudaSuccess)
             return e;
         a.order = ent;
+        if (read_staged(c, n_req))
+            a.scr = order + read_scr_ints(c, n_req);
     }
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kReadWarps * 32, smem);
     if (e != cudaSuccess)
@@ -633,5 +826,43 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kReadWarps * 32), args, smem, st);
     if (e != cudaSuccess)
         return e;
+    if (!a.scr)
+        return cudaGetLastError();
+    // staged: K, then V, rebuilt from codebook slices in shared memory
+    for (int kv = 0; kv < 2; ++kv) {
+        ReadGatherArgs g;
+        g.scr = a.scr;
+        g.order = a.order;
+        g.ends = order + 4 * n_req;
+        g.cb32 = c->cb[kv].cb32;
+        g.out = out;
+        g.dtype = dtype;
+        g.n_layers = c->Ly;
+        g.n_heads = c->H;
+        g.D = c->D;
+        g.R = a.R;
+        g.off = kv ? c->H * a.SK : 0;
+        g.kv = kv;
+        g.pooled = a.pooled;
+        const int S = c->cb[kv].stages;
+        const int Dp = gather_dp(S, c->KC);
+        g.parts = c->D / Dp;
+        const size_t gsm = static_cast<size_t>(S) * c->KC * Dp * 4;
+        const bool wide = a.R % S == 0 && g.off % S == 0;
+        const void *gk = read_gather_kernel_for(S, wide, c->KC);
+        e = cudaFuncSetAttribute(gk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(gsm > 48 * 1024 ? gsm : 48 * 1024));
+        if (e != cudaSuccess)
+            return e;
+        int gper = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&gper, gk, kThreads, gsm);
+        if (e != cudaSuccess)
+            return e;
+        void *gargs[] = {&g};
+        e = cudaLaunchKernel(gk, dim3(static_cast<unsigned>(sms * (gper > 0 ? gper : 1))), dim3(kThreads), gargs, gsm,
+                             st);
+        if (e != cudaSuccess)
+            return e;
+    }
     return cudaGetLastError();
 }
