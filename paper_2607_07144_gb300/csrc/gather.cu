@@ -335,7 +335,7 @@ struct ReadArgs {
     const fkv_decconst *dec;
     const longlong2 *T;
     unsigned *status;
-    void *scr;                     // staged reads: entry i's record symbols to scr + i R, no gather here
+    void *scr;                     // staged reads: entry i's record symbols at scr + i R
 };
 
 __host__ __device__ inline int read_tables_bytes(int N, int L)
@@ -403,14 +403,6 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
         if (bad)
             atomicOr(a.status, FKV_ST_CORRUPT);
         __syncwarp();
-        if (a.scr) {
-            // staged: the record's symbols for the codebook-slice gather
-            Sym *dst = static_cast<Sym *>(a.scr) + i * R;
-            for (int j = lane; j < R; j += 32)
-                dst[j] = my[j];
-            __syncwarp();
-            continue;
-        }
         const int l = static_cast<int>(st % a.n_layers);
 #pragma unroll 2
         for (int g = lane; g < items; g += 32) {
@@ -451,6 +443,56 @@ __global__ void __launch_bounds__(kReadWarps * 32, 3) k_read_kv(const ReadArgs a
             store8(a.out, a.dtype, q * out_vec + (static_cast<int64_t>(kv) * H + hh) * D + d0, x, y);
         }
         __syncwarp();                             // the next request reuses `my`
+    }
+}
+
+// Staged record reads, first step: the symbols of every entry's record into
+// scr + i R, one thread per (entry, span covering the record) so that every
+// lane walks a span (a record of R symbols spans about R / L of them); the
+// decoder tables are loaded once per persistent block.  An out-of-range
+// entry (stream -1, the last run) writes its request's zeros and sets
+// FKV_ST_RANGE instead.
+template <typename Sym>
+__global__ void __launch_bounds__(256) k_read_syms(const ReadArgs a, int spr)
+{
+    extern __shared__ __align__(16) uint8_t dsm[];
+    const fkvdec::Tables t = fkvdec::load(a.dec, a.T, a.N, a.L, dsm);
+    __syncthreads();
+    const int R = a.R, L = a.L;
+    const int64_t n = a.n_rec * R;
+    const int64_t out_vec = static_cast<int64_t>(2) * a.n_heads * a.D;
+    Sym *scr = static_cast<Sym *>(a.scr);
+    const int64_t items = a.n_req * spr;
+    for (int64_t it = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; it < items;
+         it += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t i = it / spr;
+        const int k = static_cast<int>(it - i * spr);
+        const int4 e = a.order[i];
+        if (e.y < 0) {
+            // out of range: this thread's share of the request's zeros
+            for (int64_t j = 2 * k; j < out_vec; j += 2 * spr)
+                store2(a.out, a.dtype, e.x * out_vec + j, 0.0f, 0.0f);
+            if (k == 0)
+                atomicOr(a.status, FKV_ST_RANGE);
+            continue;
+        }
+        const int64_t sym0 = static_cast<int64_t>(e.z) * R;
+        const int64_t u = sym0 / L + k;
+        if (u > (sym0 + R - 1) / L)
+            continue;
+        const int m = static_cast<int>(min(static_cast<int64_t>(L), n - u * L));
+        const double2 p = a.pts[e.y * a.pt_stride + u];
+        long long X = fkvdec::to_q62(p.x), Y = fkvdec::to_q62(p.y);
+        const int64_t base = u * L - sym0;
+        Sym *dst = scr + i * R;
+        fkvdec::walk<true>(t, X, Y, m, [&](int j, int c) {
+            const int64_t pos = base + m - 1 - j;
+            if (pos >= 0 && pos < R)
+                dst[pos] = static_cast<Sym>(c);
+        });
+        const long long lim = __ldg(&a.dec->alim[m]);
+        if (X > lim || X < -lim || Y > lim || Y < -lim)
+            atomicOr(a.status, FKV_ST_CORRUPT);
     }
 }
 
@@ -823,12 +865,35 @@ cudaError_t launch_read_kv(const fkv_ctx *c, const double *pts, int64_t n_stream
     if (blocks > resident)
         blocks = resident;
     void *args[] = {&a};
-    e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kReadWarps * 32), args, smem, st);
-    if (e != cudaSuccess)
-        return e;
-    if (!a.scr)
+    if (!a.scr) {
+        e = cudaLaunchKernel(kern, dim3(static_cast<unsigned>(blocks)), dim3(kReadWarps * 32), args, smem, st);
+        if (e != cudaSuccess)
+            return e;
         return cudaGetLastError();
-    // staged: K, then V, rebuilt from codebook slices in shared memory
+    }
+    // staged: the records' symbols (a thread per entry and span covering its record) ...
+    {
+        const int tsm = read_tables_bytes(a.N, a.L);
+        const void *sk = esz == 1 ? reinterpret_cast<const void *>(k_read_syms<uint8_t>)
+                                  : reinterpret_cast<const void *>(k_read_syms<uint16_t>);
+        e = cudaFuncSetAttribute(sk, cudaFuncAttributeMaxDynamicSharedMemorySize, tsm);
+        if (e != cudaSuccess)
+            return e;
+        int sper = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&sper, sk, 256, tsm);
+        if (e != cudaSuccess)
+            return e;
+        int spr = (a.R + a.L - 1) / a.L + (a.R % a.L ? 1 : 0);
+        const int64_t items = n_req * spr;
+        int64_t sblocks = static_cast<int64_t>(sms) * (sper > 0 ? sper : 1);
+        if (sblocks > (items + 255) / 256)
+            sblocks = (items + 255) / 256;
+        void *sargs[] = {&a, &spr};
+        e = cudaLaunchKernel(sk, dim3(static_cast<unsigned>(sblocks)), dim3(256), sargs, tsm, st);
+        if (e != cudaSuccess)
+            return e;
+    }
+    // ... then K and V rebuilt from codebook slices in shared memory
     for (int kv = 0; kv < 2; ++kv) {
         ReadGatherArgs g;
         g.scr = a.scr;
