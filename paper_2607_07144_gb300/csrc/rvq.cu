@@ -901,7 +901,7 @@ static_assert(SMEM <= 232448, "shared memory");
 
 template <int ESZ>
 __global__ void __launch_bounds__(v3::kThreads, 1)
-k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_per_group, int n_pairs)
+k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int n_pairs)
 {
     using namespace v3;
     constexpr int D = 128;
@@ -945,31 +945,45 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
     const int S = a.S;
     const int64_t nvec = a.batch * a.n_pos;
     const int tiles = a.tiles_per_group;
+    const int n_groups = a.n_layers * a.n_heads;
     auto cgroup = [&](int g) { return a.pooled ? g / a.n_heads : g; };
+    // The tiles of all head groups in one sequence, paired in order: slot k of
+    // pair p takes tile 2p + k, so a pair may straddle two groups (and a
+    // group's last odd tile is no half-empty pair).  *lt = the tile within its
+    // group; the group is clamped for the tile past the last one (its rows are
+    // past the data), whose codebook reads then stay in range.
+    auto slot_group = [&](int p, int k, int *lt) -> int {
+        const int64_t tau = 2 * static_cast<int64_t>(p) + k;
+        const int g = static_cast<int>(tau / tiles);
+        *lt = static_cast<int>(tau - static_cast<int64_t>(g) * tiles);
+        return g < n_groups ? g : n_groups - 1;
+    };
 
     if (warp == 0) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
-            // pieces of a slot's stage: q = 0 hi of K block 0 (with the norm
-            // operand for slot 0), 1 its lo, 2 hi of K block 1, 3 its lo;
-            // piece n goes to ring slot n & 1
+            // pieces of a slot's stage: q = 0 hi of K block 0 (with the slot's
+            // norm operand), 1 its lo, 2 hi of K block 1, 3 its lo; piece n
+            // goes to ring slot n & 1; each slot's codebook group is its tile's
             int n = 0;
             int last[2] = {-1, -1};
             bool ok = true;
             for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
-                const int cg = cgroup(p / pairs_per_group);
+                int lt;
+                const int cgs[2] = {cgroup(slot_group(p, 0, &lt)), cgroup(slot_group(p, 1, &lt))};
                 for (int s = 0; s < S && ok; ++s) {
                     for (int kq = 0; kq < 8; ++kq, ++n) {
                         const int k = kq >> 2, q = kq & 3, r = n & 1;
+                        const int cg = cgs[k];
                         if (!wait_or_abort(bar(2 + r), ((n >> 1) & 1) ^ 1, a.status, abort_flag)) {
                             ok = false;
                             break;
                         }
                         const int row0 = (cg * S + s) * 2 * kCodes + (q & 1) * kCodes;
-                        const bool aug = q == 0 && k == 0;
+                        const bool aug = q == 0;
                         mbar_arrive_expect_tx(bar(r), B_TILE + (aug ? B_AUG : 0));
                         tma_load_2d(sbase + OFF_B + r * B_TILE, &tmap, (q >> 1) * 64, row0, bar(r));
-                        if (aug)   // free: the norm MMAs of the stage before precede the piece this ring slot held
+                        if (aug)   // free: the other slot's norm MMA precedes the piece this ring slot held
                             bulk_load(sbase + OFF_BAUG, a.cbaug + static_cast<int64_t>(cg * S + s) * kCodes * 16,
                                       B_AUG, bar(r));
                         last[r] = n;
@@ -1042,11 +1056,14 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
         uint32_t hp_[2] = {0, 0}, xp_[2] = {0, 0};
         bool ok = true;
         for (int p = blockIdx.x; p < n_pairs && ok; p += gridDim.x) {
-            const int g = p / pairs_per_group;
-            int e = __ldg(&a.escale_h[g * S]);
+            int lt;
+            const int gs[2] = {slot_group(p, 0, &lt), slot_group(p, 1, &lt)};
+            int es[2] = {__ldg(&a.escale_h[gs[0] * S]), __ldg(&a.escale_h[gs[1] * S])};
             for (int s = 0; s + 1 < S && ok; ++s) {
-                const int e_next = __ldg(&a.escale_h[g * S + s + 1]);
                 for (int k = 0; k < 2 && ok; ++k) {
+                    const int g = gs[k], e = es[k];
+                    const int e_next = __ldg(&a.escale_h[g * S + s + 1]);
+                    es[k] = e_next;
                     ok = wait_or_abort(bar(11 + 4 * k + quad), hp_[k], a.status, abort_flag);
                     ok = __all_sync(0xFFFFFFFFu, ok);
                     if (!ok)
@@ -1104,7 +1121,6 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
                     fence_proxy_async_smem();
                     mbar_arrive(bar(9 + k));
                 }
-                e = e_next;
             }
         }
     } else {
@@ -1116,11 +1132,12 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
         uint8_t *ahi = base + OFF_A + k * A_SLOT;
         uint8_t *alo = ahi + A_HALF;
         uint8_t *aaug = base + OFF_AAUG + k * A_AUG;
+        const int64_t all_tiles = static_cast<int64_t>(n_groups) * tiles;
         auto row_src = [&](int p, bool *in) -> const uint4 * {
-            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
-            const int tile = 2 * q + k;
+            int tile;
+            const int g = slot_group(p, k, &tile);
             const int64_t v = static_cast<int64_t>(tile) * kRows + row;
-            *in = tile < tiles && v < nvec;
+            *in = 2 * static_cast<int64_t>(p) + k < all_tiles && v < nvec;
             if (!*in)
                 return nullptr;
             const int l = g / a.n_heads, h = g - l * a.n_heads;
@@ -1133,11 +1150,11 @@ k_rvq128(const __grid_constant__ CUtensorMap tmap, const RvqArgs a, int pairs_pe
         uint32_t fph = 0, xph = 0;
         int pc = 0;
         for (int p = blockIdx.x; p < n_pairs; p += gridDim.x) {
-            const int g = p / pairs_per_group, q = p - g * pairs_per_group;
+            int tile;
+            const int g = slot_group(p, k, &tile);
             const int l = g / a.n_heads, h = g - l * a.n_heads;
-            const int tile = 2 * q + k;
             const int64_t v = static_cast<int64_t>(tile) * kRows + row;
-            const bool valid = tile < tiles && v < nvec;
+            const bool valid = 2 * static_cast<int64_t>(p) + k < all_tiles && v < nvec;
             bool in;
             const uint4 *src = row_src(p, &in);
             // the row's operand t = x 2^-(e + er), er >= 0 keeping |t| below 2^12
@@ -1433,9 +1450,9 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
         return x->dtype == FKV_F32 ? launch_rvq64<4, 1>(cb.tmap, a, pp, np, grid, st)
                                    : launch_rvq64<2, 1>(cb.tmap, a, pp, np, grid, st);
     } else {
-        // 128-dimensional heads: 256 codewords per stage
-        const int64_t ppg = (tiles + 1) / 2;
-        const int64_t n_pairs = ppg * c->Ly * c->H;
+        // 128-dimensional heads: 256 codewords per stage, the tiles of all
+        // head groups paired in order
+        const int64_t n_pairs = (tiles * c->Ly * c->H + 1) / 2;
         if (n_pairs > 0x7FFFFFFF)
             return cudaErrorInvalidConfiguration;
         int sms = 0;
@@ -1443,17 +1460,17 @@ cudaError_t launch_rvq_encode(const fkv_ctx *c, int kv, const fkv_cache *x, int6
         if (e != cudaSuccess)
             return e;
         const unsigned grid = static_cast<unsigned>(n_pairs < sms ? n_pairs : sms);
-        const int pp = static_cast<int>(ppg), np = static_cast<int>(n_pairs);
+        const int np = static_cast<int>(n_pairs);
         if (x->dtype == FKV_F32) {
             e = cudaFuncSetAttribute(k_rvq128<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, v3::SMEM);
             if (e != cudaSuccess)
                 return e;
-            k_rvq128<4><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, pp, np);
+            k_rvq128<4><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, np);
         } else {
             e = cudaFuncSetAttribute(k_rvq128<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, v3::SMEM);
             if (e != cudaSuccess)
                 return e;
-            k_rvq128<2><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, pp, np);
+            k_rvq128<2><<<grid, v3::kThreads, v3::SMEM, st>>>(cb.tmap, a, np);
         }
     }
     return cudaGetLastError();
